@@ -1,0 +1,416 @@
+#!/usr/bin/env python
+"""Benchmark: candidate placements simulated per second on one GB300.
+
+Default workload: 8 prefill requests x 32 layers (N=3088 ops) on 8 simulated
+accelerators, K=4096 random placements (the benchmark's second config, the
+one its metric is quoted on).  One step = sim_batch over all K candidates +
+select_best, inputs resident in HBM, L2 flushed (256 MiB write) between
+steps; every step is timed with CUDA events on the launching stream.
+
+Also reported: the end-to-end rate through the public API with host buffers
+(H2D of the placements from pinned memory and D2H of the selection inside
+the timed region), the dominant kernel's roofline, the CPU oracle timed on
+this host's cores, and the SM clocks sampled during the timed region.
+
+``--impl reference`` times the CPU oracle (the reference arm of this repo:
+there is no upstream implementation) on the same workload and metric.
+``--config 1..5`` selects another workload (supplementary lines).
+Under torchrun every rank simulates its own K candidates (weak scaling,
+no data-path collective); rank 0 prints the line with the max time.
+"""
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "candidate placements simulated/sec (and op-events/sec) vs HBM/issue roofline"
+UNIT = "candidates/s"
+PROFILE = os.path.join(ROOT, "profiles", "sim_full_kernel_prefill_N3088_K4096.txt")
+KERNEL_SOURCES = [os.path.join(ROOT, "paper_2608_15762_gb300", "csrc", f)
+                  for f in ("gmgsim_kernels.cu", "gmg_layout.h")]
+
+
+def kernel_hash() -> str:
+    h = hashlib.sha256()
+    for f in KERNEL_SOURCES:
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
+
+
+def read_profile():
+    """Instruction and DRAM counts per launch of the dominant kernel from the
+    committed ncu summary, if it was taken on the current kernel source."""
+    if not os.path.exists(PROFILE):
+        return None
+    vals = {}
+    with open(PROFILE) as f:
+        for line in f:
+            if ":" in line:
+                k, v = line.split(":", 1)
+                vals[k.strip()] = v.strip()
+    if vals.get("kernel_source_sha256") != kernel_hash():
+        return None
+    try:
+        return {"inst": float(vals["inst_executed_per_launch"]),
+                "dram": float(vals["dram_bytes_per_launch"])}
+    except (KeyError, ValueError):
+        return None
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "sm_max_mhz": d.get("sm_max_mhz", 2070.0), "src": "measured"}
+    return {"hbm_gbs": 6800.0, "sm_max_mhz": 2070.0, "src": "fallback"}
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms."""
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), "--query-gpu=" + self.Q, "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[5:9]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None,
+                "sm_max_mhz": max(mx) if mx else None, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---------------------------------------------------------------------------
+# Workload preparation
+# ---------------------------------------------------------------------------
+
+class Prepared:
+    pass
+
+
+def prepare(config: int, rank: int, device):
+    import numpy as np
+    import torch
+    from paper_2608_15762_gb300 import gmgsim as G
+    from paper_2608_15762_gb300 import workloads as W
+    wl = W.make_workload(config)
+    p = Prepared()
+    p.wl = wl
+    p.g = G.gmg_create(wl.desc, device=device)
+    p.n_full = wl.n_full
+    p.n_inc = 0 if wl.moves is None else wl.moves.n_cand
+    p.K = p.n_full + p.n_inc
+    p.host_place = None
+    if p.n_full:
+        ks = range(rank * p.n_full, (rank + 1) * p.n_full)
+        rows = wl.full_rows(ks)
+        p.host_place = torch.from_numpy(rows).pin_memory()
+        p.place = p.host_place.to(device)
+    if p.n_inc:
+        p.host_base = torch.from_numpy(np.ascontiguousarray(wl.base_place)).pin_memory()
+        p.base_place = p.host_base.to(device)
+        p.host_moves = [torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
+                        for a in (wl.moves.off, wl.moves.op, wl.moves.dev)]
+        p.moves = [t.to(device) for t in p.host_moves]
+    p.out = G.SimOut.empty(p.K, wl.desc.n_dev, wl.desc.n_req, device)
+    p.scratch = G.Scratch(device)
+    p.best = torch.empty(2, dtype=torch.int64, device=device)
+    return p
+
+
+def _views(out, a, b):
+    from paper_2608_15762_gb300 import gmgsim as G
+    return G.SimOut(**{k: (None if v is None else v[a:b]) for k, v in out.__dict__.items()})
+
+
+def run_step(p, kernel_events=None):
+    """One pass of the hot path over the batch; returns kernel launches."""
+    from paper_2608_15762_gb300 import gmgsim as G
+    launches = 0
+    if p.n_full:
+        if kernel_events:
+            kernel_events[0].record()
+        G.sim_batch(p.g, p.place, out=_views(p.out, 0, p.n_full), scratch=p.scratch)
+        if kernel_events:
+            kernel_events[1].record()
+        launches += 1
+    if p.n_inc:
+        b = G.base_create(p.g, p.base_place)
+        o = _views(p.out, p.n_full, p.K)
+        if kernel_events and not p.n_full:
+            kernel_events[0].record()
+        G.sim_incremental(p.g, b, *p.moves, out=o, scratch=p.scratch)
+        if kernel_events and not p.n_full:
+            kernel_events[1].record()
+        p._base = b  # keep alive until the stream has used it
+        launches += 2
+    G.select_best(p.out, p.K, best=p.best)
+    launches += 2
+    return launches
+
+
+def run_e2e_step(p):
+    """Public API with host buffers: H2D of the inputs, the path, D2H of the
+    selection."""
+    if p.n_full:
+        p.place.copy_(p.host_place, non_blocking=True)
+    if p.n_inc:
+        p.base_place.copy_(p.host_base, non_blocking=True)
+        for d, h in zip(p.moves, p.host_moves):
+            d.copy_(h, non_blocking=True)
+    run_step(p)
+    return p.best.cpu()
+
+
+def h2d_bytes(p):
+    b = 0
+    if p.n_full:
+        b += p.host_place.numel()
+    if p.n_inc:
+        b += p.host_base.numel() + sum(t.numel() * t.element_size() for t in p.host_moves)
+    return b
+
+
+def cpu_baseline(wl, budget_s=20.0):
+    """The CPU oracle as it stands on this host's cores, on a bounded sample of
+    the same workload (whole batches until about budget_s of CPU time)."""
+    from oracle import oracle as O
+    nt = O.hw_threads()
+    if wl.n_full:
+        k = min(wl.n_full, 4096)
+        rows = wl.full_rows(range(k))
+        t0 = time.perf_counter()
+        O.simulate_batch(wl.desc, rows, nthreads=nt)
+        dt = time.perf_counter() - t0
+        sample = "%d of %d full placements" % (k, wl.n_full)
+    else:
+        from paper_2608_15762_gb300.workloads import Moves
+        k = min(wl.moves.n_cand, 2048)
+        mv = Moves(wl.moves.off[:k + 1].copy(), wl.moves.op[:wl.moves.off[k]], wl.moves.dev[:wl.moves.off[k]])
+        t0 = time.perf_counter()
+        O.incremental_batch(wl.desc, wl.base_place, mv, nthreads=nt)
+        dt = time.perf_counter() - t0
+        sample = "%d of %d incremental candidates" % (k, wl.moves.n_cand)
+    return {"value": k / dt, "unit": UNIT, "cores": nt, "kind": "oracle", "sample": sample,
+            "seconds": round(dt, 3), "op_events_per_s": k * wl.desc.n_ops / dt if wl.n_full else None}
+
+
+def reference_arm(args):
+    """--impl reference: time the CPU oracle on the host cores."""
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    from oracle import oracle as O
+    from paper_2608_15762_gb300 import workloads as W
+    wl = W.make_workload(args.config)
+    nt = O.hw_threads()
+    k = min(wl.n_full or wl.moves.n_cand, 4096 if wl.desc.n_ops < 10000 else 64)
+    if wl.n_full:
+        rows = wl.full_rows(range(k))
+
+        def step():
+            O.simulate_batch(wl.desc, rows, nthreads=nt)
+    else:
+        mv = W.Moves(wl.moves.off[:k + 1].copy(), wl.moves.op[:wl.moves.off[k]],
+                     wl.moves.dev[:wl.moves.off[k]])
+
+        def step():
+            O.incremental_batch(wl.desc, wl.base_place, mv, nthreads=nt)
+    for _ in range(args.warmup):
+        step()
+    times = []
+    for _ in range(args.steps):
+        t0 = time.perf_counter()
+        step()
+        times.append(time.perf_counter() - t0)
+    ms = 1000 * statistics.mean(times)
+    v = k / (ms / 1000)
+    line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": wl.name, "candidates_per_step": k, "n_ops": wl.desc.n_ops},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": nt, "kind": "oracle",
+                             "sample": "%d candidates per step" % k},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line))
+    return 0
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    if args.warmup < 3 and args.impl == "ours":
+        args.warmup = 3
+    if args.impl == "reference":
+        return reference_arm(args)
+
+    import torch
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+
+    from paper_2608_15762_gb300 import build as lib_build
+    lib_build.build()
+    p = prepare(args.config, rank, device)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+
+    def barrier():
+        torch.cuda.synchronize()
+        if world > 1:
+            torch.distributed.barrier()
+            torch.cuda.synchronize()
+
+    for _ in range(args.warmup):
+        run_step(p)
+    barrier()
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    step_ev, kern_ev = [], []
+    launches = 0
+    for _ in range(args.steps):
+        flush.fill_(1)
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        e[0].record()
+        launches += run_step(p, kernel_events=(e[2], e[3]))
+        e[1].record()
+        step_ev.append((e[0], e[1]))
+        kern_ev.append((e[2], e[3]))
+    barrier()
+    clocks = sampler.stop()
+    step_ms = [a.elapsed_time(b) for a, b in step_ev]
+    kern_ms = [a.elapsed_time(b) for a, b in kern_ev]
+    ms = statistics.mean(step_ms)
+    if world > 1:
+        t = torch.tensor([ms], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # end-to-end through the public API with host buffers
+    for _ in range(2):
+        run_e2e_step(p)
+    barrier()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        run_e2e_step(p)
+    barrier()
+    e2e_ms = 1000 * (time.perf_counter() - t0) / args.steps
+    if world > 1:
+        t = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        e2e_ms = float(t.item())
+
+    wl = p.wl
+    K, N, D = p.K, wl.desc.n_ops, wl.desc.n_dev
+    best = p.best.cpu().tolist()
+    value = world * K / (ms / 1000)
+    kms = statistics.mean(kern_ms)
+    # Roofline of the dominant kernel (the candidate simulation).
+    pk = peaks()
+    out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
+    alg_bytes = (p.n_full * W_ld(N) if p.n_full else 0) + K * out_bytes_per_cand
+    hbm_gbs = alg_bytes / (kms / 1000) / 1e9
+    props = torch.cuda.get_device_properties(device)
+    issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
+    prof = read_profile() if args.config == 2 else None
+    roof = {"bound": "alu", "unit": "Ginst/s", "peak": issue_peak,
+            "peak_src": "%d SMs x 4 issue slots x %.0f MHz (%s sm_max_mhz)" % (
+                props.multi_processor_count, pk["sm_max_mhz"], pk["src"]),
+            "achieved": None, "frac": None, "traffic": None,
+            "kernel": "sim_full_kernel" if p.n_full else "sim_inc_kernel",
+            "kernel_ms": kms}
+    if prof:
+        ach = prof["inst"] / (kms / 1000) / 1e9
+        roof.update(achieved=ach, frac=ach / issue_peak, traffic=prof["dram"],
+                    inst_per_launch=prof["inst"], inst_src=os.path.relpath(PROFILE, ROOT))
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "config": {"workload": wl.name, "candidates": K, "n_ops": N, "n_dev": D,
+                   "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
+                   "parallelism": "dp%d over candidates" % world},
+        "op_events_per_s": world * (p.n_full * N) / (ms / 1000) if p.n_full else None,
+        "roofline": roof,
+        "hbm": {"achieved": hbm_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": hbm_gbs / pk["hbm_gbs"], "algorithmic_bytes_per_launch": alg_bytes,
+                "note": "placement bytes read + per-candidate outputs written; the kernel is issue/latency-bound"},
+        "e2e": {"value": world * K / (e2e_ms / 1000), "unit": UNIT, "ms_per_step": e2e_ms,
+                "h2d_bytes_per_step": h2d_bytes(p), "d2h_bytes_per_step": 16},
+        "gpu_launches": launches,
+        "clocks": clocks,
+        "best": best,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl)
+    if rank == 0:
+        print(json.dumps(line))
+    if world > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def W_ld(n):
+    return max(16, (n + 15) // 16 * 16)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

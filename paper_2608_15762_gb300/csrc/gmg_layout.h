@@ -1,0 +1,158 @@
+// Device layout of a GMG and launch parameters shared by the library's host
+// code (gmgsim_host.cu) and its kernels (gmgsim_kernels.cu).  Private to the
+// library: not part of the C ABI.
+#pragma once
+
+#include <stdint.h>
+
+#include "../../include/gmgsim.h"
+
+namespace gsim {
+
+// One 64-byte record per operator: everything the event loop reads when it
+// pops, releases or readies the op, in one L1 sector pair.
+struct alignas(64) OpRec {
+  int64_t dur;       // duration (us), >= 1
+  int64_t bytes;     // output size (B)
+  int64_t release;   // arrival of the op itself (us)
+  int64_t xq;        // ceil(bytes / bw) when every link has the same bandwidth
+  uint32_t succ_off; // successors: succ[succ_off .. +nsucc), ascending
+  uint32_t nsucc;
+  uint32_t pred_off; // predecessors: pred[pred_off .. +npred); bit 31 set if this op
+  uint32_t npred;    //   is a listed consumer of that predecessor's output
+  uint32_t cons_off; // listed consumers of this op's output: cons[cons_off .. +ncons)
+  uint32_t ncons;    //   (equals the successor list when kAllCons is set)
+  int32_t req;       // request id or -1
+  uint32_t flags;    // kScored | kReqSink | kAllCons
+};
+static_assert(sizeof(OpRec) == 64, "OpRec must be 64 bytes");
+
+constexpr uint32_t kScored = 1u;   // counts in the score
+constexpr uint32_t kReqSink = 2u;  // no successor in its own request: may end the request
+constexpr uint32_t kAllCons = 4u;  // consumers = successors
+constexpr uint32_t kHoldBit = 0x80000000u;
+constexpr uint32_t kIdMask = 0x7fffffffu;
+
+// Exact ceil(n / bw) by multiply-shift (Granlund & Montgomery 1994,
+// "Division by invariant integers using multiplication", Thm 4.2): with
+// l = ceil(log2 bw), s = 53 + l and m = ceil(2^s / bw), floor(n / bw) =
+// floor(m * n / 2^s) for every 0 <= n < 2^53.
+struct LinkRec {
+  uint64_t magic;
+  int64_t bw;
+  int64_t lat;
+  int32_t shift;
+  int32_t pad;
+};
+static_assert(sizeof(LinkRec) == 32, "LinkRec must be 32 bytes");
+
+#if defined(__CUDACC__)
+#define GMG_HD __host__ __device__ __forceinline__
+#else
+#define GMG_HD inline
+#endif
+
+GMG_HD uint64_t mulhi_u64(uint64_t a, uint64_t b) {
+#if defined(__CUDA_ARCH__)
+  return __umul64hi(a, b);
+#else
+  return (uint64_t)(((unsigned __int128)a * (unsigned __int128)b) >> 64);
+#endif
+}
+
+GMG_HD int64_t ceil_div_link(int64_t n, const LinkRec& L) {
+  const uint64_t un = (uint64_t)n;
+  const uint64_t hi = mulhi_u64(un, L.magic);
+  const uint64_t lo = un * L.magic;
+  const int s = L.shift;
+  const uint64_t q = s >= 64 ? (hi >> (s - 64)) : ((hi << (64 - s)) | (lo >> s));
+  return (int64_t)q + ((int64_t)q * L.bw != n ? 1 : 0);
+}
+
+// Pointers into the caller's device workspace.
+struct DevGmg {
+  const OpRec* ops;
+  const uint32_t* succ;
+  const uint32_t* pred;
+  const uint32_t* cons;
+  const uint64_t* root_keys;  // READY keys of ops without predecessors, ascending
+  const int64_t* cap;
+  const int64_t* base;
+  const int64_t* avail0;
+  const int64_t* deadline;
+  const LinkRec* links;       // D*D, NULL when links are uniform
+  int64_t lat0;               // uniform latency
+  int64_t max_iter;           // event-loop iteration cap per candidate
+  int32_t n, D, R, nroots;
+  int32_t ib;                 // op-id bits of a packed key
+  int32_t uniform;
+};
+
+// Packed event key: time << (ib + 2) | class << ib | op.  Classes at equal
+// times: READY (an op's last input arrived) < FREE < ALLOC.
+constexpr uint32_t kReady = 0, kFree = 1, kAlloc = 2;
+
+// Candidate simulation modes.
+enum Mode : int { kFull = 0, kInc = 1, kBase = 2 };
+
+// Output pointers (device) as in sim_out_t.
+struct DevOut {
+  int64_t* makespan;
+  int64_t* score;
+  int32_t* status;
+  int32_t* viol_flag;
+  int32_t* viol_op;
+  int32_t* viol_dev;
+  int64_t* viol_time;
+  int64_t* peak;
+  int32_t* sla_miss;
+  int64_t* events;
+  int64_t* req_done;
+  int64_t* trace_start;
+  int64_t* trace_finish;
+};
+
+// Base snapshot (incremental resume points) in the base workspace.
+struct DevBase {
+  uint8_t* row;          // [ld] base placement
+  int64_t* rb;           // [N] base ready time
+  int64_t* fb;           // [N] base finish time
+  int32_t* status;       // [1]
+  // base results (outputs of the base placement)
+  int64_t* res_scalars;  // [8]: makespan, score, viol_flag, viol_op, viol_dev, viol_time, sla_miss, n_ck
+  int64_t* res_peak;     // [D]
+  int64_t* res_creq;     // [R]
+  // checkpoints c = 0 .. nck-1
+  int64_t* ck_time;      // [nck]  T_c (INT64_MAX = not recorded)
+  int64_t* ck_scalars;   // [nck*8]: qsize, rootptr, score, makespan, vflag, vt, vop, vdev
+  int64_t* ck_dev;       // [nck*3*D]: free, live, peak
+  int64_t* ck_creq;      // [nck*R]
+  uint64_t* ck_qkey;     // [nck*ckq]
+  uint32_t* ck_qpay;     // [nck*ckq]
+  int32_t nck;
+  int32_t ckq;           // entries per checkpoint queue
+  int32_t ld;
+  int32_t stride_pops;   // READY pops between checkpoints
+};
+
+struct SimParams {
+  DevGmg g;
+  DevOut out;
+  DevBase base;
+  const uint8_t* place;  // kFull: [K][ld]; kBase: base row
+  int64_t ld;
+  int32_t K;
+  int32_t qs;            // queue entries in shared memory per warp (32m+1)
+  int32_t qcap;          // total queue entries per warp
+  int32_t n_trace;
+  const int32_t* trace_k;
+  const int32_t* move_off;
+  const int32_t* move_op;
+  const uint8_t* move_dev;
+  uint8_t* scratch;
+  int64_t slot_bytes;    // scratch bytes per warp slot
+  // byte offsets inside a slot
+  int64_t off_f, off_bits, off_creq, off_qk, off_qp, off_dev, off_row;
+};
+
+}  // namespace gsim

@@ -1,0 +1,712 @@
+// Host side of the C ABI (include/gmgsim.h): validation, the device layout
+// of a GMG, scratch sizing and kernel launches.  No device memory is ever
+// allocated here: every buffer is the caller's.
+
+#include <cuda_runtime.h>
+
+#include <algorithm>
+#include <cstring>
+#include <new>
+#include <vector>
+
+#include "gmg_layout.h"
+
+namespace gsim {
+// launchers (gmgsim_kernels.cu)
+size_t select_rank_bytes();
+const void* full_kernel_ptr(bool reg);
+const void* inc_kernel_ptr(bool reg);
+cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
+cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
+cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
+cudaError_t launch_select(const int32_t* status, const int32_t* viol, const int64_t* score,
+                          const int32_t* miss, int32_t K, int32_t mode, void* tmp, int nparts,
+                          int64_t* best, cudaStream_t st);
+}  // namespace gsim
+
+using namespace gsim;
+
+namespace {
+
+constexpr int64_t kI64Max = 0x7fffffffffffffffll;
+constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
+constexpr int kDefaultWarpsPerBlock = 4;
+constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root and two child levels
+constexpr int64_t kDefaultQueueCap = 1 << 16;
+constexpr int kCheckpoints = 256;
+constexpr int kCheckpointQueue = 4096;
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct Layout {
+  size_t off_ops, off_succ, off_pred, off_cons, off_roots, off_cap, off_base, off_avail, off_dl,
+      off_links, total;
+};
+
+// Everything gmg_create derives from a description.
+struct Built {
+  int n = 0, E = 0, D = 0, R = 0, Ec = 0, nroots = 0, ib = 1;
+  bool uniform = true;
+  int64_t bw0 = 1, lat0 = 0, time_bound = 0, max_iter = 0, queue_bound = 0;
+  std::vector<OpRec> ops;
+  std::vector<uint32_t> succ, pred, cons;
+  std::vector<uint64_t> roots;
+  std::vector<int64_t> cap, base, avail0, deadline;
+  std::vector<LinkRec> links;
+  Layout L{};
+};
+
+LinkRec make_link(int64_t bw, int64_t lat) {
+  LinkRec r{};
+  int l = 0;
+  while ((int64_t(1) << l) < bw) ++l;  // l = ceil(log2 bw)
+  const int s = 53 + l;
+  const unsigned __int128 one = 1;
+  const unsigned __int128 m = ((one << s) + (unsigned __int128)(bw - 1)) / (unsigned __int128)bw;
+  r.magic = (uint64_t)m;
+  r.bw = bw;
+  r.lat = lat;
+  r.shift = s;
+  return r;
+}
+
+int64_t host_ceil(int64_t n, int64_t d) {
+  const int64_t q = n / d;
+  return q * d == n ? q : q + 1;
+}
+
+void plan(Built& b) {
+  Layout& L = b.L;
+  size_t o = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o;
+    o = align_up(o + std::max<size_t>(bytes, 1), 256);
+    return at;
+  };
+  L.off_ops = take(sizeof(OpRec) * (size_t)b.n);
+  L.off_succ = take(4 * (size_t)b.E);
+  L.off_pred = take(4 * (size_t)b.E);
+  L.off_cons = take(4 * (size_t)b.Ec);
+  L.off_roots = take(8 * (size_t)b.nroots);
+  L.off_cap = take(8 * (size_t)b.D);
+  L.off_base = take(8 * (size_t)b.D);
+  L.off_avail = take(8 * (size_t)b.D);
+  L.off_dl = take(8 * (size_t)b.R);
+  L.off_links = take(b.uniform ? 0 : sizeof(LinkRec) * (size_t)b.D * b.D);
+  L.total = o;
+}
+
+// Validate and derive.  Returns GMG_OK or an error code.
+int build(const gmg_desc_t* d, Built& b) {
+  if (!d) return GMG_EINVAL;
+  const int n = d->n_ops, D = d->n_dev, R = d->n_req;
+  if (n < 0 || d->n_edges < 0 || D < 1 || D > 256 || R < 0) return GMG_EINVAL;
+  if (n > (1 << kMaxOpsLog2)) return GMG_ERANGE;
+  if (!d->pred_off || (d->n_edges > 0 && !d->pred_idx)) return GMG_EINVAL;
+  if (n > 0 && (!d->dur_us || !d->out_bytes)) return GMG_EINVAL;
+  if (D > 1 && (!d->bw_B_per_us || !d->lat_us)) return GMG_EINVAL;
+  if (d->pred_off[0] != 0 || d->pred_off[n] != d->n_edges) return GMG_EINVAL;
+  for (int i = 0; i < n; ++i)
+    if (d->pred_off[i + 1] < d->pred_off[i]) return GMG_EINVAL;
+  b.n = n;
+  b.E = d->n_edges;
+  b.D = D;
+  b.R = R;
+  b.ib = 1;
+  while ((int64_t(1) << b.ib) < n) ++b.ib;
+  // predecessors (topological, no duplicates) and successor counts
+  std::vector<uint32_t> nsucc(n, 0);
+  b.pred.resize(b.E);
+  std::vector<int32_t> seen(n, -1);
+  for (int i = 0; i < n; ++i) {
+    for (int k = d->pred_off[i]; k < d->pred_off[i + 1]; ++k) {
+      const int p = d->pred_idx[k];
+      if (p < 0 || p >= n) return GMG_EINVAL;
+      if (p >= i) return GMG_ENOTTOPO;
+      if (seen[p] == i) return GMG_EINVAL;
+      seen[p] = i;
+      b.pred[k] = (uint32_t)p;
+      ++nsucc[p];
+    }
+  }
+  b.ops.assign(n, OpRec{});
+  uint32_t acc = 0;
+  for (int i = 0; i < n; ++i) {
+    b.ops[i].succ_off = acc;
+    acc += nsucc[i];
+  }
+  b.succ.resize(b.E);
+  std::vector<uint32_t> fill(n, 0);
+  for (int i = 0; i < n; ++i)
+    for (int k = d->pred_off[i]; k < d->pred_off[i + 1]; ++k) {
+      const int p = d->pred_idx[k];
+      b.succ[b.ops[p].succ_off + fill[p]++] = (uint32_t)i;  // ascending: i increases
+    }
+  // per-op scalars
+  for (int i = 0; i < n; ++i) {
+    OpRec& r = b.ops[i];
+    r.dur = d->dur_us[i];
+    r.bytes = d->out_bytes[i];
+    r.release = d->release_us ? d->release_us[i] : 0;
+    r.req = d->req_id ? d->req_id[i] : -1;
+    const uint8_t sc = d->scored ? d->scored[i] : 1;
+    if (r.dur < 1 || r.bytes < 0 || r.release < 0) return GMG_EINVAL;
+    if (r.req < -1 || r.req >= R) return GMG_EINVAL;
+    if (sc > 1) return GMG_EINVAL;
+    if (r.bytes >= (int64_t(1) << 53)) return GMG_ERANGE;
+    r.nsucc = nsucc[i];
+    r.pred_off = (uint32_t)d->pred_off[i];
+    r.npred = (uint32_t)(d->pred_off[i + 1] - d->pred_off[i]);
+    r.flags = sc ? kScored : 0u;
+  }
+  // consumer lists (subsets of the successors) and the hold bits on the
+  // consumers' predecessor entries
+  auto set_hold = [&](uint32_t c, uint32_t p) {
+    for (uint32_t k = b.ops[c].pred_off; k < b.ops[c].pred_off + b.ops[c].npred; ++k)
+      if ((b.pred[k] & kIdMask) == p) {
+        b.pred[k] |= kHoldBit;
+        return;
+      }
+  };
+  if (!d->cons_off) {
+    for (int i = 0; i < n; ++i) {
+      b.ops[i].flags |= kAllCons;
+      b.ops[i].cons_off = b.ops[i].succ_off;
+      b.ops[i].ncons = b.ops[i].nsucc;
+      for (uint32_t k = 0; k < b.ops[i].nsucc; ++k) set_hold(b.succ[b.ops[i].succ_off + k], i);
+    }
+  } else {
+    if (d->cons_off[0] != 0) return GMG_EINVAL;
+    for (int i = 0; i < n; ++i)
+      if (d->cons_off[i + 1] < d->cons_off[i]) return GMG_EINVAL;
+    if (d->cons_off[n] > 0 && !d->cons_idx) return GMG_EINVAL;
+    std::vector<int32_t> mark(n, -1);
+    for (int i = 0; i < n; ++i) {
+      OpRec& r = b.ops[i];
+      for (uint32_t k = 0; k < r.nsucc; ++k) mark[b.succ[r.succ_off + k]] = i;
+      const int a = d->cons_off[i], e = d->cons_off[i + 1];
+      for (int k = a; k < e; ++k) {
+        const int c = d->cons_idx[k];
+        if (c < 0 || c >= n || mark[c] != i) return GMG_EINVAL;  // not a successor, or repeated
+        mark[c] = -2 - i;
+      }
+      if ((uint32_t)(e - a) == r.nsucc) {
+        r.flags |= kAllCons;
+        r.cons_off = r.succ_off;
+        r.ncons = r.nsucc;
+        for (uint32_t k = 0; k < r.nsucc; ++k) set_hold(b.succ[r.succ_off + k], i);
+      } else {
+        r.cons_off = (uint32_t)b.cons.size();
+        r.ncons = (uint32_t)(e - a);
+        for (int k = a; k < e; ++k) {
+          b.cons.push_back((uint32_t)d->cons_idx[k]);
+          set_hold((uint32_t)d->cons_idx[k], i);
+        }
+      }
+    }
+  }
+  b.Ec = (int)b.cons.size();
+  // request sinks: no successor in the same request
+  for (int i = 0; i < n; ++i) {
+    OpRec& r = b.ops[i];
+    if (r.req < 0) continue;
+    bool sink = true;
+    for (uint32_t k = 0; k < r.nsucc && sink; ++k)
+      if (b.ops[b.succ[r.succ_off + k]].req == r.req) sink = false;
+    if (sink) r.flags |= kReqSink;
+  }
+  // accelerators
+  b.cap.resize(D);
+  b.base.resize(D);
+  b.avail0.resize(D);
+  for (int e = 0; e < D; ++e) {
+    b.cap[e] = d->cap_bytes ? d->cap_bytes[e] : kI64Max;
+    b.base[e] = d->base_bytes ? d->base_bytes[e] : 0;
+    b.avail0[e] = d->avail0_us ? d->avail0_us[e] : 0;
+    if (b.cap[e] < 0 || b.base[e] < 0 || b.base[e] > b.cap[e] || b.avail0[e] < 0) return GMG_EINVAL;
+  }
+  b.deadline.resize(R);
+  for (int r = 0; r < R; ++r) b.deadline[r] = d->deadline_us ? d->deadline_us[r] : kI64Max;
+  // links
+  int64_t min_bw = kI64Max, max_lat = 0;
+  b.uniform = true;
+  bool first = true;
+  for (int s = 0; s < D; ++s)
+    for (int e = 0; e < D; ++e) {
+      if (s == e) continue;
+      const int64_t bw = d->bw_B_per_us[(size_t)s * D + e], lat = d->lat_us[(size_t)s * D + e];
+      if (bw < 1 || lat < 0) return GMG_EINVAL;
+      if (bw >= (int64_t(1) << 62)) return GMG_ERANGE;
+      if (first) {
+        b.bw0 = bw;
+        b.lat0 = lat;
+        first = false;
+      } else if (bw != b.bw0 || lat != b.lat0) {
+        b.uniform = false;
+      }
+      min_bw = std::min(min_bw, bw);
+      max_lat = std::max(max_lat, lat);
+    }
+  if (D == 1) {
+    min_bw = 1;
+    b.bw0 = 1;
+    b.lat0 = 0;
+  }
+  if (!b.uniform) {
+    b.links.resize((size_t)D * D);
+    for (int s = 0; s < D; ++s)
+      for (int e = 0; e < D; ++e)
+        b.links[(size_t)s * D + e] =
+            s == e ? make_link(1, 0)
+                   : make_link(d->bw_B_per_us[(size_t)s * D + e], d->lat_us[(size_t)s * D + e]);
+  }
+  for (int i = 0; i < n; ++i) b.ops[i].xq = host_ceil(b.ops[i].bytes, b.bw0);
+  // Bounds: every time <= start + all durations + one transfer per edge and
+  // per op; it must fit the packed key (61 - ib bits); scores and byte totals
+  // must fit int64.
+  typedef __int128 i128;
+  i128 t = 0, mem = 0, iters = 16, qb = 16;
+  for (int e = 0; e < D; ++e) {
+    t = std::max<i128>(t, b.avail0[e]);
+    mem += b.base[e];
+  }
+  for (int i = 0; i < n; ++i) t = std::max<i128>(t, b.ops[i].release);
+  const i128 tlim = i128(1) << (61 - b.ib);
+  for (int i = 0; i < n; ++i) {
+    const OpRec& r = b.ops[i];
+    const i128 mx = i128(r.bytes / min_bw + 1) + max_lat;
+    const uint32_t copies = std::min<uint32_t>(r.nsucc, (uint32_t)(D - 1));
+    t += r.dur + mx * i128(r.nsucc + 1);
+    mem += i128(r.bytes) * i128(copies + 1);
+    iters += 3 + 2 * i128(copies);
+    qb += (r.npred ? 1 : 0) + 2 + 2 * i128(copies);
+    if (t >= tlim || mem >= (i128(1) << 62)) return GMG_ERANGE;
+  }
+  if (t * i128(std::max(n, 1)) >= (i128(1) << 62)) return GMG_ERANGE;
+  b.time_bound = (int64_t)t;
+  b.max_iter = (int64_t)iters;
+  b.queue_bound = (int64_t)qb;
+  // roots, by (release, id)
+  for (int i = 0; i < n; ++i)
+    if (b.ops[i].npred == 0)
+      b.roots.push_back(((uint64_t)b.ops[i].release << (b.ib + 2)) | (uint64_t)i);
+  std::sort(b.roots.begin(), b.roots.end());
+  b.nroots = (int)b.roots.size();
+  plan(b);
+  return GMG_OK;
+}
+
+int device_sms() {
+  int dev = 0, sms = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return -1;
+  if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return -1;
+  return sms;
+}
+
+}  // namespace
+
+struct gmg {
+  DevGmg dg;
+  gmg_info_t info;
+  int64_t queue_bound;
+};
+
+struct gmg_base {
+  DevBase db;
+  const gmg* g;
+  uint8_t* slot;
+  int qs, qcap;
+};
+
+namespace {
+
+struct Launch {
+  bool reg;
+  int wpb, qs, qcap, grid;
+  size_t smem;
+  int64_t slots;
+  SimParams P;  // offsets filled
+};
+
+int queue_cap(const gmg* g, const sim_opts_t* o) {
+  int64_t c = (o && o->queue_cap > 0) ? o->queue_cap : std::min<int64_t>(g->queue_bound, kDefaultQueueCap);
+  return (int)std::max<int64_t>(c, 1);
+}
+
+int shared_entries(int qcap) {
+  const int m = std::min(kSharedQueueEntries, qcap);
+  return ((m + 30) / 32) * 32 + 1;  // 32m + 1 >= m
+}
+
+// Slot layout and grid for K candidates of kind `inc`.
+int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& L) {
+  const DevGmg& G = g->dg;
+  L.reg = G.D <= 32;
+  L.wpb = (o && o->warps_per_block > 0) ? o->warps_per_block : kDefaultWarpsPerBlock;
+  if (L.wpb > 4) return GMG_EINVAL;
+  L.qcap = queue_cap(g, o);
+  L.qs = shared_entries(L.qcap);
+  L.smem = (size_t)L.wpb * L.qs * 12;
+  SimParams& P = L.P;
+  std::memset(&P, 0, sizeof(P));
+  size_t o2 = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = o2;
+    o2 = align_up(o2 + std::max<size_t>(bytes, 1), 256);
+    return (int64_t)at;
+  };
+  const int64_t spill = std::max<int64_t>(L.qcap - L.qs, 0);
+  P.off_f = take(8 * (size_t)G.n);
+  P.off_bits = take(4 * (size_t)((G.n + 31) / 32) + 16);
+  P.off_creq = take(8 * (size_t)G.R);
+  P.off_qk = take(8 * (size_t)spill);
+  P.off_qp = take(4 * (size_t)spill);
+  P.off_dev = take(L.reg ? 0 : 24 * (size_t)G.D);
+  P.off_row = take(inc ? (size_t)align_up(std::max(G.n, 1), 16) : 0);
+  P.slot_bytes = (int64_t)o2;
+  P.qs = L.qs;
+  P.qcap = L.qcap;
+  const int sms = device_sms();
+  if (sms <= 0) return GMG_ECUDA;
+  int bps = 0;
+  const void* fn = inc ? inc_kernel_ptr(L.reg) : full_kernel_ptr(L.reg);
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
+    return GMG_ECUDA;
+  bps = std::max(bps, 1);
+  const int64_t need = (std::max<int64_t>(K, 1) + L.wpb - 1) / L.wpb;
+  L.grid = (int)std::min<int64_t>(need, (int64_t)sms * bps);
+  L.slots = (int64_t)L.grid * L.wpb;
+  P.g = G;
+  return GMG_OK;
+}
+
+bool aligned(const void* p, size_t a) { return ((uintptr_t)p % a) == 0; }
+
+int check_out(const sim_out_t* o, const sim_opts_t* opts) {
+  if (!o || !o->makespan || !o->score || !o->status || !o->viol_flag || !o->viol_op ||
+      !o->viol_dev || !o->viol_time || !o->peak || !o->sla_miss || !o->events)
+    return GMG_EINVAL;
+  if (opts && opts->n_trace < 0) return GMG_EINVAL;
+  if (opts && opts->n_trace > 0 && (!opts->d_trace_k || !o->trace_start || !o->trace_finish))
+    return GMG_EINVAL;
+  if (opts)
+    for (int r : opts->reserved)
+      if (r != 0) return GMG_EINVAL;
+  return GMG_OK;
+}
+
+void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
+  P.out.makespan = o->makespan;
+  P.out.score = o->score;
+  P.out.status = o->status;
+  P.out.viol_flag = o->viol_flag;
+  P.out.viol_op = o->viol_op;
+  P.out.viol_dev = o->viol_dev;
+  P.out.viol_time = o->viol_time;
+  P.out.peak = o->peak;
+  P.out.sla_miss = o->sla_miss;
+  P.out.events = o->events;
+  P.out.req_done = o->req_done;
+  P.out.trace_start = o->trace_start;
+  P.out.trace_finish = o->trace_finish;
+  P.n_trace = opts ? opts->n_trace : 0;
+  P.trace_k = opts ? opts->d_trace_k : nullptr;
+}
+
+struct BasePlan {
+  size_t off_row, off_rb, off_fb, off_status, off_res, off_peak, off_creq, off_cktime, off_cksc,
+      off_ckdev, off_ckcreq, off_ckqk, off_ckqp, off_slot, total;
+  int nck, ckq, ld, stride;
+  Launch L;
+};
+
+int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
+  const DevGmg& G = g->dg;
+  Launch& L = B.L;
+  int rc = plan_launch(g, 1, o, false, L);
+  if (rc) return rc;
+  L.wpb = 1;
+  L.smem = (size_t)L.qs * 12;
+  B.nck = kCheckpoints;
+  B.ckq = std::min(L.qcap, kCheckpointQueue);
+  B.ld = (int)align_up(std::max(G.n, 1), 16);
+  B.stride = std::max(1, G.n / (B.nck - 1));
+  size_t off = 0;
+  auto take = [&](size_t bytes) {
+    const size_t at = off;
+    off = align_up(off + std::max<size_t>(bytes, 1), 256);
+    return at;
+  };
+  B.off_row = take(B.ld);
+  B.off_rb = take(8 * (size_t)G.n);
+  B.off_fb = take(8 * (size_t)G.n);
+  B.off_status = take(16);
+  B.off_res = take(64);
+  B.off_peak = take(8 * (size_t)G.D);
+  B.off_creq = take(8 * (size_t)G.R);
+  B.off_cktime = take(8 * (size_t)B.nck);
+  B.off_cksc = take(64 * (size_t)B.nck);
+  B.off_ckdev = take(24 * (size_t)G.D * B.nck);
+  B.off_ckcreq = take(8 * (size_t)G.R * B.nck);
+  B.off_ckqk = take(8 * (size_t)B.ckq * B.nck);
+  B.off_ckqp = take(4 * (size_t)B.ckq * B.nck);
+  B.off_slot = take((size_t)L.P.slot_bytes);
+  B.total = off;
+  return GMG_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+size_t gmg_workspace_bytes(const gmg_desc_t* desc) {
+  Built b;
+  if (build(desc, b) != GMG_OK) return 0;
+  return b.L.total;
+}
+
+int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t stream, gmg_t** out) {
+  if (!out) return GMG_EINVAL;
+  *out = nullptr;
+  Built b;
+  int rc = build(desc, b);
+  if (rc) return rc;
+  if (!d_ws || !aligned(d_ws, 256) || ws_bytes < b.L.total) return GMG_EWS;
+  std::vector<uint8_t> host;
+  try {
+    host.assign(b.L.total, 0);
+  } catch (const std::bad_alloc&) {
+    return GMG_ENOMEM;
+  }
+  const Layout& L = b.L;
+  auto put = [&](size_t off, const void* src, size_t bytes) {
+    if (bytes) std::memcpy(host.data() + off, src, bytes);
+  };
+  put(L.off_ops, b.ops.data(), sizeof(OpRec) * b.ops.size());
+  put(L.off_succ, b.succ.data(), 4 * b.succ.size());
+  put(L.off_pred, b.pred.data(), 4 * b.pred.size());
+  put(L.off_cons, b.cons.data(), 4 * b.cons.size());
+  put(L.off_roots, b.roots.data(), 8 * b.roots.size());
+  put(L.off_cap, b.cap.data(), 8 * b.cap.size());
+  put(L.off_base, b.base.data(), 8 * b.base.size());
+  put(L.off_avail, b.avail0.data(), 8 * b.avail0.size());
+  put(L.off_dl, b.deadline.data(), 8 * b.deadline.size());
+  if (!b.uniform) put(L.off_links, b.links.data(), sizeof(LinkRec) * b.links.size());
+  cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  if (cudaMemcpyAsync(d_ws, host.data(), b.L.total, cudaMemcpyHostToDevice, st) != cudaSuccess)
+    return GMG_ECUDA;
+  if (cudaStreamSynchronize(st) != cudaSuccess) return GMG_ECUDA;
+  gmg* g = new (std::nothrow) gmg;
+  if (!g) return GMG_ENOMEM;
+  uint8_t* w = static_cast<uint8_t*>(d_ws);
+  DevGmg& G = g->dg;
+  G.ops = reinterpret_cast<const OpRec*>(w + L.off_ops);
+  G.succ = reinterpret_cast<const uint32_t*>(w + L.off_succ);
+  G.pred = reinterpret_cast<const uint32_t*>(w + L.off_pred);
+  G.cons = reinterpret_cast<const uint32_t*>(w + L.off_cons);
+  G.root_keys = reinterpret_cast<const uint64_t*>(w + L.off_roots);
+  G.cap = reinterpret_cast<const int64_t*>(w + L.off_cap);
+  G.base = reinterpret_cast<const int64_t*>(w + L.off_base);
+  G.avail0 = reinterpret_cast<const int64_t*>(w + L.off_avail);
+  G.deadline = reinterpret_cast<const int64_t*>(w + L.off_dl);
+  G.links = b.uniform ? nullptr : reinterpret_cast<const LinkRec*>(w + L.off_links);
+  G.lat0 = b.lat0;
+  G.max_iter = b.max_iter;
+  G.n = b.n;
+  G.D = b.D;
+  G.R = b.R;
+  G.nroots = b.nroots;
+  G.ib = b.ib;
+  G.uniform = b.uniform ? 1 : 0;
+  gmg_info_t& I = g->info;
+  std::memset(&I, 0, sizeof(I));
+  I.n_ops = b.n;
+  I.n_edges = b.E;
+  I.n_dev = b.D;
+  I.n_req = b.R;
+  I.n_roots = b.nroots;
+  I.id_bits = b.ib;
+  I.time_bits = 61 - b.ib;
+  I.uniform_links = G.uniform;
+  I.time_bound = b.time_bound;
+  g->queue_bound = b.queue_bound;
+  I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
+  *out = g;
+  return GMG_OK;
+}
+
+void gmg_destroy(gmg_t* g) { delete g; }
+
+int gmg_get_info(const gmg_t* g, gmg_info_t* info) {
+  if (!g || !info) return GMG_EINVAL;
+  *info = g->info;
+  return GMG_OK;
+}
+
+size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
+  if (!g || K < 0) return 0;
+  Launch L;
+  if (plan_launch(g, K, opts, false, L)) return 0;
+  return (size_t)L.slots * (size_t)L.P.slot_bytes;
+}
+
+int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, const sim_opts_t* opts,
+              const sim_out_t* d_out, void* d_scratch, size_t scratch_bytes, gmg_stream_t stream) {
+  if (!g || K < 0) return GMG_EINVAL;
+  int rc = check_out(d_out, opts);
+  if (rc) return rc;
+  if (K == 0) return GMG_OK;
+  if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
+  Launch L;
+  rc = plan_launch(g, K, opts, false, L);
+  if (rc) return rc;
+  if (!d_scratch || !aligned(d_scratch, 256) ||
+      scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
+    return GMG_EWS;
+  SimParams& P = L.P;
+  fill_out(P, d_out, opts);
+  P.place = d_place;
+  P.ld = ld;
+  P.K = K;
+  P.scratch = static_cast<uint8_t*>(d_scratch);
+  cudaError_t e = launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
+}
+
+size_t base_workspace_bytes(const gmg_t* g, const sim_opts_t* opts) {
+  if (!g) return 0;
+  BasePlan B;
+  if (plan_base(g, opts, B)) return 0;
+  return B.total;
+}
+
+int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* opts, void* d_base_ws,
+                size_t ws_bytes, gmg_stream_t stream, gmg_base_t** out) {
+  if (!out) return GMG_EINVAL;
+  *out = nullptr;
+  if (!g || !d_base_place || !aligned(d_base_place, 16)) return GMG_EINVAL;
+  if (opts)
+    for (int r : opts->reserved)
+      if (r != 0) return GMG_EINVAL;
+  BasePlan B;
+  int rc = plan_base(g, opts, B);
+  if (rc) return rc;
+  if (!d_base_ws || !aligned(d_base_ws, 256) || ws_bytes < B.total) return GMG_EWS;
+  gmg_base* b = new (std::nothrow) gmg_base;
+  if (!b) return GMG_ENOMEM;
+  uint8_t* w = static_cast<uint8_t*>(d_base_ws);
+  DevBase& D = b->db;
+  D.row = w + B.off_row;
+  D.rb = reinterpret_cast<int64_t*>(w + B.off_rb);
+  D.fb = reinterpret_cast<int64_t*>(w + B.off_fb);
+  D.status = reinterpret_cast<int32_t*>(w + B.off_status);
+  D.res_scalars = reinterpret_cast<int64_t*>(w + B.off_res);
+  D.res_peak = reinterpret_cast<int64_t*>(w + B.off_peak);
+  D.res_creq = reinterpret_cast<int64_t*>(w + B.off_creq);
+  D.ck_time = reinterpret_cast<int64_t*>(w + B.off_cktime);
+  D.ck_scalars = reinterpret_cast<int64_t*>(w + B.off_cksc);
+  D.ck_dev = reinterpret_cast<int64_t*>(w + B.off_ckdev);
+  D.ck_creq = reinterpret_cast<int64_t*>(w + B.off_ckcreq);
+  D.ck_qkey = reinterpret_cast<uint64_t*>(w + B.off_ckqk);
+  D.ck_qpay = reinterpret_cast<uint32_t*>(w + B.off_ckqp);
+  D.nck = B.nck;
+  D.ckq = B.ckq;
+  D.ld = B.ld;
+  D.stride_pops = B.stride;
+  b->g = g;
+  b->slot = w + B.off_slot;
+  b->qs = B.L.qs;
+  b->qcap = B.L.qcap;
+  SimParams P = B.L.P;
+  P.base = D;
+  P.place = d_base_place;
+  P.ld = B.ld;
+  P.K = 1;
+  P.scratch = b->slot;
+  cudaError_t e = launch_base(B.L.reg, P, B.L.smem, reinterpret_cast<cudaStream_t>(stream));
+  if (e != cudaSuccess) {
+    delete b;
+    return GMG_ECUDA;
+  }
+  *out = b;
+  return GMG_OK;
+}
+
+void base_destroy(gmg_base_t* b) { delete b; }
+
+size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
+  if (!g || K < 0) return 0;
+  Launch L;
+  if (plan_launch(g, K, opts, true, L)) return 0;
+  return (size_t)L.slots * (size_t)L.P.slot_bytes;
+}
+
+int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_off, const int32_t* d_move_op,
+                    const uint8_t* d_move_dev, int32_t K, const sim_opts_t* opts, const sim_out_t* d_out,
+                    void* d_scratch, size_t scratch_bytes, gmg_stream_t stream) {
+  if (!g || !b || b->g != g || K < 0) return GMG_EINVAL;
+  int rc = check_out(d_out, opts);
+  if (rc) return rc;
+  if (K == 0) return GMG_OK;
+  if (!d_move_off) return GMG_EINVAL;
+  Launch L;
+  rc = plan_launch(g, K, opts, true, L);
+  if (rc) return rc;
+  if (!d_scratch || !aligned(d_scratch, 256) ||
+      scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
+    return GMG_EWS;
+  SimParams& P = L.P;
+  fill_out(P, d_out, opts);
+  P.base = b->db;
+  P.ld = b->db.ld;
+  P.K = K;
+  P.move_off = d_move_off;
+  P.move_op = d_move_op;
+  P.move_dev = d_move_dev;
+  P.scratch = static_cast<uint8_t*>(d_scratch);
+  cudaError_t e = launch_inc(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
+}
+
+size_t select_best_tmp_bytes(int32_t K) {
+  if (K < 0) return 0;
+  const int nparts = (int)std::min<int64_t>(std::max<int64_t>((K + 255) / 256, 1), 1024);
+  return (size_t)nparts * select_rank_bytes();
+}
+
+int select_best(const sim_out_t* d_out, int32_t K, int32_t score_mode, int64_t* d_best, void* d_tmp,
+                size_t tmp_bytes, gmg_stream_t stream) {
+  if (!d_out || !d_best || K < 0 || (score_mode != 0 && score_mode != 1)) return GMG_EINVAL;
+  if (!d_out->status || !d_out->viol_flag || !d_out->score || !d_out->sla_miss) return GMG_EINVAL;
+  const int nparts = (int)std::min<int64_t>(std::max<int64_t>((K + 255) / 256, 1), 1024);
+  if (!d_tmp || tmp_bytes < (size_t)nparts * select_rank_bytes() || !aligned(d_tmp, 16)) return GMG_EWS;
+  cudaError_t e = launch_select(d_out->status, d_out->viol_flag, d_out->score, d_out->sla_miss, K,
+                                score_mode, d_tmp, nparts, d_best, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
+}
+
+const char* gmg_strerror(int code) {
+  switch (code) {
+    case GMG_OK: return "ok";
+    case GMG_EINVAL: return "invalid argument or graph";
+    case GMG_ENOTTOPO: return "predecessor id not smaller than its op id";
+    case GMG_ERANGE: return "times or byte totals exceed the supported range";
+    case GMG_EWS: return "workspace or scratch too small or misaligned";
+    case GMG_ECUDA: return "CUDA runtime error";
+    case GMG_ENOMEM: return "host allocation failed";
+    case GMG_SIM_BADDEV: return "candidate: placement device id out of range";
+    case GMG_SIM_MOVE_RANGE: return "candidate: move op or device out of range";
+    case GMG_SIM_MOVE_DUP: return "candidate: op moved twice";
+    case GMG_SIM_BADBASE: return "candidate: invalid base placement";
+    case GMG_SIM_QUEUE: return "candidate: event queue capacity exceeded";
+    case GMG_SIM_LOOP: return "candidate: event loop iteration cap exceeded";
+    default: return "unknown code";
+  }
+}
+
+int64_t gmg_ceil_div_host(int64_t n, int64_t d) {
+  if (n < 0 || d < 1 || n >= (int64_t(1) << 53) || d >= (int64_t(1) << 62)) return -1;
+  return ceil_div_link(n, make_link(d, 0));
+}
+
+}  // extern "C"

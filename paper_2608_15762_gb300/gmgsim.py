@@ -1,0 +1,380 @@
+"""Thin Python binding of the C ABI in ``include/gmgsim.h``.
+
+Argument marshalling only: every step of the simulation runs in the CUDA
+kernels of ``libgmgsim.so``.  PyTorch provides device memory and streams.
+If the library is missing the calls raise; there is no fallback path.
+
+Names follow the C ABI: ``gmg_create``, ``sim_batch``, ``base_create``,
+``sim_incremental``, ``select_best`` (plus the sizing helpers).
+"""
+from __future__ import annotations
+
+import ctypes as C
+import os
+from dataclasses import dataclass
+from typing import Optional
+
+import numpy as np
+
+HERE = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(HERE, "libgmgsim.so")
+
+GMG_OK, GMG_EINVAL, GMG_ENOTTOPO, GMG_ERANGE, GMG_EWS, GMG_ECUDA, GMG_ENOMEM = 0, -1, -2, -3, -4, -5, -6
+SIM_OK, SIM_BADDEV, SIM_MOVE_RANGE, SIM_MOVE_DUP, SIM_BADBASE, SIM_QUEUE, SIM_LOOP = range(7)
+
+EXPORTED = ("gmg_workspace_bytes", "gmg_create", "gmg_destroy", "gmg_get_info", "sim_scratch_bytes",
+            "sim_batch", "base_workspace_bytes", "base_create", "base_destroy", "inc_scratch_bytes",
+            "sim_incremental", "select_best_tmp_bytes", "select_best", "gmg_strerror",
+            "gmg_ceil_div_host")
+
+
+class GmgError(RuntimeError):
+    def __init__(self, code: int, what: str):
+        super().__init__("%s failed: %s (%d)" % (what, strerror(code), code))
+        self.code = code
+
+
+class _Desc(C.Structure):
+    _fields_ = [("n_ops", C.c_int32), ("n_edges", C.c_int32), ("n_dev", C.c_int32),
+                ("n_req", C.c_int32)] + [(n, C.c_void_p) for n in (
+                    "pred_off", "pred_idx", "cons_off", "cons_idx", "dur_us", "out_bytes",
+                    "release_us", "req_id", "scored", "deadline_us", "cap_bytes", "base_bytes",
+                    "avail0_us", "bw_B_per_us", "lat_us")]
+
+
+class _Opts(C.Structure):
+    _fields_ = [("score_mode", C.c_int32), ("n_trace", C.c_int32), ("d_trace_k", C.c_void_p),
+                ("queue_cap", C.c_int32), ("warps_per_block", C.c_int32),
+                ("reserved", C.c_int32 * 4)]
+
+
+class _Out(C.Structure):
+    _fields_ = [(n, C.c_void_p) for n in (
+        "makespan", "score", "status", "viol_flag", "viol_op", "viol_dev", "viol_time", "peak",
+        "sla_miss", "events", "req_done", "trace_start", "trace_finish")]
+
+
+class _Info(C.Structure):
+    _fields_ = [("n_ops", C.c_int32), ("n_edges", C.c_int32), ("n_dev", C.c_int32),
+                ("n_req", C.c_int32), ("n_roots", C.c_int32), ("id_bits", C.c_int32),
+                ("time_bits", C.c_int32), ("uniform_links", C.c_int32),
+                ("time_bound", C.c_int64), ("default_queue_cap", C.c_int64)]
+
+
+_LIB = None
+
+
+def lib():
+    """Load libgmgsim.so (raises if it has not been built)."""
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError("libgmgsim.so is not built; run `python -m paper_2608_15762_gb300.build`")
+        L = C.CDLL(LIB_PATH)
+        vp, i32, i64, sz = C.c_void_p, C.c_int32, C.c_int64, C.c_size_t
+        sig = {
+            "gmg_workspace_bytes": ([vp], sz),
+            "gmg_create": ([vp, vp, sz, vp, vp], C.c_int),
+            "gmg_destroy": ([vp], None),
+            "gmg_get_info": ([vp, vp], C.c_int),
+            "sim_scratch_bytes": ([vp, i32, vp], sz),
+            "sim_batch": ([vp, vp, i32, i32, vp, vp, vp, sz, vp], C.c_int),
+            "base_workspace_bytes": ([vp, vp], sz),
+            "base_create": ([vp, vp, vp, vp, sz, vp, vp], C.c_int),
+            "base_destroy": ([vp], None),
+            "inc_scratch_bytes": ([vp, i32, vp], sz),
+            "sim_incremental": ([vp, vp, vp, vp, vp, i32, vp, vp, vp, sz, vp], C.c_int),
+            "select_best_tmp_bytes": ([i32], sz),
+            "select_best": ([vp, i32, i32, vp, vp, sz, vp], C.c_int),
+            "gmg_strerror": ([C.c_int], C.c_char_p),
+            "gmg_ceil_div_host": ([i64, i64], i64),
+        }
+        for name, (args, res) in sig.items():
+            f = getattr(L, name)
+            f.argtypes = args
+            f.restype = res
+        _LIB = L
+    return _LIB
+
+
+def strerror(code: int) -> str:
+    return lib().gmg_strerror(int(code)).decode()
+
+
+def _stream_handle(stream) -> Optional[int]:
+    import torch
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return int(s.cuda_stream) or None
+
+
+def _np_ptr(a):
+    return None if a is None else a.ctypes.data
+
+
+class _DescHolder:
+    def __init__(self, desc):
+        d = desc.normalized()
+        self.d = d
+        self.c = _Desc(d.n_ops, d.n_edges, d.n_dev, d.n_req, _np_ptr(d.pred_off), _np_ptr(d.pred_idx),
+                       _np_ptr(d.cons_off), _np_ptr(d.cons_idx), _np_ptr(d.dur), _np_ptr(d.out_bytes),
+                       _np_ptr(d.release), _np_ptr(d.req_id), _np_ptr(d.scored), _np_ptr(d.deadline),
+                       _np_ptr(d.cap), _np_ptr(d.base), _np_ptr(d.avail0), _np_ptr(d.bw), _np_ptr(d.lat))
+
+
+def gmg_workspace_bytes(desc) -> int:
+    h = _DescHolder(desc)
+    return int(lib().gmg_workspace_bytes(C.addressof(h.c)))
+
+
+def _opts(score_mode=0, trace_k=None, queue_cap=0, warps_per_block=0) -> _Opts:
+    o = _Opts()
+    o.score_mode = score_mode
+    o.n_trace = 0 if trace_k is None else int(trace_k.numel())
+    o.d_trace_k = None if trace_k is None else trace_k.data_ptr()
+    o.queue_cap = queue_cap
+    o.warps_per_block = warps_per_block
+    return o
+
+
+def _aligned_empty(nbytes: int, device, align: int = 256):
+    """A uint8 device tensor view whose data pointer is `align`-aligned."""
+    import torch
+    buf = torch.empty(max(int(nbytes), 1) + align, dtype=torch.uint8, device=device)
+    off = (-buf.data_ptr()) % align
+    return buf[off:off + max(int(nbytes), 1)]
+
+
+class Gmg:
+    """A created GMG: host handle + the device workspace it borrows."""
+
+    def __init__(self, desc, device="cuda", stream=None):
+        import torch
+        self.desc = desc.normalized()
+        self._h = _DescHolder(self.desc)
+        nbytes = lib().gmg_workspace_bytes(C.addressof(self._h.c))
+        if nbytes == 0:
+            # let gmg_create report the reason
+            nbytes = 256
+        self.device = torch.device(device)
+        self.ws = _aligned_empty(nbytes, self.device)
+        handle = C.c_void_p()
+        rc = lib().gmg_create(C.addressof(self._h.c), self.ws.data_ptr(), self.ws.numel(),
+                              _stream_handle(stream), C.addressof(handle))
+        if rc != GMG_OK:
+            raise GmgError(rc, "gmg_create")
+        self.handle = handle
+
+    @property
+    def info(self) -> dict:
+        i = _Info()
+        rc = lib().gmg_get_info(self.handle, C.addressof(i))
+        if rc:
+            raise GmgError(rc, "gmg_get_info")
+        return {n: getattr(i, n) for n, _ in _Info._fields_}
+
+    @property
+    def n_ops(self):
+        return self.desc.n_ops
+
+    @property
+    def n_dev(self):
+        return self.desc.n_dev
+
+    @property
+    def n_req(self):
+        return self.desc.n_req
+
+    def close(self):
+        if getattr(self, "handle", None):
+            lib().gmg_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def gmg_create(desc, device="cuda", stream=None) -> Gmg:
+    return Gmg(desc, device, stream)
+
+
+@dataclass
+class SimOut:
+    """Device output tensors for K candidates (fields of sim_out_t)."""
+    makespan: "object"
+    score: "object"
+    status: "object"
+    viol_flag: "object"
+    viol_op: "object"
+    viol_dev: "object"
+    viol_time: "object"
+    peak: "object"
+    sla_miss: "object"
+    events: "object"
+    req_done: "object" = None
+    trace_start: "object" = None
+    trace_finish: "object" = None
+
+    @staticmethod
+    def empty(K: int, n_dev: int, n_req: int, device, req_done=False, n_trace=0, n_ops=0) -> "SimOut":
+        import torch
+        i64, i32 = torch.int64, torch.int32
+        return SimOut(
+            makespan=torch.empty(K, dtype=i64, device=device),
+            score=torch.empty(K, dtype=i64, device=device),
+            status=torch.empty(K, dtype=i32, device=device),
+            viol_flag=torch.empty(K, dtype=i32, device=device),
+            viol_op=torch.empty(K, dtype=i32, device=device),
+            viol_dev=torch.empty(K, dtype=i32, device=device),
+            viol_time=torch.empty(K, dtype=i64, device=device),
+            peak=torch.empty((K, n_dev), dtype=i64, device=device),
+            sla_miss=torch.empty(K, dtype=i32, device=device),
+            events=torch.empty(K, dtype=i64, device=device),
+            req_done=torch.empty((K, n_req), dtype=i64, device=device) if req_done else None,
+            trace_start=torch.empty((n_trace, n_ops), dtype=i64, device=device) if n_trace else None,
+            trace_finish=torch.empty((n_trace, n_ops), dtype=i64, device=device) if n_trace else None)
+
+    def _c(self) -> _Out:
+        def p(t):
+            return None if t is None else t.data_ptr()
+        return _Out(p(self.makespan), p(self.score), p(self.status), p(self.viol_flag), p(self.viol_op),
+                    p(self.viol_dev), p(self.viol_time), p(self.peak), p(self.sla_miss), p(self.events),
+                    p(self.req_done), p(self.trace_start), p(self.trace_finish))
+
+    def to_numpy(self) -> dict:
+        return {k: (None if v is None else v.cpu().numpy()) for k, v in self.__dict__.items()}
+
+
+def sim_scratch_bytes(g: Gmg, K: int, **opt) -> int:
+    o = _opts(**opt)
+    return int(lib().sim_scratch_bytes(g.handle, K, C.addressof(o)))
+
+
+def inc_scratch_bytes(g: Gmg, K: int, **opt) -> int:
+    o = _opts(**opt)
+    return int(lib().inc_scratch_bytes(g.handle, K, C.addressof(o)))
+
+
+class Scratch:
+    """A reusable aligned device scratch buffer, grown on demand."""
+
+    def __init__(self, device):
+        self.device = device
+        self.buf = None
+
+    def get(self, nbytes: int):
+        if self.buf is None or self.buf.numel() < nbytes:
+            self.buf = _aligned_empty(nbytes, self.device)
+        return self.buf
+
+
+def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scratch] = None,
+              req_done=False, trace_k=None, queue_cap=0, warps_per_block=0, stream=None) -> SimOut:
+    """Simulate every row of ``place`` (CUDA uint8 [K, ld], ld % 16 == 0)."""
+    import torch
+    assert place.dtype == torch.uint8 and place.dim() == 2 and place.is_contiguous()
+    K, ld = place.shape
+    n_trace = 0 if trace_k is None else int(trace_k.numel())
+    if out is None:
+        out = SimOut.empty(K, g.n_dev, g.n_req, place.device, req_done, n_trace, g.n_ops)
+    o = _opts(0, trace_k, queue_cap, warps_per_block)
+    need = lib().sim_scratch_bytes(g.handle, K, C.addressof(o))
+    scratch = scratch or Scratch(place.device)
+    buf = scratch.get(need)
+    co = out._c()
+    rc = lib().sim_batch(g.handle, place.data_ptr(), K, ld, C.addressof(o), C.addressof(co),
+                         buf.data_ptr(), buf.numel(), _stream_handle(stream))
+    if rc != GMG_OK:
+        raise GmgError(rc, "sim_batch")
+    return out
+
+
+class Base:
+    """A recorded base schedule (base_create) and the workspace it borrows."""
+
+    def __init__(self, g: Gmg, base_place, queue_cap=0, stream=None):
+        import torch
+        assert base_place.dtype == torch.uint8 and base_place.is_contiguous()
+        ld = (g.n_ops + 15) // 16 * 16
+        row = torch.zeros(max(ld, 16), dtype=torch.uint8, device=base_place.device)
+        row[:base_place.numel()] = base_place[:ld].reshape(-1)
+        self.row = row
+        self.g = g
+        o = _opts(0, None, queue_cap)
+        nbytes = lib().base_workspace_bytes(g.handle, C.addressof(o))
+        self.ws = _aligned_empty(nbytes, base_place.device)
+        h = C.c_void_p()
+        rc = lib().base_create(g.handle, row.data_ptr(), C.addressof(o), self.ws.data_ptr(),
+                               self.ws.numel(), _stream_handle(stream), C.addressof(h))
+        if rc != GMG_OK:
+            raise GmgError(rc, "base_create")
+        self.handle = h
+
+    def close(self):
+        if getattr(self, "handle", None):
+            lib().base_destroy(self.handle)
+            self.handle = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+
+def base_create(g: Gmg, base_place, queue_cap=0, stream=None) -> Base:
+    return Base(g, base_place, queue_cap, stream)
+
+
+def sim_incremental(g: Gmg, base: Base, move_off, move_op, move_dev, out: Optional[SimOut] = None,
+                    scratch: Optional[Scratch] = None, req_done=False, trace_k=None, queue_cap=0,
+                    warps_per_block=0, stream=None) -> SimOut:
+    """K move lists (CUDA int32 off[K+1], int32 op[M], uint8 dev[M]) against ``base``."""
+    K = int(move_off.numel()) - 1
+    n_trace = 0 if trace_k is None else int(trace_k.numel())
+    if out is None:
+        out = SimOut.empty(K, g.n_dev, g.n_req, move_off.device, req_done, n_trace, g.n_ops)
+    o = _opts(0, trace_k, queue_cap, warps_per_block)
+    need = lib().inc_scratch_bytes(g.handle, K, C.addressof(o))
+    scratch = scratch or Scratch(move_off.device)
+    buf = scratch.get(need)
+    co = out._c()
+    rc = lib().sim_incremental(g.handle, base.handle, move_off.data_ptr(),
+                               move_op.data_ptr() if move_op.numel() else None,
+                               move_dev.data_ptr() if move_dev.numel() else None, K, C.addressof(o),
+                               C.addressof(co), buf.data_ptr(), buf.numel(), _stream_handle(stream))
+    if rc != GMG_OK:
+        raise GmgError(rc, "sim_incremental")
+    return out
+
+
+def select_best(out: SimOut, K: Optional[int] = None, score_mode: int = 0, best=None, tmp=None,
+                stream=None):
+    """Device int64[2] = (best candidate or -1, its score)."""
+    import torch
+    K = int(out.score.numel()) if K is None else K
+    dev = out.score.device
+    if best is None:
+        best = torch.empty(2, dtype=torch.int64, device=dev)
+    need = lib().select_best_tmp_bytes(K)
+    if tmp is None or tmp.numel() < need:
+        tmp = _aligned_empty(need, dev)
+    co = out._c()
+    rc = lib().select_best(C.addressof(co), K, score_mode, best.data_ptr(), tmp.data_ptr(), tmp.numel(),
+                           _stream_handle(stream))
+    if rc != GMG_OK:
+        raise GmgError(rc, "select_best")
+    return best
+
+
+def ceil_div_host(n: int, d: int) -> int:
+    return int(lib().gmg_ceil_div_host(n, d))
+
+
+def moves_to_device(moves, device):
+    import torch
+    return (torch.from_numpy(np.ascontiguousarray(moves.off, np.int32)).to(device),
+            torch.from_numpy(np.ascontiguousarray(moves.op, np.int32)).to(device),
+            torch.from_numpy(np.ascontiguousarray(moves.dev, np.uint8)).to(device))

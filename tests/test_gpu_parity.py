@@ -1,0 +1,189 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle, bit for
+bit on every output field (all times and sizes are int64)."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from gpu_common import compare, oracle_rows, torch_place  # noqa: E402
+from helpers import mk, row  # noqa: E402
+from oracle import oracle as O  # noqa: E402
+from paper_2608_15762_gb300 import gmgsim as G  # noqa: E402
+from paper_2608_15762_gb300 import workloads as W  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_15762_gb300 import build
+    build.build()
+    assert torch.cuda.is_available()
+
+
+def _random_case(seed, n, D, **kw):
+    d = W.random_desc(seed, n, D, **kw)
+    g = np.random.default_rng(seed)
+    K = 37
+    ld = W.placement_ld(n)
+    rows = np.zeros((K, ld), np.uint8)
+    rows[:, :n] = g.integers(0, D, (K, n))
+    return d, rows
+
+
+@pytest.mark.parametrize("seed,n,D,kw", [
+    (1, 1, 1, {}),
+    (2, 7, 2, {}),
+    (3, 33, 3, dict(explicit_cons=True)),
+    (4, 64, 4, dict(link_hetero=False)),
+    (5, 150, 8, dict(explicit_cons=True, dur_hi=2000)),
+    (6, 257, 5, dict(max_pred=6)),
+    (7, 300, 32, dict(explicit_cons=True)),
+    (8, 200, 33, {}),          # accelerator state in scratch arrays
+    (9, 500, 256, dict(explicit_cons=True, bytes_hi=1 << 30)),
+    (10, 1000, 16, dict(edge_p=0.9, max_pred=4)),
+    (11, 90, 6, dict(with_release=False, with_avail0=False, cap=1 << 40)),
+])
+def test_random_dags_bit_exact(seed, n, D, kw):
+    d, rows = _random_case(seed, n, D, **kw)
+    g = G.gmg_create(d)
+    K = rows.shape[0]
+    tk = torch.tensor([0, 5, K - 1], dtype=torch.int32, device="cuda")
+    out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk)
+    best = G.select_best(out)
+    best1 = G.select_best(out, score_mode=1)
+    torch.cuda.synchronize()
+    got = out.to_numpy()
+    s, pk, rq = oracle_rows(d, rows)
+    compare(got, s, pk, rq)
+    for slot, k in enumerate([0, 5, K - 1]):
+        r = O.simulate(d, rows[k])
+        assert np.array_equal(got["trace_start"][slot], r["start"])
+        assert np.array_equal(got["trace_finish"][slot], r["finish"])
+    assert best.cpu().tolist() == list(O.select_best(s, 0))
+    assert best1.cpu().tolist() == list(O.select_best(s, 1))
+
+
+def test_bad_device_rows_and_empty_graph():
+    d, rows = _random_case(12, 40, 3)
+    rows[3, 17] = 3
+    rows[9, 39] = 255
+    rows[11, 40] = 200       # padding byte beyond n_ops: ignored
+    g = G.gmg_create(d)
+    out = G.sim_batch(g, torch_place(rows), req_done=True)
+    torch.cuda.synchronize()
+    s, pk, rq = oracle_rows(d, rows)
+    compare(out.to_numpy(), s, pk, rq)
+    st = out.status.cpu().numpy()
+    assert st[3] == G.SIM_BADDEV and st[9] == G.SIM_BADDEV and st[11] == 0
+    e = mk([], [], n_dev=2)
+    ge = G.gmg_create(e)
+    oe = G.sim_batch(ge, torch_place(np.zeros((4, 16), np.uint8)))
+    torch.cuda.synchronize()
+    assert oe.status.cpu().tolist() == [0] * 4 and oe.score.cpu().tolist() == [0] * 4
+
+
+def test_golden_examples_on_gpu():
+    import json, glob, os
+    for path in sorted(glob.glob(os.path.join(os.path.dirname(__file__), "golden", "*.json"))):
+        fx = json.load(open(path))
+        gr = fx["graph"]
+        for case in fx["cases"]:
+            d = mk(gr["preds"], gr["dur"], gr["out_bytes"], n_dev=gr["n_dev"], bw=gr["bw"],
+                   lat=gr["lat"], release=gr.get("release"), avail0=gr.get("avail0"),
+                   req_id=gr.get("req_id"), deadline=gr.get("deadline"), cap=case["cap"])
+            g = G.gmg_create(d)
+            rows = row(fx["place"])[None, :]
+            tk = torch.tensor([0], dtype=torch.int32, device="cuda")
+            out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk).to_numpy()
+            assert out["trace_start"][0].tolist() == case["start"]
+            assert out["trace_finish"][0].tolist() == case["finish"]
+            assert out["peak"][0].tolist() == case["peak"]
+            assert out["makespan"][0] == case["makespan"] and out["score"][0] == case["score"]
+            viol = None if not out["viol_flag"][0] else [int(out["viol_time"][0]),
+                                                         int(out["viol_op"][0]),
+                                                         int(out["viol_dev"][0])]
+            assert viol == case["viol"]
+
+
+def test_queue_capacity_status():
+    d, rows = _random_case(13, 120, 4)
+    g = G.gmg_create(d)
+    out = G.sim_batch(g, torch_place(rows), queue_cap=3)
+    torch.cuda.synchronize()
+    st = out.status.cpu().numpy()
+    assert (st == G.SIM_QUEUE).any()
+    sc = out.score.cpu().numpy()
+    assert (sc[st == G.SIM_QUEUE] == np.iinfo(np.int64).max).all()
+    best = G.select_best(out).cpu().tolist()
+    assert best[0] == -1 or st[best[0]] == 0
+
+
+@pytest.mark.parametrize("wpb", [1, 2, 3, 4])
+def test_launch_shapes_agree(wpb):
+    d, rows = _random_case(14, 200, 8)
+    g = G.gmg_create(d)
+    out = G.sim_batch(g, torch_place(rows), req_done=True, warps_per_block=wpb)
+    torch.cuda.synchronize()
+    s, pk, rq = oracle_rows(d, rows)
+    compare(out.to_numpy(), s, pk, rq)
+
+
+# ---------------------------------------------------------------------------
+# The workloads
+# ---------------------------------------------------------------------------
+
+def test_workload_tiny_all_candidates():
+    wl = W.config1()
+    rows = wl.all_full_rows()
+    g = G.gmg_create(wl.desc)
+    out = G.sim_batch(g, torch_place(rows), req_done=True)
+    best = G.select_best(out)
+    torch.cuda.synchronize()
+    s, pk, rq = oracle_rows(wl.desc, rows)
+    compare(out.to_numpy(), s, pk, rq)
+    assert best.cpu().tolist() == list(O.select_best(s, 0))
+
+
+def test_workload_prefill_all_candidates():
+    wl = W.config2()
+    rows = wl.all_full_rows()
+    g = G.gmg_create(wl.desc)
+    out = G.sim_batch(g, torch_place(rows), req_done=True)
+    best = G.select_best(out)
+    best1 = G.select_best(out, score_mode=1)
+    torch.cuda.synchronize()
+    s, pk, rq = oracle_rows(wl.desc, rows)
+    compare(out.to_numpy(), s, pk, rq)
+    assert best.cpu().tolist() == list(O.select_best(s, 0))
+    assert best1.cpu().tolist() == list(O.select_best(s, 1))
+    assert (s["sla_miss"] > 0).any()
+
+
+def test_workload_memory_tight_sampled():
+    wl = W.config4()
+    K = wl.n_full
+    ks = np.random.default_rng(44).choice(K, 24, replace=False)
+    ks.sort()
+    g = G.gmg_create(wl.desc)
+    place = torch_place(wl.all_full_rows())
+    out = G.sim_batch(g, place, req_done=True)
+    torch.cuda.synchronize()
+    got = out.to_numpy()
+    s, pk, rq = oracle_rows(wl.desc, wl.full_rows(ks))
+    compare(got, s, pk, rq, ks=ks)
+    frac = float(got["viol_flag"].mean())
+    assert 0.25 < frac < 0.35, frac
+    assert (got["status"] == 0).all() and (got["events"] == wl.desc.n_ops).all()
+
+
+def test_workload_large_full_half_sampled():
+    wl = W.config5()
+    ks = np.random.default_rng(55).choice(wl.n_full, 8, replace=False)
+    ks.sort()
+    g = G.gmg_create(wl.desc)
+    rows = wl.full_rows(ks)
+    out = G.sim_batch(g, torch_place(rows), req_done=True)
+    torch.cuda.synchronize()
+    s, pk, rq = oracle_rows(wl.desc, rows)
+    compare(out.to_numpy(), s, pk, rq)
