@@ -31,6 +31,8 @@ constexpr uint32_t kScored = 1u;   // counts in the score
 constexpr uint32_t kReqSink = 2u;  // no successor in its own request: may end the request
 constexpr uint32_t kAllCons = 4u;  // consumers = successors
 constexpr uint32_t kHoldBit = 0x80000000u;
+constexpr uint32_t kSibNone = 0xffffffffu;  // the only listed consumer
+constexpr uint32_t kSibMany = 0xfffffffeu;  // three or more listed consumers
 constexpr uint32_t kIdMask = 0x7fffffffu;
 
 // Exact ceil(n / bw) by multiply-shift (Granlund & Montgomery 1994,
@@ -74,6 +76,8 @@ struct DevGmg {
   const OpRec* ops;
   const uint32_t* succ;
   const uint32_t* pred;
+  const uint32_t* psib;       // per predecessor entry of a holding consumer: the other
+                              // listed consumer of that predecessor (kSibNone / kSibMany)
   const uint32_t* cons;
   const uint64_t* root_keys;  // READY keys of ops without predecessors, ascending
   const int64_t* cap;
@@ -85,6 +89,8 @@ struct DevGmg {
   int64_t max_iter;           // event-loop iteration cap per candidate
   int32_t n, D, R, nroots;
   int32_t ib;                 // op-id bits of a packed key
+  int32_t tb;                 // time bits needed (every time < 2^tb)
+  int32_t dev_key;            // 1 if an accelerator id fits above (time, class, op) in 64 bits
   int32_t uniform;
 };
 
@@ -117,6 +123,7 @@ struct DevBase {
   uint8_t* row;          // [ld] base placement
   int64_t* rb;           // [N] base ready time
   int64_t* fb;           // [N] base finish time
+  int64_t* hb;           // [N] base hold time (latest outgoing arrival)
   int32_t* status;       // [1]
   // base results (outputs of the base placement)
   int64_t* res_scalars;  // [8]: makespan, score, viol_flag, viol_op, viol_dev, viol_time, sla_miss, n_ck
@@ -124,13 +131,17 @@ struct DevBase {
   int64_t* res_creq;     // [R]
   // checkpoints c = 0 .. nck-1
   int64_t* ck_time;      // [nck]  T_c (INT64_MAX = not recorded)
-  int64_t* ck_scalars;   // [nck*8]: qsize, rootptr, score, makespan, vflag, vt, vop, vdev
+  int64_t* ck_scalars;   // [nck*8]: qsize, rootptr, score, makespan, vflag, vt, vop<<32|vdev, log size
   int64_t* ck_dev;       // [nck*3*D]: free, live, peak
   int64_t* ck_creq;      // [nck*R]
-  uint64_t* ck_qkey;     // [nck*ckq]
-  uint32_t* ck_qpay;     // [nck*ckq]
+  uint64_t* ck_qkey;     // [nck*ckq] READY heap
+  uint64_t* ck_mkey;     // [nck*ckm] HBM event log entries
+  uint8_t* ck_mdev;      // [nck*ckm] their accelerators (when not inside the entries)
+  uint32_t* ck_bits;     // [nck*ck_words] simulated-op bitmap
   int32_t nck;
-  int32_t ckq;           // entries per checkpoint queue
+  int32_t ckq;           // READY entries per checkpoint
+  int32_t ckm;           // HBM events per checkpoint
+  int32_t ck_words;      // bitmap words per checkpoint
   int32_t ld;
   int32_t stride_pops;   // READY pops between checkpoints
 };
@@ -142,8 +153,12 @@ struct SimParams {
   const uint8_t* place;  // kFull: [K][ld]; kBase: base row
   int64_t ld;
   int32_t K;
-  int32_t qs;            // queue entries in shared memory per warp (32m+1)
-  int32_t qcap;          // total queue entries per warp
+  int32_t qs;            // READY heap slots in shared memory per warp (32m+1, >= 33)
+  int32_t qcap;          // READY heap slots per warp
+  int32_t ms;            // HBM event log slots in shared memory per warp
+  int32_t mcap;          // HBM event log slots per warp
+  int32_t sortcap;       // sort area entries per warp (power of two, >= max(32, n_dev))
+  int32_t drain_trigger; // drain the log after this many new events
   int32_t n_trace;
   const int32_t* trace_k;
   const int32_t* move_off;
@@ -152,7 +167,7 @@ struct SimParams {
   uint8_t* scratch;
   int64_t slot_bytes;    // scratch bytes per warp slot
   // byte offsets inside a slot
-  int64_t off_f, off_bits, off_creq, off_qk, off_qp, off_dev, off_row;
+  int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row;
 };
 
 }  // namespace gsim

@@ -19,6 +19,7 @@ const void* inc_kernel_ptr(bool reg);
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
+cudaError_t set_smem_limits(int smem);
 cudaError_t launch_select(const int32_t* status, const int32_t* viol, const int64_t* score,
                           const int32_t* miss, int32_t K, int32_t mode, void* tmp, int nparts,
                           int64_t* best, cudaStream_t st);
@@ -31,25 +32,30 @@ namespace {
 constexpr int64_t kI64Max = 0x7fffffffffffffffll;
 constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
 constexpr int kDefaultWarpsPerBlock = 4;
-constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root and two child levels
+constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
 constexpr int64_t kDefaultQueueCap = 1 << 16;
+constexpr int kSharedLogEntries = 160;
+constexpr int64_t kDefaultLogCap = 1 << 17;
+constexpr int kSortCap = 128;             // power of two; raised to n_dev's power of two
+constexpr int kDrainTrigger = 64;
 constexpr int kCheckpoints = 256;
 constexpr int kCheckpointQueue = 4096;
+constexpr int kCheckpointLog = 8192;
 
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
-  size_t off_ops, off_succ, off_pred, off_cons, off_roots, off_cap, off_base, off_avail, off_dl,
-      off_links, total;
+  size_t off_ops, off_succ, off_pred, off_sib, off_cons, off_roots, off_cap, off_base, off_avail,
+      off_dl, off_links, total;
 };
 
 // Everything gmg_create derives from a description.
 struct Built {
   int n = 0, E = 0, D = 0, R = 0, Ec = 0, nroots = 0, ib = 1;
   bool uniform = true;
-  int64_t bw0 = 1, lat0 = 0, time_bound = 0, max_iter = 0, queue_bound = 0;
+  int64_t bw0 = 1, lat0 = 0, time_bound = 0, max_iter = 0, queue_bound = 0, log_bound = 0;
   std::vector<OpRec> ops;
-  std::vector<uint32_t> succ, pred, cons;
+  std::vector<uint32_t> succ, pred, sib, cons;
   std::vector<uint64_t> roots;
   std::vector<int64_t> cap, base, avail0, deadline;
   std::vector<LinkRec> links;
@@ -86,6 +92,7 @@ void plan(Built& b) {
   L.off_ops = take(sizeof(OpRec) * (size_t)b.n);
   L.off_succ = take(4 * (size_t)b.E);
   L.off_pred = take(4 * (size_t)b.E);
+  L.off_sib = take(4 * (size_t)b.E);
   L.off_cons = take(4 * (size_t)b.Ec);
   L.off_roots = take(8 * (size_t)b.nroots);
   L.off_cap = take(8 * (size_t)b.D);
@@ -206,6 +213,21 @@ int build(const gmg_desc_t* d, Built& b) {
     }
   }
   b.Ec = (int)b.cons.size();
+  // For every (predecessor p -> holding consumer c) entry: the other listed
+  // consumer of p, so that c can tell whether it is p's last one there.
+  b.sib.assign(b.E, kSibNone);
+  for (int p = 0; p < n; ++p) {
+    const OpRec& r = b.ops[p];
+    const uint32_t* lst = (r.flags & kAllCons) ? b.succ.data() + r.succ_off : b.cons.data() + r.cons_off;
+    for (uint32_t u = 0; u < r.ncons; ++u) {
+      const uint32_t c = lst[u];
+      uint32_t v = kSibNone;
+      if (r.ncons == 2) v = lst[1 - u];
+      else if (r.ncons > 2) v = kSibMany;
+      for (uint32_t k = b.ops[c].pred_off; k < b.ops[c].pred_off + b.ops[c].npred; ++k)
+        if ((b.pred[k] & kIdMask) == (uint32_t)p) b.sib[k] = v;
+    }
+  }
   // request sinks: no successor in the same request
   for (int i = 0; i < n; ++i) {
     OpRec& r = b.ops[i];
@@ -265,7 +287,7 @@ int build(const gmg_desc_t* d, Built& b) {
   // per op; it must fit the packed key (61 - ib bits); scores and byte totals
   // must fit int64.
   typedef __int128 i128;
-  i128 t = 0, mem = 0, iters = 16, qb = 16;
+  i128 t = 0, mem = 0, iters = 16, qb = 16, lb = 16;
   for (int e = 0; e < D; ++e) {
     t = std::max<i128>(t, b.avail0[e]);
     mem += b.base[e];
@@ -278,14 +300,16 @@ int build(const gmg_desc_t* d, Built& b) {
     const uint32_t copies = std::min<uint32_t>(r.nsucc, (uint32_t)(D - 1));
     t += r.dur + mx * i128(r.nsucc + 1);
     mem += i128(r.bytes) * i128(copies + 1);
-    iters += 3 + 2 * i128(copies);
-    qb += (r.npred ? 1 : 0) + 2 + 2 * i128(copies);
+    iters += 1;
+    qb += r.npred ? 1 : 0;
+    lb += 2 + 2 * i128(copies);
     if (t >= tlim || mem >= (i128(1) << 62)) return GMG_ERANGE;
   }
   if (t * i128(std::max(n, 1)) >= (i128(1) << 62)) return GMG_ERANGE;
   b.time_bound = (int64_t)t;
   b.max_iter = (int64_t)iters;
   b.queue_bound = (int64_t)qb;
+  b.log_bound = (int64_t)lb;
   // roots, by (release, id)
   for (int i = 0; i < n; ++i)
     if (b.ops[i].npred == 0)
@@ -309,6 +333,7 @@ struct gmg {
   DevGmg dg;
   gmg_info_t info;
   int64_t queue_bound;
+  int64_t log_bound;
 };
 
 struct gmg_base {
@@ -322,21 +347,28 @@ namespace {
 
 struct Launch {
   bool reg;
-  int wpb, qs, qcap, grid;
+  int wpb, grid;
   size_t smem;
   int64_t slots;
-  SimParams P;  // offsets filled
+  SimParams P;  // sizes and slot offsets filled
 };
 
 int queue_cap(const gmg* g, const sim_opts_t* o) {
-  int64_t c = (o && o->queue_cap > 0) ? o->queue_cap : std::min<int64_t>(g->queue_bound, kDefaultQueueCap);
+  const int64_t c = (o && o->queue_cap > 0) ? o->queue_cap : std::min<int64_t>(g->queue_bound, kDefaultQueueCap);
   return (int)std::max<int64_t>(c, 1);
 }
 
-int shared_entries(int qcap) {
-  const int m = std::min(kSharedQueueEntries, qcap);
-  return ((m + 30) / 32) * 32 + 1;  // 32m + 1 >= m
+int log_cap(const gmg* g, const sim_opts_t* o) {
+  const int64_t c = (o && o->queue_cap > 0) ? 2 * (int64_t)o->queue_cap
+                                           : std::min<int64_t>(g->log_bound, kDefaultLogCap);
+  return (int)std::max<int64_t>(c, 1);
 }
+
+size_t smem_per_warp(const SimParams& P) {
+  return align_up((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9, 16) + (size_t)P.g.D * 24;
+}
+
+bool g_smem_set = false;
 
 // Slot layout and grid for K candidates of kind `inc`.
 int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& L) {
@@ -344,30 +376,44 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   L.reg = G.D <= 32;
   L.wpb = (o && o->warps_per_block > 0) ? o->warps_per_block : kDefaultWarpsPerBlock;
   if (L.wpb > 4) return GMG_EINVAL;
-  L.qcap = queue_cap(g, o);
-  L.qs = shared_entries(L.qcap);
-  L.smem = (size_t)L.wpb * L.qs * 12;
   SimParams& P = L.P;
   std::memset(&P, 0, sizeof(P));
+  P.g = G;
+  P.qcap = queue_cap(g, o);
+  P.qs = kSharedQueueEntries;   // >= 33 (the root's children are always in shared memory)
+  P.mcap = log_cap(g, o);
+  P.ms = kSharedLogEntries;
+  P.sortcap = kSortCap;
+  while (P.sortcap < G.D) P.sortcap <<= 1;
+  P.drain_trigger = kDrainTrigger;
+  L.smem = (size_t)L.wpb * smem_per_warp(P);
   size_t o2 = 0;
   auto take = [&](size_t bytes) {
     const size_t at = o2;
     o2 = align_up(o2 + std::max<size_t>(bytes, 1), 256);
     return (int64_t)at;
   };
-  const int64_t spill = std::max<int64_t>(L.qcap - L.qs, 0);
+  const int64_t qspill = std::max<int64_t>(P.qcap - P.qs, 0);
+  const int64_t mspill = std::max<int64_t>(P.mcap - P.ms, 0);
   P.off_f = take(8 * (size_t)G.n);
+  P.off_hold = take(8 * (size_t)G.n);
   P.off_bits = take(4 * (size_t)((G.n + 31) / 32) + 16);
   P.off_creq = take(8 * (size_t)G.R);
-  P.off_qk = take(8 * (size_t)spill);
-  P.off_qp = take(4 * (size_t)spill);
-  P.off_dev = take(L.reg ? 0 : 24 * (size_t)G.D);
+  P.off_qk = take(8 * (size_t)qspill);
+  P.off_mk = take(8 * (size_t)mspill);
+  P.off_md = take((size_t)mspill);
   P.off_row = take(inc ? (size_t)align_up(std::max(G.n, 1), 16) : 0);
   P.slot_bytes = (int64_t)o2;
-  P.qs = L.qs;
-  P.qcap = L.qcap;
   const int sms = device_sms();
   if (sms <= 0) return GMG_ECUDA;
+  if (!g_smem_set) {
+    // the largest per-block request: 4 warps with 256 accelerators
+    SimParams big = P;
+    big.g.D = 256;
+    big.sortcap = 256;
+    if (set_smem_limits(4 * (int)smem_per_warp(big)) != cudaSuccess) return GMG_ECUDA;
+    g_smem_set = true;
+  }
   int bps = 0;
   const void* fn = inc ? inc_kernel_ptr(L.reg) : full_kernel_ptr(L.reg);
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
@@ -414,9 +460,9 @@ void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
 }
 
 struct BasePlan {
-  size_t off_row, off_rb, off_fb, off_status, off_res, off_peak, off_creq, off_cktime, off_cksc,
-      off_ckdev, off_ckcreq, off_ckqk, off_ckqp, off_slot, total;
-  int nck, ckq, ld, stride;
+  size_t off_row, off_rb, off_fb, off_hb, off_status, off_res, off_peak, off_creq, off_cktime,
+      off_cksc, off_ckdev, off_ckcreq, off_ckqk, off_ckmk, off_ckmd, off_ckbits, off_slot, total;
+  int nck, ckq, ckm, ckw, ld, stride;
   Launch L;
 };
 
@@ -426,9 +472,11 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   int rc = plan_launch(g, 1, o, false, L);
   if (rc) return rc;
   L.wpb = 1;
-  L.smem = (size_t)L.qs * 12;
+  L.smem = smem_per_warp(L.P);
   B.nck = kCheckpoints;
-  B.ckq = std::min(L.qcap, kCheckpointQueue);
+  B.ckq = std::min(L.P.qcap, kCheckpointQueue);
+  B.ckm = std::min(L.P.mcap, kCheckpointLog);
+  B.ckw = (G.n + 31) / 32;
   B.ld = (int)align_up(std::max(G.n, 1), 16);
   B.stride = std::max(1, G.n / (B.nck - 1));
   size_t off = 0;
@@ -440,6 +488,7 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   B.off_row = take(B.ld);
   B.off_rb = take(8 * (size_t)G.n);
   B.off_fb = take(8 * (size_t)G.n);
+  B.off_hb = take(8 * (size_t)G.n);
   B.off_status = take(16);
   B.off_res = take(64);
   B.off_peak = take(8 * (size_t)G.D);
@@ -449,7 +498,9 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   B.off_ckdev = take(24 * (size_t)G.D * B.nck);
   B.off_ckcreq = take(8 * (size_t)G.R * B.nck);
   B.off_ckqk = take(8 * (size_t)B.ckq * B.nck);
-  B.off_ckqp = take(4 * (size_t)B.ckq * B.nck);
+  B.off_ckmk = take(8 * (size_t)B.ckm * B.nck);
+  B.off_ckmd = take((size_t)B.ckm * B.nck);
+  B.off_ckbits = take(4 * (size_t)B.ckw * B.nck);
   B.off_slot = take((size_t)L.P.slot_bytes);
   B.total = off;
   return GMG_OK;
@@ -485,6 +536,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   put(L.off_ops, b.ops.data(), sizeof(OpRec) * b.ops.size());
   put(L.off_succ, b.succ.data(), 4 * b.succ.size());
   put(L.off_pred, b.pred.data(), 4 * b.pred.size());
+  put(L.off_sib, b.sib.data(), 4 * b.sib.size());
   put(L.off_cons, b.cons.data(), 4 * b.cons.size());
   put(L.off_roots, b.roots.data(), 8 * b.roots.size());
   put(L.off_cap, b.cap.data(), 8 * b.cap.size());
@@ -503,6 +555,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.ops = reinterpret_cast<const OpRec*>(w + L.off_ops);
   G.succ = reinterpret_cast<const uint32_t*>(w + L.off_succ);
   G.pred = reinterpret_cast<const uint32_t*>(w + L.off_pred);
+  G.psib = reinterpret_cast<const uint32_t*>(w + L.off_sib);
   G.cons = reinterpret_cast<const uint32_t*>(w + L.off_cons);
   G.root_keys = reinterpret_cast<const uint64_t*>(w + L.off_roots);
   G.cap = reinterpret_cast<const int64_t*>(w + L.off_cap);
@@ -517,6 +570,9 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.R = b.R;
   G.nroots = b.nroots;
   G.ib = b.ib;
+  G.tb = 1;
+  while (G.tb < 62 && (int64_t(1) << G.tb) <= b.time_bound) ++G.tb;
+  G.dev_key = (G.tb + G.ib + 2 + 8 <= 63) ? 1 : 0;
   G.uniform = b.uniform ? 1 : 0;
   gmg_info_t& I = g->info;
   std::memset(&I, 0, sizeof(I));
@@ -530,6 +586,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   I.uniform_links = G.uniform;
   I.time_bound = b.time_bound;
   g->queue_bound = b.queue_bound;
+  g->log_bound = b.log_bound;
   I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
   *out = g;
   return GMG_OK;
@@ -599,6 +656,7 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   D.row = w + B.off_row;
   D.rb = reinterpret_cast<int64_t*>(w + B.off_rb);
   D.fb = reinterpret_cast<int64_t*>(w + B.off_fb);
+  D.hb = reinterpret_cast<int64_t*>(w + B.off_hb);
   D.status = reinterpret_cast<int32_t*>(w + B.off_status);
   D.res_scalars = reinterpret_cast<int64_t*>(w + B.off_res);
   D.res_peak = reinterpret_cast<int64_t*>(w + B.off_peak);
@@ -608,15 +666,19 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   D.ck_dev = reinterpret_cast<int64_t*>(w + B.off_ckdev);
   D.ck_creq = reinterpret_cast<int64_t*>(w + B.off_ckcreq);
   D.ck_qkey = reinterpret_cast<uint64_t*>(w + B.off_ckqk);
-  D.ck_qpay = reinterpret_cast<uint32_t*>(w + B.off_ckqp);
+  D.ck_mkey = reinterpret_cast<uint64_t*>(w + B.off_ckmk);
+  D.ck_mdev = w + B.off_ckmd;
+  D.ck_bits = reinterpret_cast<uint32_t*>(w + B.off_ckbits);
   D.nck = B.nck;
   D.ckq = B.ckq;
+  D.ckm = B.ckm;
+  D.ck_words = B.ckw;
   D.ld = B.ld;
   D.stride_pops = B.stride;
   b->g = g;
   b->slot = w + B.off_slot;
-  b->qs = B.L.qs;
-  b->qcap = B.L.qcap;
+  b->qs = B.L.P.qs;
+  b->qcap = B.L.P.qcap;
   SimParams P = B.L.P;
   P.base = D;
   P.place = d_base_place;

@@ -3,40 +3,40 @@
 // One warp simulates one candidate placement (Algorithm 1 evaluates the
 // candidate partitions "in parallel"; here every warp of a persistent grid
 // takes candidates k = warp, warp + W, ...).  Inside a warp the simulation
-// is the event-driven loop of Sec. 3.3.3, restated as one ordered sweep over
-// packed 64-bit event keys (time, class, op):
+// is the event-driven loop of Sec. 3.3.3 restated as one ordered sweep:
 //
-//   READY(r_i, i)  op i's last input has arrived (Sec. 3.3.2 ready time);
-//                  popping it starts i on its accelerator at
-//                  s_i = max(r_i, accelerator free time): every queue runs its
-//                  ops in (ready time, id) order, one at a time (Sec. 3.3.2,
-//                  Sec. 3.5.1), which is exactly "an idle queue starts the
-//                  ready op with the earliest ready time".
-//   FREE(t, i)@e   a copy of i's output on accelerator e is released.
-//   ALLOC(t, i)@e  a copy of i's output is allocated on e (its own output at
-//                  s_i; a receive buffer at f_i, Recv before Send, Sec. 3.5.2).
+//   READY(r_i, i)  op i's last input has arrived (Sec. 3.3.2 ready time).
+//                  Taking READY keys in (r, id) order and starting each op
+//                  at s_i = max(r_i, accelerator free time) makes every queue
+//                  run its ops in (ready time, id) order, one at a time
+//                  (Sec. 3.3.2, Sec. 3.5.1) -- exactly "an idle queue starts
+//                  the ready op with the earliest ready time".
+//   FREE / ALLOC   HBM events of the copies of an op's output: the op's own
+//                  buffer at s_i, a receive buffer on every other accelerator
+//                  of a successor at f_i (Recv before Send, Sec. 3.5.2), each
+//                  released by its last listed consumer there (Sec. 3.3.2).
 //
-// Every key pushed while handling key k is larger than k (successors are
-// ready no earlier than f_i > r_i, memory events happen at >= s_i with a
-// larger class), so the queue is monotone and memory events come out in
-// (time, frees-before-allocs, op) order: live bytes, per-accelerator peaks and
-// the first capacity violation (Sec. 3.3.2 HBM residency, Sec. 3.4.2 OOM
-// discard) are tracked online, with no sort.
+// READY keys live in a warp-cooperative 32-ary min-heap: the 32 children of
+// a node are compared by the 32 lanes at once (one coalesced load, two
+// redux.sync), so a pop costs log32(size) warp steps.  Ops without
+// predecessors never enter it: their keys are pre-sorted on the host.
 //
-// The queue is a 32-ary min-heap whose 32 children of a node are examined by
-// the 32 lanes at once (one coalesced load + two redux.sync), so a pop costs
-// log32(size) warp steps.  Its first `qs` entries live in shared memory, the
-// rest in the warp's global scratch.  Ops without predecessors never enter
-// the heap: their READY keys are pre-sorted on the host and merged in.
+// HBM events are appended to a per-warp log in O(1).  Every event produced
+// while handling READY(r, .) happens at a time >= r, so once the next READY
+// key has time T, every logged event with time < T is final and no later
+// event can precede it.  Such events are drained in batches: extracted into
+// shared memory, bitonic-sorted by (time, frees before allocs, op), and
+// applied in order to the per-accelerator live bytes, which gives the peaks
+// and the first capacity violation (Sec. 3.4.2 OOM discard) exactly.
 //
 // Lanes also fan out over successor lists (readiness, transfer arrivals,
-// distinct receiving accelerators via __match_any_sync), predecessor lists
-// (ready-time maxima) and consumer lists (last-consumer releases).  With at
-// most 32 accelerators, lane d keeps accelerator d's free time, live bytes
-// and peak in registers.
+// distinct receiving accelerators via __match_any_sync) and predecessor
+// lists (ready-time maxima, last-consumer releases).  With at most 32
+// accelerators, lane d keeps accelerator d's free time, live bytes and peak
+// in registers.
 //
 // No wait in these kernels depends on another warp or block; the only loop
-// without a data-bounded trip count is the event loop, capped at
+// whose trip count is not bounded by the data is the event loop, capped at
 // g.max_iter iterations (status GMG_SIM_LOOP).
 
 #include <cuda_runtime.h>
@@ -66,6 +66,7 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
 }
 
 __device__ __forceinline__ unsigned lane_id() { return threadIdx.x & 31u; }
+__device__ __forceinline__ uint32_t lanes_below() { return (1u << lane_id()) - 1u; }
 
 // 16-byte pieces of an OpRec, loaded through the read-only path.
 __device__ __forceinline__ longlong2 op_durbytes(const OpRec* ops, uint32_t i) {
@@ -88,224 +89,200 @@ struct KeyCodec {
     return ((uint64_t)t << (ib + 2)) | ((uint64_t)cls << ib) | (uint64_t)op;
   }
   __device__ __forceinline__ int64_t time(uint64_t k) const { return (int64_t)(k >> (ib + 2)); }
+  __device__ __forceinline__ uint64_t time_floor(int64_t t) const { return (uint64_t)t << (ib + 2); }
   __device__ __forceinline__ uint32_t cls(uint64_t k) const { return (uint32_t)(k >> ib) & 3u; }
   __device__ __forceinline__ uint32_t op(uint64_t k) const { return (uint32_t)(k & mask); }
 };
 
 // ---------------------------------------------------------------------------
-// Warp-cooperative 32-ary min-heap.  All lanes call every method with the
-// same arguments; lane 0 performs the stores.
+// READY keys: warp-cooperative 32-ary min-heap.  Slots [0, qs) are in shared
+// memory (qs >= 33, so the root and its children always are), the rest in
+// the warp's global scratch.  All lanes call every method with the same
+// arguments; lane 0 performs the stores.
 // ---------------------------------------------------------------------------
-struct WarpHeap {
-  uint64_t* sk;  // shared: keys [qs]
-  uint32_t* sp;  // shared: payloads [qs]
-  uint64_t* gk;  // global spill: keys [cap - qs]
-  uint32_t* gp;  // global spill: payloads
+struct ReadyHeap {
+  uint64_t* sk;
+  uint64_t* gk;
   int qs, cap, size;
 
   __device__ __forceinline__ uint64_t* kp(int i) const { return i < qs ? sk + i : gk + (i - qs); }
-  __device__ __forceinline__ uint32_t* pp(int i) const { return i < qs ? sp + i : gp + (i - qs); }
+  __device__ __forceinline__ uint64_t top() const { return size > 0 ? sk[0] : kKeyMax; }
 
-  // Place (x, xp) at `pos` and move it down until its children are >= x.
-  __device__ void sift_down(int pos, uint64_t x, uint32_t xp) {
+  __device__ void sift_down(int pos, uint64_t x) {
     const unsigned lane = lane_id();
     while (true) {
       const int c0 = pos * 32 + 1;
       if (c0 >= size) break;
       const int idx = c0 + (int)lane;
-      const uint64_t ck = idx < size ? *kp(idx) : kKeyMax;
+      uint64_t ck = kKeyMax;
+      if (idx < size) ck = c0 == 1 ? sk[idx] : *kp(idx);
       const uint64_t m = warp_min_u64(ck);
       if (m >= x) break;
       const int src = __ffs(__ballot_sync(kFullMask, ck == m)) - 1;
-      uint32_t mp = 0;
-      if ((int)lane == src) mp = *pp(idx);
-      mp = __shfl_sync(kFullMask, mp, src);
-      if (lane == 0) {
-        *kp(pos) = m;
-        *pp(pos) = mp;
-      }
+      if (lane == 0) *kp(pos) = m;
       pos = c0 + src;
     }
-    if (lane == 0) {
-      *kp(pos) = x;
-      *pp(pos) = xp;
-    }
+    if (lane == 0) *kp(pos) = x;
     __syncwarp();
   }
 
-  // Remove the minimum (the caller has read it).
   __device__ void pop() {
     const int n = --size;
     if (n == 0) return;
     const uint64_t x = *kp(n);
-    const uint32_t xp = *pp(n);
-    sift_down(0, x, xp);
+    sift_down(0, x);
   }
 
-  __device__ bool push(uint64_t key, uint32_t pay) {
+  __device__ bool push(uint64_t key) {
     if (size >= cap) return false;
-    const unsigned lane = lane_id();
     int pos = size++;
     while (pos > 0) {
       const int par = (pos - 1) >> 5;
       const uint64_t pk = *kp(par);
       if (pk <= key) break;
-      const uint32_t ppay = *pp(par);
-      if (lane == 0) {
-        *kp(pos) = pk;
-        *pp(pos) = ppay;
-      }
+      if (lane_id() == 0) *kp(pos) = pk;
       pos = par;
     }
-    if (lane == 0) {
-      *kp(pos) = key;
-      *pp(pos) = pay;
-    }
+    if (lane_id() == 0) *kp(pos) = key;
     __syncwarp();
     return true;
   }
 
-  // Append without ordering (followed by heapify()).
-  __device__ bool append(uint64_t key, uint32_t pay) {
-    if (size >= cap) return false;
-    if (lane_id() == 0) {
-      *kp(size) = key;
-      *pp(size) = pay;
-    }
-    ++size;
-    __syncwarp();
-    return true;
-  }
-
-  // Floyd's bottom-up construction.
   __device__ void heapify() {
     if (size < 2) return;
     for (int pos = (size - 2) / 32; pos >= 0; --pos) {
       const uint64_t x = *kp(pos);
-      const uint32_t xp = *pp(pos);
       __syncwarp();
-      sift_down(pos, x, xp);
+      sift_down(pos, x);
     }
   }
 };
 
 // ---------------------------------------------------------------------------
-// Per-accelerator state: free time, live bytes, peak bytes.
+// HBM event log: unordered 8-byte entries -- (accelerator << ds) | key when
+// the accelerator id fits above the key, else the key with the accelerator
+// in a side byte array.  Slots [0, ms) are in shared memory, the rest in
+// global scratch.
+// ---------------------------------------------------------------------------
+struct MemLog {
+  uint64_t* sk;
+  uint8_t* sd;
+  uint64_t* gk;
+  uint8_t* gd;
+  int ms, cap, n;
+
+  __device__ __forceinline__ uint64_t* kp(int i) const { return i < ms ? sk + i : gk + (i - ms); }
+  __device__ __forceinline__ uint8_t* dp(int i) const { return i < ms ? sd + i : gd + (i - ms); }
+};
+
+// ---------------------------------------------------------------------------
+// Per-accelerator state.  Free times: with at most 32 accelerators lane d
+// holds accelerator d's in a register, else a shared array.  Live and peak
+// bytes: shared arrays (the drain updates them a batch at a time).
 // ---------------------------------------------------------------------------
 template <bool kReg>
-struct Devices;
-
-// D <= 32: lane d holds accelerator d in registers.
-template <>
-struct Devices<true> {
-  int64_t fr, lv, pk, cp;
+struct Devices {
+  int64_t fr_reg;
+  int64_t* fr;  // shared [D] (when !kReg)
+  int64_t* lv;  // shared [D]
+  int64_t* pk;  // shared [D]
   int D;
-  __device__ void setup(const DevGmg& g, int64_t* /*mem*/) {
+  __device__ void setup(const DevGmg& g, int64_t* sm) {
     D = g.D;
-    cp = lane_id() < (unsigned)D ? g.cap[lane_id()] : kI64Max;
+    fr = sm;
+    lv = sm + (kReg ? 0 : D);
+    pk = lv + D;
   }
   __device__ void reset(const DevGmg& g) {
     const unsigned l = lane_id();
-    fr = l < (unsigned)D ? g.avail0[l] : 0;
-    lv = l < (unsigned)D ? g.base[l] : 0;
-    pk = lv;
-  }
-  __device__ __forceinline__ int64_t get_free(int d) const { return __shfl_sync(kFullMask, fr, d); }
-  __device__ __forceinline__ void set_free(int d, int64_t v) {
-    if ((int)lane_id() == d) fr = v;
-  }
-  __device__ __forceinline__ bool alloc(int d, int64_t b) {
-    bool over = false;
-    if ((int)lane_id() == d) {
-      lv += b;
-      pk = lv > pk ? lv : pk;
-      over = lv > cp;
-    }
-    return __ballot_sync(kFullMask, over) != 0;
-  }
-  __device__ __forceinline__ void release(int d, int64_t b) {
-    if ((int)lane_id() == d) lv -= b;
-  }
-  __device__ void save(int64_t* dst) const {
-    const unsigned l = lane_id();
-    if (l < (unsigned)D) {
-      dst[l] = fr;
-      dst[D + l] = lv;
-      dst[2 * D + l] = pk;
-    }
-  }
-  __device__ void load(const int64_t* src) {
-    const unsigned l = lane_id();
-    if (l < (unsigned)D) {
-      fr = src[l];
-      lv = src[D + l];
-      pk = src[2 * D + l];
-    }
-  }
-  __device__ void write_peak(int64_t* dst) const {
-    if (lane_id() < (unsigned)D) dst[lane_id()] = pk;
-  }
-};
-
-// Any D: arrays in the warp's scratch; all lanes read, lane 0 writes.
-template <>
-struct Devices<false> {
-  int64_t* fr;
-  int64_t* lv;
-  int64_t* pk;
-  const int64_t* cp;
-  int D;
-  __device__ void setup(const DevGmg& g, int64_t* mem) {
-    D = g.D;
-    fr = mem;
-    lv = mem + D;
-    pk = mem + 2 * D;
-    cp = g.cap;
-  }
-  __device__ void reset(const DevGmg& g) {
-    for (int d = lane_id(); d < D; d += 32) {
-      fr[d] = g.avail0[d];
+    for (int d = l; d < D; d += 32) {
       lv[d] = g.base[d];
       pk[d] = g.base[d];
+      if (!kReg) fr[d] = g.avail0[d];
     }
+    if (kReg) fr_reg = l < (unsigned)D ? g.avail0[l] : 0;
     __syncwarp();
   }
-  __device__ __forceinline__ int64_t get_free(int d) const { return fr[d]; }
-  __device__ __forceinline__ void set_free(int d, int64_t v) {
-    if (lane_id() == 0) fr[d] = v;
+  __device__ __forceinline__ int64_t get_free(int d) const {
+    if (kReg) return __shfl_sync(kFullMask, fr_reg, d);
+    return fr[d];
   }
-  __device__ __forceinline__ bool alloc(int d, int64_t b) {
+  __device__ __forceinline__ void set_free(int d, int64_t v) {
+    if (kReg) {
+      if ((int)lane_id() == d) fr_reg = v;
+    } else {
+      __syncwarp();
+      if (lane_id() == 0) fr[d] = v;
+    }
+  }
+  // One event at a time (used when accelerator ids do not fit in the sort key).
+  __device__ __forceinline__ bool alloc(int d, int64_t b, int64_t cap) {
     const int64_t v = lv[d] + b;
     const int64_t p = pk[d];
+    __syncwarp();
     if (lane_id() == 0) {
       lv[d] = v;
       if (v > p) pk[d] = v;
     }
-    return v > __ldg(cp + d);
+    __syncwarp();
+    return v > cap;
   }
   __device__ __forceinline__ void release(int d, int64_t b) {
     const int64_t v = lv[d] - b;
+    __syncwarp();
     if (lane_id() == 0) lv[d] = v;
+    __syncwarp();
   }
   __device__ void save(int64_t* dst) const {
-    for (int d = lane_id(); d < D; d += 32) {
-      dst[d] = fr[d];
+    const unsigned l = lane_id();
+    for (int d = l; d < D; d += 32) {
+      if (!kReg) dst[d] = fr[d];
       dst[D + d] = lv[d];
       dst[2 * D + d] = pk[d];
     }
+    if (kReg && l < (unsigned)D) dst[l] = fr_reg;
   }
   __device__ void load(const int64_t* src) {
-    for (int d = lane_id(); d < D; d += 32) {
-      fr[d] = src[d];
+    const unsigned l = lane_id();
+    for (int d = l; d < D; d += 32) {
+      if (!kReg) fr[d] = src[d];
       lv[d] = src[D + d];
       pk[d] = src[2 * D + d];
     }
+    if (kReg) fr_reg = l < (unsigned)D ? src[l] : 0;
     __syncwarp();
   }
   __device__ void write_peak(int64_t* dst) const {
     for (int d = lane_id(); d < D; d += 32) dst[d] = pk[d];
   }
 };
+
+// Shared-memory carve-up per warp: READY heap head, event-log head, sort
+// area, accelerator state.
+struct WarpSmem {
+  uint64_t* heap;   // [qs]
+  uint64_t* logk;   // [ms]
+  uint64_t* sortk;  // [sortcap]
+  uint8_t* logd;    // [ms]
+  uint8_t* sortd;   // [sortcap]
+  int64_t* dev;     // [3*D] (2*D used when free times are in registers)
+};
+
+__device__ __forceinline__ size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
+
+__device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P, unsigned wib) {
+  const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9);
+  const size_t per = head + (size_t)P.g.D * 24;
+  uint8_t* b = smem + per * wib;
+  WarpSmem w;
+  w.heap = reinterpret_cast<uint64_t*>(b);
+  w.logk = w.heap + P.qs;
+  w.sortk = w.logk + P.ms;
+  w.logd = reinterpret_cast<uint8_t*>(w.sortk + P.sortcap);
+  w.sortd = w.logd + P.ms;
+  w.dev = reinterpret_cast<int64_t*>(b + head);
+  return w;
+}
 
 // ---------------------------------------------------------------------------
 // One warp's simulator.
@@ -315,19 +292,25 @@ struct Sim {
   const SimParams& P;
   const DevGmg& g;
   KeyCodec kc;
-  WarpHeap q;
+  ReadyHeap q;
+  MemLog log;
+  uint64_t* sortk;
+  uint8_t* sortd;
+  int sortcap;
+  int ds;           // accelerator shift of a log entry
+  uint64_t lowmask; // key part of a log entry
   Devices<kReg> dv;
   const uint8_t* row;
   int64_t* fbuf;
+  int64_t* hold;
   uint32_t* bits;
   int64_t* creq;
   // incremental resume
   const int64_t* rb;
   const int64_t* fb;
-  const uint8_t* brow;
   int64_t Tc, T0;
   // running results
-  int rootptr;
+  int rootptr, trig;
   int64_t score, makespan, iters, nev, readypops, last_t;
   int32_t vflag, vop, vdev, status;
   int64_t vt;
@@ -337,27 +320,24 @@ struct Sim {
   __device__ Sim(const SimParams& p) : P(p), g(p.g) {
     kc.ib = g.ib;
     kc.mask = (1ull << g.ib) - 1ull;
+    ds = g.ib + 2 + g.tb;
+    lowmask = g.dev_key ? (1ull << ds) - 1ull : kKeyMax;
   }
 
-  __device__ __forceinline__ bool bit(uint32_t x) const { return (bits[x >> 5] >> (x & 31u)) & 1u; }
-
-  // Has op x been simulated (is its finish time known)?
-  __device__ __forceinline__ bool popped(uint32_t x) const {
-    if (kMode == kInc) return bit(x) || rb[x] < Tc;
-    return bit(x);
-  }
+  __device__ __forceinline__ bool popped(uint32_t x) const { return (bits[x >> 5] >> (x & 31u)) & 1u; }
+  // Finish time of a simulated op (incremental: ops before the resume point
+  // keep their base finish).
   __device__ __forceinline__ int64_t fin(uint32_t x) const {
-    if (kMode == kInc && !bit(x)) return fb[x];
+    if (kMode == kInc && rb[x] < Tc) return fb[x];
     return fbuf[x];
   }
 
   // Transfer estimator of one output over link d -> e (d != e), Sec. 3.3.1.
   __device__ __forceinline__ int64_t xfer(int d, int e, int64_t bytes, int64_t xq) const {
     if (g.uniform) return xq + g.lat0;
-    const LinkRec* L = g.links + (d * g.D + e);
+    const longlong2* L = reinterpret_cast<const longlong2*>(g.links + (d * g.D + e));
+    const longlong2 a = __ldg(L), b = __ldg(L + 1);
     LinkRec l;
-    const longlong2 a = __ldg(reinterpret_cast<const longlong2*>(L));
-    const longlong2 b = __ldg(reinterpret_cast<const longlong2*>(L) + 1);
     l.magic = (uint64_t)a.x;
     l.bw = a.y;
     l.lat = b.x;
@@ -365,26 +345,54 @@ struct Sim {
     return ceil_div_link(bytes, l) + l.lat;
   }
 
-  __device__ __forceinline__ void push(uint64_t key, uint32_t pay) {
-    if (status) return;
-    if (!q.push(key, pay)) status = GMG_SIM_QUEUE;
+  // Latest arrival of p's output at another accelerator (or f_p): the
+  // earliest its source copy may be released.  Per lane.
+  __device__ int64_t lane_hold(uint32_t p, int64_t fp, int dp) const {
+    const int64_t pb = op_durbytes(g.ops, p).y;
+    const int64_t pxq = op_relxq(g.ops, p).y;
+    const uint4 ls = op_lists(g.ops, p);
+    int64_t h = fp;
+    for (uint32_t u = 0; u < ls.y; ++u) {
+      const int du = row[__ldg(g.succ + ls.x + u)];
+      if (du != dp) {
+        const int64_t a = fp + xfer(dp, du, pb, pxq);
+        h = a > h ? a : h;
+      }
+    }
+    return h;
   }
-  __device__ __forceinline__ void append(uint64_t key, uint32_t pay) {
-    if (status) return;
-    if (!q.append(key, pay)) status = GMG_SIM_QUEUE;
+  __device__ __forceinline__ int64_t hold_of(uint32_t p, int dp) const {
+    if (kMode == kInc && rb[p] < Tc) return lane_hold(p, fb[p], dp);
+    return hold[p];
   }
 
-  // Push (key, pay) of every lane in `mask`, in lane order.
-  template <bool kAppend>
-  __device__ __forceinline__ void push_lanes(uint32_t mask, uint64_t key, uint32_t pay) {
-    while (mask) {
-      const int src = __ffs(mask) - 1;
-      mask &= mask - 1;
-      const uint64_t k = __shfl_sync(kFullMask, key, src);
-      const uint32_t p = __shfl_sync(kFullMask, pay, src);
-      if (kAppend) append(k, p);
-      else push(k, p);
+  __device__ __forceinline__ void push_ready(uint64_t key) {
+    if (status) return;
+    if (!q.push(key)) status = GMG_SIM_QUEUE;
+  }
+  // Every lane with `want` logs (key, dev).  Uniform call.
+  __device__ __forceinline__ void log_event(bool want, uint64_t key, int dev) {
+    const uint32_t b = __ballot_sync(kFullMask, want);
+    if (b == 0u || status) return;
+    const int cnt = __popc(b);
+    const int pos = log.n + __popc(b & lanes_below());
+    const uint64_t e = g.dev_key ? (((uint64_t)(dev & 0xff) << ds) | key) : key;
+    if (log.n + cnt <= log.ms) {
+      if (want) {
+        log.sk[pos] = e;
+        if (!g.dev_key) log.sd[pos] = (uint8_t)dev;
+      }
+    } else {
+      if (log.n + cnt > log.cap) {
+        status = GMG_SIM_QUEUE;
+        return;
+      }
+      if (want) {
+        *log.kp(pos) = e;
+        if (!g.dev_key) *log.dp(pos) = (uint8_t)dev;
+      }
     }
+    log.n += cnt;
   }
 
   __device__ void reset_common() {
@@ -394,6 +402,8 @@ struct Sim {
     for (int r = lane; r < g.R; r += 32) creq[r] = 0;
     dv.reset(g);
     q.size = 0;
+    log.n = 0;
+    trig = P.drain_trigger;
     rootptr = 0;
     score = makespan = 0;
     iters = nev = readypops = 0;
@@ -416,7 +426,7 @@ struct Sim {
     const uint4 cs = op_cons(g.ops, i);
     const int64_t dur = db.x, bytes = db.y, xq = rx.y;
     const uint32_t succ_off = ls.x, nsucc = ls.y, pred_off = ls.z, npred = ls.w;
-    const uint32_t cons_off = cs.x, ncons = cs.y, flags = cs.w;
+    const uint32_t flags = cs.w;
     const int d = row[i];
     const int64_t fd = dv.get_free(d);
     const int64_t s = r > fd ? r : fd;
@@ -433,13 +443,12 @@ struct Sim {
     makespan = f > makespan ? f : makespan;
     if (kMode != kInc || r >= T0) ++nev;
     ++readypops;
+    // the op's own output is allocated when it starts
+    log_event(lane == 0, kc.make(s, kAlloc, i), d);
     __syncwarp();
 
-    // The op's own output is allocated when it starts.
-    push(kc.make(s, kAlloc, i), (uint32_t)d);
-
     // Successors: transfers, readiness, receive copies.
-    int64_t hold = f;   // latest arrival of an outgoing transfer (or f)
+    int64_t hm = f;  // latest arrival of an outgoing transfer (or f)
     bool local_succ = false;
     for (uint32_t c0 = 0; c0 < nsucc; c0 += 32) {
       const uint32_t t = c0 + lane;
@@ -456,9 +465,9 @@ struct Sim {
         const uint4 jls = op_lists(g.ops, j);
         rj = jrx.x > arr ? jrx.x : arr;
         rdy = true;
+        // ready once every other predecessor has finished; its ready time is
+        // the latest arrival over all of them
         if (jls.w > 1) {
-          // Ready only when every other predecessor has finished; its ready
-          // time is the latest arrival over all of them.
           for (uint32_t k = 0; k < jls.w; ++k) {
             const uint32_t p = __ldg(g.pred + jls.z + k) & kIdMask;
             if (p == i) continue;
@@ -468,16 +477,17 @@ struct Sim {
             }
             const int dp = row[p];
             int64_t a = fin(p);
-            if (dp != dj) {
-              const longlong2 pdb = op_durbytes(g.ops, p);
-              a += xfer(dp, dj, pdb.y, op_relxq(g.ops, p).y);
-            }
+            if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
             rj = a > rj ? a : rj;
           }
         }
       }
-      push_lanes<false>(__ballot_sync(kFullMask, rdy), kc.make(rj, kReady, j), 0u);
-
+      uint32_t m = __ballot_sync(kFullMask, rdy);
+      while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        push_ready(__shfl_sync(kFullMask, kc.make(rj, kReady, j), src));
+      }
       const bool rem = v && dj != d;
       local_succ |= __any_sync(kFullMask, v && dj == d);
       const uint32_t peers = __match_any_sync(kFullMask, rem ? (uint32_t)dj : (256u + lane));
@@ -489,96 +499,289 @@ struct Sim {
             break;
           }
       }
-      const uint64_t hm = warp_max_u64(leader ? (uint64_t)arr : 0ull);
-      hold = (int64_t)hm > hold ? (int64_t)hm : hold;
-      // One receive copy per distinct remote accelerator, allocated when the
-      // transfer starts.
-      const uint32_t lead_mask = __ballot_sync(kFullMask, leader);
-      push_lanes<false>(lead_mask, kc.make(f, kAlloc, i), (uint32_t)dj);
+      const int64_t hl = (int64_t)warp_max_u64(leader ? (uint64_t)arr : 0ull);
+      hm = hl > hm ? hl : hm;
+      // one receive copy per distinct remote accelerator, allocated when the
+      // transfer starts
+      log_event(leader, kc.make(f, kAlloc, i), dj);
       if (!(flags & kAllCons)) {
-        // A receive copy with no listed consumer there is released on arrival.
+        // a receive copy with no listed consumer there is released on arrival
         bool nocons = false;
         if (leader) {
           nocons = true;
-          for (uint32_t u = 0; u < ncons; ++u)
-            if (row[__ldg(g.cons + cons_off + u)] == dj) {
+          for (uint32_t u = 0; u < cs.y; ++u)
+            if (row[__ldg(g.cons + cs.x + u)] == dj) {
               nocons = false;
               break;
             }
         }
-        push_lanes<false>(__ballot_sync(kFullMask, nocons), kc.make(arr, kFree, i), (uint32_t)dj);
+        log_event(nocons, kc.make(arr, kFree, i), dj);
       }
     }
-    // The source copy: released by its last local consumer, or now-known.
+    // The source copy: released now-known if no listed consumer is local,
+    // else by its last local consumer (which reads hold[i]).
     bool local_cons = local_succ;
     if (!(flags & kAllCons)) {
       bool lc = false;
-      for (uint32_t c0 = 0; c0 < ncons; c0 += 32) {
+      for (uint32_t c0 = 0; c0 < cs.y; c0 += 32) {
         const uint32_t t = c0 + lane;
-        if (t < ncons && row[__ldg(g.cons + cons_off + t)] == d) lc = true;
+        if (t < cs.y && row[__ldg(g.cons + cs.x + t)] == d) lc = true;
       }
       local_cons = __any_sync(kFullMask, lc);
     }
-    if (!local_cons) push(kc.make(hold, kFree, i), (uint32_t)d);
+    if (local_cons) {
+      if (lane == 0) hold[i] = hm;
+    } else {
+      log_event(lane == 0, kc.make(hm, kFree, i), d);
+    }
 
-    // Inputs this op holds: if it is the last listed consumer of a
+    // Inputs held by this op: if it is the last listed consumer of a
     // predecessor's output on this accelerator, that copy is released at f
-    // (the source copy also waits for the predecessor's outgoing arrivals).
-    for (uint32_t k = 0; k < npred; ++k) {
-      const uint32_t pe = __ldg(g.pred + pred_off + k);
-      if (!(pe & kHoldBit)) continue;
-      const uint32_t p = pe & kIdMask;
-      const uint4 pls = op_lists(g.ops, p);
-      const uint4 pcs = op_cons(g.ops, p);
-      const bool all = (pcs.w & kAllCons) != 0;
-      const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
-      const uint32_t nl = all ? pls.y : pcs.y;
-      bool pending = false;
-      for (uint32_t c0 = 0; c0 < nl; c0 += 32) {
-        const uint32_t t = c0 + lane;
-        if (t < nl) {
-          const uint32_t c = __ldg(lst + t);
-          if (c != i && row[c] == d && !popped(c)) pending = true;
-        }
-      }
-      if (__any_sync(kFullMask, pending)) continue;
-      const int dp = row[p];
+    // (the source copy not before the predecessor's transfers arrived).
+    for (uint32_t c0 = 0; c0 < npred; c0 += 32) {
+      const uint32_t t = c0 + lane;
+      bool rel = false;
       int64_t T = f;
-      if (dp == d) {
-        const int64_t fp = fin(p);
-        const int64_t pb = op_durbytes(g.ops, p).y;
-        const int64_t pxq = op_relxq(g.ops, p).y;
-        uint64_t mx = 0;
-        for (uint32_t c0 = 0; c0 < pls.y; c0 += 32) {
-          const uint32_t t = c0 + lane;
-          if (t < pls.y) {
-            const int du = row[__ldg(g.succ + pls.x + t)];
-            if (du != dp) {
-              const uint64_t a = (uint64_t)(fp + xfer(dp, du, pb, pxq));
-              mx = a > mx ? a : mx;
+      uint32_t p = 0;
+      if (t < npred) {
+        const uint32_t pe = __ldg(g.pred + pred_off + t);
+        p = pe & kIdMask;
+        if (pe & kHoldBit) {
+          const uint32_t sb = __ldg(g.psib + pred_off + t);
+          if (sb == kSibNone) {
+            rel = true;
+          } else if (sb != kSibMany) {
+            rel = !(row[sb] == d && !popped(sb));
+          } else {
+            const uint4 pls = op_lists(g.ops, p);
+            const uint4 pcs = op_cons(g.ops, p);
+            const bool all = (pcs.w & kAllCons) != 0;
+            const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
+            const uint32_t nl = all ? pls.y : pcs.y;
+            rel = true;
+            for (uint32_t u = 0; u < nl; ++u) {
+              const uint32_t c = __ldg(lst + u);
+              if (c != i && row[c] == d && !popped(c)) {
+                rel = false;
+                break;
+              }
+            }
+          }
+          if (rel) {
+            const int dp = row[p];
+            if (dp == d) {
+              const int64_t h = hold_of(p, dp);
+              T = h > T ? h : T;
             }
           }
         }
-        const int64_t m = (int64_t)warp_max_u64(mx);
-        T = m > T ? m : T;
       }
-      push(kc.make(T, kFree, p), (uint32_t)d);
+      log_event(rel, kc.make(T, kFree, p), d);
+    }
+    __syncwarp();
+  }
+
+  // Apply sorted events one at a time (accelerator ids not in the key).
+  __device__ void apply_serial(int m) {
+    for (int e = 0; e < m; ++e) {
+      const uint64_t k = sortk[e];
+      const int dev = sortd[e];
+      const uint32_t op = kc.op(k);
+      const int64_t b = op_durbytes(g.ops, op).y;
+      if (kc.cls(k) == kFree) {
+        dv.release(dev, b);
+      } else if (dv.alloc(dev, b, __ldg(g.cap + dev))) {
+        const int64_t t = kc.time(k);
+        if (!vflag || (t == vt && (int32_t)op == vop && dev < vdev)) {
+          vflag = 1;
+          vt = t;
+          vop = (int32_t)op;
+          vdev = dev;
+        }
+      }
+    }
+    __syncwarp();
+  }
+
+  // Apply events sorted by (accelerator, time, class, op), 32 at a time:
+  // each accelerator's events are contiguous, so a segmented warp scan of
+  // the byte deltas gives the live bytes after every event, a segmented max
+  // scan the peak, and a warp min the first capacity violation.
+  __device__ void apply_segmented(int m) {
+    const unsigned lane = lane_id();
+    const int ds = g.ib + 2 + g.tb;
+    const uint64_t tmask = (1ull << g.tb) - 1ull;
+    uint64_t vmin = kKeyMax;
+    for (int c0 = 0; c0 < m; c0 += 32) {
+      const int idx = c0 + (int)lane;
+      const bool v = idx < m;
+      const uint64_t key = v ? sortk[idx] : 0ull;
+      const int dev = v ? (int)(key >> ds) : -1 - (int)lane;
+      const uint32_t op = (uint32_t)(key & kc.mask);
+      const bool isalloc = v && kc.cls(key) == kAlloc;
+      int64_t delta = 0;
+      if (v) {
+        const int64_t b = op_durbytes(g.ops, op).y;
+        delta = isalloc ? b : -b;
+      }
+      int64_t s = delta;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int64_t o = __shfl_up_sync(kFullMask, s, off);
+        const int od = __shfl_up_sync(kFullMask, dev, off);
+        if ((int)lane >= off && od == dev) s += o;
+      }
+      const int64_t live = (v ? dv.lv[dev] : 0) + s;
+      int64_t pm = isalloc ? live : INT64_MIN;
+#pragma unroll
+      for (int off = 1; off < 32; off <<= 1) {
+        const int64_t o = __shfl_up_sync(kFullMask, pm, off);
+        const int od = __shfl_up_sync(kFullMask, dev, off);
+        if ((int)lane >= off && od == dev && o > pm) pm = o;
+      }
+      const int nd = __shfl_down_sync(kFullMask, dev, 1);
+      const bool last = v && (lane == 31 || nd != dev);
+      const bool over = isalloc && live > __ldg(g.cap + dev);
+      const uint64_t vk = over ? ((((key >> (g.ib + 2)) & tmask) << (g.ib + 8)) | ((uint64_t)op << 8) |
+                                  (uint64_t)dev)
+                               : kKeyMax;
+      const uint64_t cm = warp_min_u64(vk);
+      vmin = cm < vmin ? cm : vmin;
+      __syncwarp();
+      if (last) {
+        dv.lv[dev] = live;
+        if (pm > dv.pk[dev]) dv.pk[dev] = pm;
+      }
+      __syncwarp();
+    }
+    // every event of this drain is later than every event already applied,
+    // so an earlier violation stands
+    if (!vflag && vmin != kKeyMax) {
+      vflag = 1;
+      vt = (int64_t)(vmin >> (g.ib + 8));
+      vop = (int32_t)((vmin >> 8) & kc.mask);
+      vdev = (int32_t)(vmin & 0xffu);
     }
   }
 
-  __device__ __forceinline__ void mem_event(uint32_t cls, uint32_t op, int64_t t, uint32_t pay) {
-    const int e = (int)(pay & 0xffu);
-    const int64_t b = op_durbytes(g.ops, op).y;
-    if (cls == kFree) {
-      dv.release(e, b);
-    } else if (dv.alloc(e, b)) {
-      if (!vflag || (t == vt && (int32_t)op == vop && e < vdev)) {
-        vflag = 1;
-        vt = t;
-        vop = (int32_t)op;
-        vdev = e;
+  __device__ int count_below(uint64_t kmax) const {
+    int c = 0;
+    for (int c0 = 0; c0 < log.n; c0 += 32) {
+      const int idx = c0 + (int)lane_id();
+      const bool take = idx < log.n && (*log.kp(idx) & lowmask) < kmax;
+      c += __popc(__ballot_sync(kFullMask, take));
+    }
+    return c;
+  }
+
+  // Move the logged events whose key part is < kmax to the sort area (their
+  // number is known to fit) and compact the rest; returns their number.
+  __device__ int extract(uint64_t kmax) {
+    const unsigned lane = lane_id();
+    const bool side = !g.dev_key;
+    int m = 0, keep = 0;
+    const int n = log.n;
+    for (int c0 = 0; c0 < n; c0 += 32) {
+      const int idx = c0 + (int)lane;
+      const bool v = idx < n;
+      uint64_t e = kKeyMax;
+      uint8_t dv8 = 0;
+      if (v) {
+        if (idx < log.ms) {
+          e = log.sk[idx];
+          if (side) dv8 = log.sd[idx];
+        } else {
+          e = *log.kp(idx);
+          if (side) dv8 = *log.dp(idx);
+        }
+      }
+      const bool take = v && (e & lowmask) < kmax;
+      const uint32_t bt = __ballot_sync(kFullMask, take);
+      const uint32_t bk = __ballot_sync(kFullMask, v && !take);
+      if (take) {
+        const int pos = m + __popc(bt & lanes_below());
+        sortk[pos] = e;
+        if (side) sortd[pos] = dv8;
+      } else if (v) {
+        const int pos = keep + __popc(bk & lanes_below());  // pos <= idx: in place
+        *log.kp(pos) = e;
+        if (side) *log.dp(pos) = dv8;
+      }
+      m += __popc(bt);
+      keep += __popc(bk);
+      __syncwarp();
+    }
+    log.n = keep;
+    return m;
+  }
+
+  // Bitonic sort of sortk[0, m) (and the side bytes alongside), padded to a
+  // power of two >= 32.
+  __device__ void sort_area(int m) {
+    const unsigned lane = lane_id();
+    const bool side = !g.dev_key;
+    int p2 = 32;
+    while (p2 < m) p2 <<= 1;
+    for (int x = m + (int)lane; x < p2; x += 32) sortk[x] = kKeyMax;
+    __syncwarp();
+    for (int k = 2; k <= p2; k <<= 1) {
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        for (int t = lane; t < (p2 >> 1); t += 32) {
+          const int i = ((t & ~(j - 1)) << 1) | (t & (j - 1));
+          const int l = i + j;
+          const uint64_t a = sortk[i], b = sortk[l];
+          const bool asc = (i & k) == 0;
+          if ((a > b) == asc) {
+            sortk[i] = b;
+            sortk[l] = a;
+            if (side) {
+              const uint8_t da = sortd[i], db = sortd[l];
+              sortd[i] = db;
+              sortd[l] = da;
+            }
+          }
+        }
+        __syncwarp();
       }
     }
+  }
+
+  // Apply every logged event that can no longer be preceded (time < t_next).
+  __device__ void drain(int64_t t_next) {
+    const uint64_t lim = t_next == kI64Max ? kKeyMax : kc.time_floor(t_next);
+    while (log.n > 0) {
+      uint64_t kmax = lim;
+      if (log.n > sortcap) {
+        const int due = count_below(lim);
+        if (due == 0) break;
+        if (due > sortcap) {
+          // Rare: more due events than the sort area.  Bisect a key bound
+          // with at most sortcap events below it (at most n_dev <= sortcap
+          // events share a key part).
+          uint64_t lo = kKeyMax;
+          for (int c0 = 0; c0 < log.n; c0 += 32) {
+            const int idx = c0 + (int)lane_id();
+            const uint64_t kk = idx < log.n ? (*log.kp(idx) & lowmask) : kKeyMax;
+            lo = kk < lo ? kk : lo;
+          }
+          lo = warp_min_u64(lo) + 1;  // 1 <= count_below(lo) <= sortcap
+          uint64_t hi = lim;          // count_below(hi) > sortcap
+          while (hi - lo > 1) {
+            const uint64_t mid = lo + (hi - lo) / 2;
+            if (count_below(mid) <= sortcap) lo = mid;
+            else hi = mid;
+          }
+          kmax = lo;
+        }
+      }
+      const int m = extract(kmax);
+      if (m == 0) break;
+      sort_area(m);
+      if (g.dev_key) apply_segmented(m);
+      else apply_serial(m);
+      if (kmax == lim) break;
+    }
+    trig = log.n + P.drain_trigger;
   }
 
   __device__ void maybe_checkpoint(uint64_t next_key);
@@ -587,34 +790,28 @@ struct Sim {
   __device__ void run() {
     if (status) return;
     while (true) {
-      const uint64_t top = q.size > 0 ? *q.kp(0) : kKeyMax;
+      const uint64_t top = q.top();
       const uint64_t rk = rootptr < g.nroots ? __ldg(g.root_keys + rootptr) : kKeyMax;
-      if (kMode == kBase) maybe_checkpoint(rk < top ? rk : top);
-      uint64_t key;
-      uint32_t pay = 0;
+      const uint64_t nk = rk < top ? rk : top;
+      if (kMode == kBase) maybe_checkpoint(nk);
+      if (nk == kKeyMax) break;
+      if (log.n >= trig) drain(kc.time(nk));
       if (rk < top) {
-        key = rk;
         ++rootptr;
-      } else if (top != kKeyMax) {
-        key = top;
-        pay = *q.pp(0);
+      } else {
         __syncwarp();
         q.pop();
-      } else {
-        break;
       }
       if (++iters > g.max_iter) {
         status = GMG_SIM_LOOP;
         break;
       }
-      const uint32_t cls = kc.cls(key), op = kc.op(key);
-      const int64_t t = kc.time(key);
+      const int64_t t = kc.time(nk);
       last_t = t;
-      if (cls == kReady) start_op(op, t);
-      else mem_event(cls, op, t, pay);
-      __syncwarp();
+      start_op(kc.op(nk), t);
       if (status) break;
     }
+    if (!status) drain(kI64Max);
   }
 
   __device__ void write_invalid(int64_t k, int32_t st) {
@@ -643,6 +840,7 @@ struct Sim {
   }
 
   __device__ int trace_slot(int64_t k) const {
+    if (P.n_trace == 0) return -1;
     int ts = -1;
     for (int t = lane_id(); t < P.n_trace; t += 32)
       if (P.trace_k[t] == k) ts = t;
@@ -709,8 +907,9 @@ struct Sim {
 };
 
 // Base-mode checkpoint: at a time boundary (nothing at the next key's time
-// processed yet), save the complete simulator state; an incremental
-// candidate whose resume time T0 is >= that time may restart from it.
+// handled yet), save the complete simulator state -- simulated-op bitmap,
+// accelerator state, READY heap, event log, partial results.  An
+// incremental candidate whose resume time T0 is >= that time restarts there.
 template <bool kReg, int kMode>
 __device__ void Sim<kReg, kMode>::maybe_checkpoint(uint64_t next_key) {
   if (kMode != kBase) return;
@@ -719,7 +918,7 @@ __device__ void Sim<kReg, kMode>::maybe_checkpoint(uint64_t next_key) {
   const int64_t tn = kc.time(next_key);
   if (tn <= last_t) return;
   const unsigned lane = lane_id();
-  if (q.size <= B.ckq) {
+  if (q.size <= B.ckq && log.n <= B.ckm) {
     int64_t* sc = B.ck_scalars + (int64_t)ck * 8;
     if (lane == 0) {
       B.ck_time[ck] = tn;
@@ -729,15 +928,18 @@ __device__ void Sim<kReg, kMode>::maybe_checkpoint(uint64_t next_key) {
       sc[3] = makespan;
       sc[4] = vflag;
       sc[5] = vt;
-      sc[6] = vop;
-      sc[7] = vdev;
+      sc[6] = ((int64_t)vop << 32) | (uint32_t)vdev;
+      sc[7] = log.n;
     }
     dv.save(B.ck_dev + (int64_t)ck * 3 * g.D);
     for (int r = lane; r < g.R; r += 32) B.ck_creq[(int64_t)ck * g.R + r] = creq[r];
-    for (int x = lane; x < q.size; x += 32) {
-      B.ck_qkey[(int64_t)ck * B.ckq + x] = *q.kp(x);
-      B.ck_qpay[(int64_t)ck * B.ckq + x] = *q.pp(x);
+    for (int x = lane; x < q.size; x += 32) B.ck_qkey[(int64_t)ck * B.ckq + x] = *q.kp(x);
+    for (int x = lane; x < log.n; x += 32) {
+      B.ck_mkey[(int64_t)ck * B.ckm + x] = *log.kp(x);
+      B.ck_mdev[(int64_t)ck * B.ckm + x] = *log.dp(x);
     }
+    const int words = (g.n + 31) >> 5;
+    for (int w = lane; w < words; w += 32) B.ck_bits[(int64_t)ck * B.ck_words + w] = bits[w];
   } else if (lane == 0) {
     B.ck_time[ck] = kI64Max;
   }
@@ -747,21 +949,30 @@ __device__ void Sim<kReg, kMode>::maybe_checkpoint(uint64_t next_key) {
 }
 
 template <bool kReg, int kMode>
-__device__ void setup_slot(Sim<kReg, kMode>& S, const SimParams& P, unsigned warp_in_block,
-                           int64_t slot, uint8_t* smem) {
+__device__ void setup_slot(Sim<kReg, kMode>& S, const SimParams& P, unsigned wib, int64_t slot,
+                           uint8_t* smem) {
   uint8_t* sl = P.scratch + slot * P.slot_bytes;
-  S.q.sk = reinterpret_cast<uint64_t*>(smem) + (int64_t)warp_in_block * P.qs;
-  S.q.sp = reinterpret_cast<uint32_t*>(smem + (size_t)blockDim.x / 32 * P.qs * 8) +
-           (int64_t)warp_in_block * P.qs;
+  const WarpSmem w = carve_smem(smem, P, wib);
+  S.q.sk = w.heap;
   S.q.gk = reinterpret_cast<uint64_t*>(sl + P.off_qk);
-  S.q.gp = reinterpret_cast<uint32_t*>(sl + P.off_qp);
   S.q.qs = P.qs;
   S.q.cap = P.qcap;
   S.q.size = 0;
+  S.log.sk = w.logk;
+  S.log.sd = w.logd;
+  S.log.gk = reinterpret_cast<uint64_t*>(sl + P.off_mk);
+  S.log.gd = sl + P.off_md;
+  S.log.ms = P.ms;
+  S.log.cap = P.mcap;
+  S.log.n = 0;
+  S.sortk = w.sortk;
+  S.sortd = w.sortd;
+  S.sortcap = P.sortcap;
   S.fbuf = reinterpret_cast<int64_t*>(sl + P.off_f);
+  S.hold = reinterpret_cast<int64_t*>(sl + P.off_hold);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
   S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
-  S.dv.setup(P.g, reinterpret_cast<int64_t*>(sl + P.off_dev));
+  S.dv.setup(P.g, w.dev);
   S.T0 = -1;
   S.Tc = 0;
 }
@@ -770,7 +981,7 @@ __device__ void setup_slot(Sim<kReg, kMode>& S, const SimParams& P, unsigned war
 // sim_batch: K full placements.
 // ---------------------------------------------------------------------------
 template <bool kReg>
-__global__ void __launch_bounds__(128) sim_full_kernel(const __grid_constant__ SimParams P) {
+__global__ void __launch_bounds__(128, 7) sim_full_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
@@ -804,6 +1015,7 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
     *reinterpret_cast<uint4*>(B.row + c) = *reinterpret_cast<const uint4*>(P.place + c);
   for (int c = lane; c < B.nck; c += 32) B.ck_time[c] = kI64Max;
   S.fbuf = B.fb;
+  S.hold = B.hb;
   S.row = P.place;
   __syncwarp();
   if (S.row_has_bad_device(P.place)) {
@@ -813,7 +1025,6 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
   S.reset_common();
   S.ck = 0;
   S.next_ck = 0;
-  S.last_t = -1;
   // checkpoint 0: the initial state, valid for every resume time >= 0
   S.maybe_checkpoint(S.kc.make(0, kReady, 0));
   S.run();
@@ -870,11 +1081,6 @@ __device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k,
   }
   bad_range = __any_sync(kFullMask, bad_range);
   dup = __any_sync(kFullMask, dup);
-  __syncwarp();
-  for (int t = lane; t < nm; t += 32) {
-    const int32_t op = P.move_op[m0 + t];
-    if (op >= 0 && op < g.n) atomicAnd(&S.bits[op >> 5], ~(1u << (op & 31)));
-  }
   __syncwarp();
   if (B.status[0] != GMG_SIM_OK) {
     S.write_invalid(k, GMG_SIM_BADBASE);
@@ -943,84 +1149,90 @@ __device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k,
   for (int c = lane; c < B.nck; c += 32)
     if (B.ck_time[c] <= S.T0) best = c;
   const int c = __reduce_max_sync(kFullMask, best);
-  // Restore the simulator state of checkpoint c.
   const int64_t* sc = B.ck_scalars + (int64_t)c * 8;
-  S.Tc = B.ck_time[c];
   const int qsz = (int)sc[0];
-  if (qsz > S.q.cap) {
+  const int msz = (int)sc[7];
+  if (qsz > S.q.cap || msz > S.log.cap) {
     S.write_invalid(k, GMG_SIM_QUEUE);
     return;
   }
+  // Restore the simulator state of checkpoint c.
+  S.Tc = B.ck_time[c];
   S.rootptr = (int)sc[1];
   S.score = sc[2];
   S.makespan = sc[3];
   S.vflag = (int32_t)sc[4];
   S.vt = sc[5];
-  S.vop = (int32_t)sc[6];
-  S.vdev = (int32_t)sc[7];
+  S.vop = (int32_t)(sc[6] >> 32);
+  S.vdev = (int32_t)(sc[6] & 0xffffffff);
   S.iters = 0;
   S.nev = 0;
   S.readypops = 0;
   S.last_t = -1;
   S.status = GMG_SIM_OK;
+  S.trig = P.drain_trigger;
   S.dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
   for (int r = lane; r < g.R; r += 32) S.creq[r] = B.ck_creq[(int64_t)c * g.R + r];
-  // Copy the checkpoint queue, dropping events that the moves invalidate and
-  // re-keying moved ops that were ready at T_c:
-  //  * READY(x) of a moved x: its inputs' transfer times change;
-  //  * FREE / remote ALLOC events of an op p with a moved successor: the set
-  //    of receiving accelerators and last consumers of p's output changed
-  //    (they are all at times >= f_p >= T0 and are regenerated below).
+  for (int w = lane; w < words; w += 32) S.bits[w] = B.ck_bits[(int64_t)c * B.ck_words + w];
+  // READY keys at T_c; a moved op's key is recomputed (its inputs' transfer
+  // times change; its predecessors all finished before T_c).
+  for (int x = lane; x < qsz; x += 32) {
+    uint64_t key = B.ck_qkey[(int64_t)c * B.ckq + x];
+    const uint32_t op = S.kc.op(key);
+    if (crow[op] != B.row[op]) {
+      const int dx = crow[op];
+      const uint4 ls = op_lists(g.ops, op);
+      int64_t rx = op_relxq(g.ops, op).x;
+      for (uint32_t u = 0; u < ls.w; ++u) {
+        const uint32_t p = __ldg(g.pred + ls.z + u) & kIdMask;
+        const int dp = crow[p];
+        int64_t a = S.fb[p];
+        if (dp != dx) a += S.xfer(dp, dx, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
+        rx = a > rx ? a : rx;
+      }
+      key = S.kc.make(rx, kReady, op);
+    }
+    *S.q.kp(x) = key;
+  }
+  S.q.size = qsz;
+  // Logged HBM events at T_c, except those of an op p with a moved
+  // successor: the receiving accelerators and last consumers of p's output
+  // changed (its receive allocations and releases all happen at times
+  // >= f_p >= T0), so they are regenerated below.
   int outn = 0;
-  for (int c0 = 0; c0 < qsz; c0 += 32) {
+  for (int c0 = 0; c0 < msz; c0 += 32) {
     const int idx = c0 + (int)lane;
-    const bool v = idx < qsz;
-    uint64_t key = 0;
-    uint32_t pay = 0;
+    const bool v = idx < msz;
+    uint64_t e = 0;
+    uint8_t dv8 = 0;
     bool keep = false;
     if (v) {
-      key = B.ck_qkey[(int64_t)c * B.ckq + idx];
-      pay = B.ck_qpay[(int64_t)c * B.ckq + idx];
+      e = B.ck_mkey[(int64_t)c * B.ckm + idx];
+      dv8 = B.ck_mdev[(int64_t)c * B.ckm + idx];
       keep = true;
-      const uint32_t cls = S.kc.cls(key), op = S.kc.op(key);
-      if (cls == kReady) {
-        if (crow[op] != B.row[op]) {
-          const int dx = crow[op];
-          const uint4 ls = op_lists(g.ops, op);
-          int64_t rx = op_relxq(g.ops, op).x;
-          for (uint32_t u = 0; u < ls.w; ++u) {
-            const uint32_t p = __ldg(g.pred + ls.z + u) & kIdMask;
-            const int dp = crow[p];
-            int64_t a = S.fb[p];
-            if (dp != dx) a += S.xfer(dp, dx, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
-            rx = a > rx ? a : rx;
-          }
-          key = S.kc.make(rx, kReady, op);
-        }
-      } else {
-        const uint4 ls = op_lists(g.ops, op);
-        bool moved_succ = false;
-        for (uint32_t u = 0; u < ls.y && !moved_succ; ++u) {
-          const uint32_t j = __ldg(g.succ + ls.x + u);
-          moved_succ = crow[j] != B.row[j];
-        }
-        if (moved_succ && (cls == kFree || (int)(pay & 0xffu) != B.row[op])) keep = false;
+      const uint32_t cls = S.kc.cls(e), op = S.kc.op(e);
+      const int dev = g.dev_key ? (int)(e >> S.ds) : (int)dv8;
+      const uint4 ls = op_lists(g.ops, op);
+      bool moved_succ = false;
+      for (uint32_t u = 0; u < ls.y && !moved_succ; ++u) {
+        const uint32_t j = __ldg(g.succ + ls.x + u);
+        moved_succ = crow[j] != B.row[j];
       }
+      if (moved_succ && (cls == kFree || dev != B.row[op])) keep = false;
     }
-    __syncwarp();
     const uint32_t bal = __ballot_sync(kFullMask, keep);
-    const int pos = outn + __popc(bal & ((1u << lane) - 1u));
     if (keep) {
-      *S.q.kp(pos) = key;
-      *S.q.pp(pos) = pay;
+      const int pos = outn + __popc(bal & lanes_below());
+      *S.log.kp(pos) = e;
+      *S.log.dp(pos) = dv8;
     }
     outn += __popc(bal);
-    __syncwarp();
   }
-  S.q.size = outn;
-  // Regenerate the memory events of every predecessor p (simulated before
-  // T_c) of a moved op under the candidate placement.  Each p is handled by
-  // its smallest-id moved successor.
+  S.log.n = outn;
+  __syncwarp();
+  // Regenerate the HBM events of every predecessor p (finished before T_c)
+  // of a moved op under the candidate placement; each p once, by its
+  // smallest-id moved successor.
   for (int c0 = 0; c0 < nm; c0 += 32) {
     const int t = c0 + (int)lane;
     int32_t x = -1;
@@ -1064,10 +1276,10 @@ __device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k,
   S.finish(k);
 }
 
-// Memory events of op p (finished before the resume point) under the
-// candidate placement: receive copies on every remote accelerator of its
-// successors (allocated at f_p), and the releases that are already
-// determined because every listed consumer on that accelerator has finished.
+// HBM events of op p (finished before the resume point) under the candidate
+// placement: receive copies on every remote accelerator of its successors
+// (allocated at f_p), and the releases that are already determined because
+// every listed consumer on that accelerator has finished.
 template <bool kReg>
 __device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
   const DevGmg& g = S.g;
@@ -1080,7 +1292,7 @@ __device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
   const bool all = (pcs.w & kAllCons) != 0;
   const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
   const uint32_t nl = all ? pls.y : pcs.y;
-  int64_t hold = fp;
+  int64_t hm = fp;
   for (uint32_t c0 = 0; c0 < pls.y; c0 += 32) {
     const uint32_t t = c0 + lane;
     const bool v = t < pls.y;
@@ -1099,9 +1311,9 @@ __device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
           leader = false;
           break;
         }
-    const uint64_t hm = warp_max_u64(leader ? (uint64_t)arr : 0ull);
-    hold = (int64_t)hm > hold ? (int64_t)hm : hold;
-    S.template push_lanes<true>(__ballot_sync(kFullMask, leader), S.kc.make(fp, kAlloc, p), (uint32_t)du);
+    const int64_t hl = (int64_t)warp_max_u64(leader ? (uint64_t)arr : 0ull);
+    hm = hl > hm ? hl : hm;
+    S.log_event(leader, S.kc.make(fp, kAlloc, p), du);
     bool rel = false;
     int64_t tr = arr;
     if (leader) {
@@ -1117,7 +1329,7 @@ __device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
         tr = fc > tr ? fc : tr;
       }
     }
-    S.template push_lanes<true>(__ballot_sync(kFullMask, rel), S.kc.make(tr, kFree, p), (uint32_t)du);
+    S.log_event(rel, S.kc.make(tr, kFree, p), du);
   }
   // source copy
   bool pending = false;
@@ -1137,11 +1349,11 @@ __device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
   }
   if (__any_sync(kFullMask, pending)) return;
   const int64_t m = (int64_t)warp_max_u64(mx);
-  S.append(S.kc.make(m > hold ? m : hold, kFree, p), (uint32_t)dp);
+  S.log_event(lane == 0, S.kc.make(m > hm ? m : hm, kFree, p), dp);
 }
 
 template <bool kReg>
-__global__ void __launch_bounds__(128) sim_inc_kernel(const __grid_constant__ SimParams P) {
+__global__ void __launch_bounds__(128, 7) sim_inc_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
@@ -1150,15 +1362,14 @@ __global__ void __launch_bounds__(128) sim_inc_kernel(const __grid_constant__ Si
   setup_slot(S, P, wib, slot, smem);
   S.rb = P.base.rb;
   S.fb = P.base.fb;
-  S.brow = P.base.row;
   uint8_t* crow = P.scratch + slot * P.slot_bytes + P.off_row;
   for (int64_t k = slot; k < P.K; k += nslots) inc_candidate(S, P, k, crow);
 }
 
 // ---------------------------------------------------------------------------
 // select_best (Algorithm 1, BestRecordedCandidateResult): block argmin of
-// the packed rank, then a one-block final argmin.
-// rank = (status != 0 || infeasible) ? none : (mode ? sla_miss : 0, score, k)
+// (mode ? sla_miss : 0, score, k) over eligible candidates, then a one-block
+// final argmin.
 // ---------------------------------------------------------------------------
 struct Rank {
   int64_t a;  // sla_miss (mode 1) or 0; INT64_MAX = not eligible
@@ -1236,6 +1447,17 @@ const void* full_kernel_ptr(bool reg) {
 }
 const void* inc_kernel_ptr(bool reg) {
   return reg ? (const void*)sim_inc_kernel<true> : (const void*)sim_inc_kernel<false>;
+}
+
+cudaError_t set_smem_limits(int smem) {
+  const void* fns[] = {(const void*)sim_full_kernel<true>, (const void*)sim_full_kernel<false>,
+                       (const void*)sim_inc_kernel<true>,  (const void*)sim_inc_kernel<false>,
+                       (const void*)sim_base_kernel<true>, (const void*)sim_base_kernel<false>};
+  for (const void* f : fns) {
+    const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    if (e != cudaSuccess) return e;
+  }
+  return cudaSuccess;
 }
 
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
