@@ -171,6 +171,31 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld,
               const sim_opts_t* opts, const sim_out_t* d_out, void* d_scratch,
               size_t scratch_bytes, gmg_stream_t stream);
 
+/* Size of the library's own scratch buffer used by sim_batch_noalloc. */
+#define GMG_NOALLOC_SCRATCH_BYTES ((size_t)32 << 20)
+
+/* sim_batch without a caller scratch buffer (the paper has no counterpart;
+ * this is a deployment convenience).  Some callers cannot allocate device
+ * memory when they evaluate placements: a scheduler loop that runs under a
+ * fixed device-memory budget, code embedded in another framework that owns
+ * the allocator, or a host that must not allocate after start-up.  This call
+ * takes only the placements and the output arrays; the per-warp scratch is a
+ * GMG_NOALLOC_SCRATCH_BYTES buffer compiled into the library, present on every
+ * GPU that loads the library until the process exits.  It never calls
+ * cudaMalloc or cudaFree.  Results are identical to sim_batch; with large
+ * graphs fewer warps run at once because fewer scratch slots fit.
+ *   - Returns GMG_EWS if one warp's scratch for this graph does not fit in
+ *     the buffer (about 16 bytes per op plus queue spill space), other
+ *     arguments and errors as sim_batch.
+ *   - The first call on each device looks up the buffer's device address
+ *     (with that device current); make that first call before any stream
+ *     capture.
+ *   - All calls share the buffer and find the previous call's data in it;
+ *     nothing needs clearing (the kernel initialises what it reads), but two
+ *     calls that could run at the same time on the GPU race: order them. */
+int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld,
+                      const sim_opts_t* opts, const sim_out_t* d_out, gmg_stream_t stream);
+
 /* Bytes of device workspace base_create needs. */
 size_t base_workspace_bytes(const gmg_t* g, const sim_opts_t* opts);
 

@@ -6,6 +6,7 @@
 
 #include <algorithm>
 #include <cstring>
+#include <mutex>
 #include <new>
 #include <vector>
 
@@ -627,6 +628,79 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   P.K = K;
   P.scratch = static_cast<uint8_t*>(d_scratch);
   cudaError_t e = launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
+  return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
+}
+
+// ---------------------------------------------------------------------------
+// sim_batch_noalloc: sim_batch for callers that cannot allocate device memory.
+//
+// Its per-warp scratch is a fixed buffer that lives in the library itself
+// (below), so a caller hands over only the placements and the output arrays.
+// The buffer is GMG_NOALLOC_SCRATCH_BYTES large and exists on every GPU that
+// loads the library until the process exits.  Every call reuses it and finds
+// the previous call's contents there; the kernel initialises every scratch
+// word it reads for each candidate, so nothing has to be cleared between
+// calls.  Two calls whose kernels could overlap on the GPU would race on the
+// buffer: order them on one stream (or with events).
+// ---------------------------------------------------------------------------
+static __device__ __align__(256) uint8_t g_noalloc_scratch[GMG_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+std::mutex g_noalloc_mu;
+void* g_noalloc_ptr[kMaxDevices] = {};
+
+// The buffer's device address on the current device.  Host code may not use
+// the symbol itself as an address, so the runtime is asked once per device
+// (with that device current) and the answer is kept.
+int noalloc_scratch(uint8_t** out) {
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return GMG_ECUDA;
+  if (dev < 0 || dev >= kMaxDevices) return GMG_ECUDA;
+  std::lock_guard<std::mutex> lock(g_noalloc_mu);
+  if (!g_noalloc_ptr[dev]) {
+    void* p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || !p) return GMG_ECUDA;
+    g_noalloc_ptr[dev] = p;
+  }
+  *out = static_cast<uint8_t*>(g_noalloc_ptr[dev]);
+  return GMG_OK;
+}
+
+}  // namespace
+
+extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld,
+                                 const sim_opts_t* opts, const sim_out_t* d_out, gmg_stream_t stream) {
+  if (!g || K < 0) return GMG_EINVAL;
+  int rc = check_out(d_out, opts);
+  if (rc) return rc;
+  if (K == 0) return GMG_OK;
+  if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
+  Launch L;
+  rc = plan_launch(g, K, opts, false, L);
+  if (rc) return rc;
+  // As many warp slots as the fixed buffer holds (each warp then takes more
+  // candidates in turn); a graph whose single slot does not fit is refused.
+  const int64_t fit = (int64_t)(GMG_NOALLOC_SCRATCH_BYTES / (size_t)L.P.slot_bytes);
+  if (fit < 1) return GMG_EWS;
+  if (fit < L.wpb) {
+    sim_opts_t one = opts ? *opts : sim_opts_t{};
+    one.warps_per_block = 1;
+    rc = plan_launch(g, K, &one, false, L);
+    if (rc) return rc;
+  }
+  L.grid = (int)std::min<int64_t>(L.grid, fit / L.wpb);
+  uint8_t* scratch = nullptr;
+  rc = noalloc_scratch(&scratch);
+  if (rc) return rc;
+  SimParams& P = L.P;
+  fill_out(P, d_out, opts);
+  P.place = d_place;
+  P.ld = ld;
+  P.K = K;
+  P.scratch = scratch;
+  const cudaError_t e = launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 

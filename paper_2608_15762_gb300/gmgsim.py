@@ -23,7 +23,7 @@ GMG_OK, GMG_EINVAL, GMG_ENOTTOPO, GMG_ERANGE, GMG_EWS, GMG_ECUDA, GMG_ENOMEM = 0
 SIM_OK, SIM_BADDEV, SIM_MOVE_RANGE, SIM_MOVE_DUP, SIM_BADBASE, SIM_QUEUE, SIM_LOOP = range(7)
 
 EXPORTED = ("gmg_workspace_bytes", "gmg_create", "gmg_destroy", "gmg_get_info", "sim_scratch_bytes",
-            "sim_batch", "base_workspace_bytes", "base_create", "base_destroy", "inc_scratch_bytes",
+            "sim_batch", "sim_batch_noalloc", "base_workspace_bytes", "base_create", "base_destroy", "inc_scratch_bytes",
             "sim_incremental", "select_best_tmp_bytes", "select_best", "gmg_strerror",
             "gmg_ceil_div_host")
 
@@ -79,6 +79,7 @@ def lib():
             "gmg_get_info": ([vp, vp], C.c_int),
             "sim_scratch_bytes": ([vp, i32, vp], sz),
             "sim_batch": ([vp, vp, i32, i32, vp, vp, vp, sz, vp], C.c_int),
+            "sim_batch_noalloc": ([vp, vp, i32, i32, vp, vp, vp], C.c_int),
             "base_workspace_bytes": ([vp, vp], sz),
             "base_create": ([vp, vp, vp, vp, sz, vp, vp], C.c_int),
             "base_destroy": ([vp], None),
@@ -288,6 +289,25 @@ def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scr
                          buf.data_ptr(), buf.numel(), _stream_handle(stream))
     if rc != GMG_OK:
         raise GmgError(rc, "sim_batch")
+    return out
+
+
+def sim_batch_noalloc(g: Gmg, place, out: Optional[SimOut] = None, req_done=False, trace_k=None,
+                      stream=None) -> SimOut:
+    """Like sim_batch, but the library supplies the scratch from its own fixed
+    device buffer (for callers that cannot allocate device memory)."""
+    import torch
+    assert place.dtype == torch.uint8 and place.dim() == 2 and place.is_contiguous()
+    K, ld = place.shape
+    n_trace = 0 if trace_k is None else int(trace_k.numel())
+    if out is None:
+        out = SimOut.empty(K, g.n_dev, g.n_req, place.device, req_done, n_trace, g.n_ops)
+    o = _opts(0, trace_k)
+    co = out._c()
+    rc = lib().sim_batch_noalloc(g.handle, place.data_ptr(), K, ld, C.addressof(o), C.addressof(co),
+                                 _stream_handle(stream))
+    if rc != GMG_OK:
+        raise GmgError(rc, "sim_batch_noalloc")
     return out
 
 

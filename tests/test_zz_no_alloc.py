@@ -1,0 +1,73 @@
+"""sim_batch_noalloc: the variant of sim_batch for callers that cannot
+allocate device memory (its scratch is a fixed buffer inside the library).
+Its results must equal sim_batch's on consecutive calls, which also shows
+that leftovers of one call in the shared buffer do not leak into the next."""
+import ctypes as C
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from paper_2608_15762_gb300 import gmgsim as G  # noqa: E402
+from paper_2608_15762_gb300 import workloads as W  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+FIELDS = ("status", "makespan", "score", "viol_flag", "viol_op", "viol_dev", "viol_time", "peak",
+          "sla_miss", "events", "req_done", "trace_start", "trace_finish")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_15762_gb300 import build
+    build.build()
+    assert torch.cuda.is_available()
+
+
+def _rows(seed, K, n, D):
+    g = np.random.default_rng(seed)
+    rows = np.zeros((K, W.placement_ld(n)), np.uint8)
+    rows[:, :n] = g.integers(0, D, (K, n))
+    return torch.from_numpy(rows).cuda()
+
+
+@pytest.mark.parametrize("which", ["tiny", "random"])
+def test_same_results_as_sim_batch_on_two_calls(which):
+    if which == "tiny":
+        wl = W.config1()
+        desc = wl.desc
+        batches = [torch.from_numpy(wl.all_full_rows()).cuda(), _rows(9, 300, desc.n_ops, desc.n_dev)]
+    else:
+        desc = W.random_desc(21, 700, 40, explicit_cons=True)
+        batches = [_rows(1, 257, 700, 40), _rows(2, 128, 700, 40)]
+    g = G.gmg_create(desc)
+    for place in batches:
+        tk = torch.tensor([0, place.shape[0] - 1], dtype=torch.int32, device="cuda")
+        ref = G.sim_batch(g, place, req_done=True, trace_k=tk)
+        got = G.sim_batch_noalloc(g, place, req_done=True, trace_k=tk)
+        torch.cuda.synchronize()
+        a, b = ref.to_numpy(), got.to_numpy()
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f]), f
+
+
+def test_refuses_a_graph_whose_scratch_does_not_fit():
+    n = 3 << 20   # one warp's scratch alone is ~16 bytes per op: > 32 MiB
+    pred_off = np.arange(n + 1, dtype=np.int32) - 1
+    pred_off[0] = 0
+    desc = W.GmgDesc(n_dev=2, pred_off=pred_off, pred_idx=np.arange(n - 1, dtype=np.int32),
+                     dur=np.ones(n, np.int64), out_bytes=np.ones(n, np.int64),
+                     release=np.zeros(n, np.int64), req_id=np.full(n, -1, np.int32),
+                     scored=np.ones(n, np.uint8), deadline=np.zeros(0, np.int64),
+                     cap=np.full(2, 1 << 40, np.int64), base=np.zeros(2, np.int64),
+                     avail0=np.zeros(2, np.int64), bw=np.ones(4, np.int64),
+                     lat=np.zeros(4, np.int64)).normalized()
+    g = G.gmg_create(desc)
+    place = torch.zeros((1, W.placement_ld(n)), dtype=torch.uint8, device="cuda")
+    out = G.SimOut.empty(1, 2, 0, place.device)
+    co = out._c()
+    o = G._opts()
+    rc = G.lib().sim_batch_noalloc(g.handle, place.data_ptr(), 1, place.shape[1], C.addressof(o),
+                                   C.addressof(co), None)
+    assert rc == G.GMG_EWS
