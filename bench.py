@@ -223,8 +223,10 @@ def cpu_baseline(wl, budget_s=20.0):
     the same workload (whole batches until about budget_s of CPU time)."""
     from oracle import oracle as O
     nt = O.hw_threads()
+    # about 20 s of oracle work on 16 cores: ~3e8 op-events
+    budget = max(16, int(3e8 // max(wl.desc.n_ops, 1)))
     if wl.n_full:
-        k = min(wl.n_full, 4096)
+        k = min(wl.n_full, budget)
         rows = wl.full_rows(range(k))
         t0 = time.perf_counter()
         O.simulate_batch(wl.desc, rows, nthreads=nt)
@@ -232,7 +234,7 @@ def cpu_baseline(wl, budget_s=20.0):
         sample = "%d of %d full placements" % (k, wl.n_full)
     else:
         from paper_2608_15762_gb300.workloads import Moves
-        k = min(wl.moves.n_cand, 2048)
+        k = min(wl.moves.n_cand, budget)
         mv = Moves(wl.moves.off[:k + 1].copy(), wl.moves.op[:wl.moves.off[k]], wl.moves.dev[:wl.moves.off[k]])
         t0 = time.perf_counter()
         O.incremental_batch(wl.desc, wl.base_place, mv, nthreads=nt)
@@ -251,7 +253,7 @@ def reference_arm(args):
     from paper_2608_15762_gb300 import workloads as W
     wl = W.make_workload(args.config)
     nt = O.hw_threads()
-    k = min(wl.n_full or wl.moves.n_cand, 4096 if wl.desc.n_ops < 10000 else 64)
+    k = min(wl.n_full or wl.moves.n_cand, max(16, int(3e7 // max(wl.desc.n_ops, 1))))
     if wl.n_full:
         rows = wl.full_rows(range(k))
 

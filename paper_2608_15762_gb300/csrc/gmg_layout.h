@@ -76,8 +76,8 @@ struct DevGmg {
   const OpRec* ops;
   const uint32_t* succ;
   const uint32_t* pred;
-  const uint32_t* psib;       // per predecessor entry of a holding consumer: the other
-                              // listed consumer of that predecessor (kSibNone / kSibMany)
+  const uint2* predsib;       // per predecessor entry: {pred | hold bit, the other listed
+                              // consumer of that predecessor (kSibNone / kSibMany)}
   const uint32_t* cons;
   const uint64_t* root_keys;  // READY keys of ops without predecessors, ascending
   const int64_t* cap;

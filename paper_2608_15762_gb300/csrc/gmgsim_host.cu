@@ -15,8 +15,8 @@
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
 size_t select_rank_bytes();
-const void* full_kernel_ptr(bool reg);
-const void* inc_kernel_ptr(bool reg);
+const void* full_kernel_ptr(bool reg, bool key);
+const void* inc_kernel_ptr(bool reg, bool key);
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
@@ -38,7 +38,7 @@ constexpr int64_t kDefaultQueueCap = 1 << 16;
 constexpr int kSharedLogEntries = 160;
 constexpr int64_t kDefaultLogCap = 1 << 17;
 constexpr int kSortCap = 128;             // power of two; raised to n_dev's power of two
-constexpr int kDrainTrigger = 64;
+constexpr int kDrainTrigger = 48;
 constexpr int kCheckpoints = 256;
 constexpr int kCheckpointQueue = 4096;
 constexpr int kCheckpointLog = 8192;
@@ -93,7 +93,7 @@ void plan(Built& b) {
   L.off_ops = take(sizeof(OpRec) * (size_t)b.n);
   L.off_succ = take(4 * (size_t)b.E);
   L.off_pred = take(4 * (size_t)b.E);
-  L.off_sib = take(4 * (size_t)b.E);
+  L.off_sib = take(8 * (size_t)b.E);
   L.off_cons = take(4 * (size_t)b.Ec);
   L.off_roots = take(8 * (size_t)b.nroots);
   L.off_cap = take(8 * (size_t)b.D);
@@ -416,7 +416,7 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     g_smem_set = true;
   }
   int bps = 0;
-  const void* fn = inc ? inc_kernel_ptr(L.reg) : full_kernel_ptr(L.reg);
+  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0) : full_kernel_ptr(L.reg, G.dev_key != 0);
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
     return GMG_ECUDA;
   bps = std::max(bps, 1);
@@ -537,7 +537,14 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   put(L.off_ops, b.ops.data(), sizeof(OpRec) * b.ops.size());
   put(L.off_succ, b.succ.data(), 4 * b.succ.size());
   put(L.off_pred, b.pred.data(), 4 * b.pred.size());
-  put(L.off_sib, b.sib.data(), 4 * b.sib.size());
+  {
+    std::vector<uint32_t> ps(2 * (size_t)b.E);
+    for (int k = 0; k < b.E; ++k) {
+      ps[2 * (size_t)k] = b.pred[k];
+      ps[2 * (size_t)k + 1] = b.sib[k];
+    }
+    put(L.off_sib, ps.data(), 4 * ps.size());
+  }
   put(L.off_cons, b.cons.data(), 4 * b.cons.size());
   put(L.off_roots, b.roots.data(), 8 * b.roots.size());
   put(L.off_cap, b.cap.data(), 8 * b.cap.size());
@@ -556,7 +563,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.ops = reinterpret_cast<const OpRec*>(w + L.off_ops);
   G.succ = reinterpret_cast<const uint32_t*>(w + L.off_succ);
   G.pred = reinterpret_cast<const uint32_t*>(w + L.off_pred);
-  G.psib = reinterpret_cast<const uint32_t*>(w + L.off_sib);
+  G.predsib = reinterpret_cast<const uint2*>(w + L.off_sib);
   G.cons = reinterpret_cast<const uint32_t*>(w + L.off_cons);
   G.root_keys = reinterpret_cast<const uint64_t*>(w + L.off_roots);
   G.cap = reinterpret_cast<const int64_t*>(w + L.off_cap);

@@ -287,12 +287,13 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
 // ---------------------------------------------------------------------------
 // One warp's simulator.
 // ---------------------------------------------------------------------------
-template <bool kReg, int kMode>
+template <bool kReg, int kMode, bool kKey>
 struct Sim {
   const SimParams& P;
   const DevGmg& g;
   KeyCodec kc;
-  ReadyHeap q;
+  ReadyHeap q;      // READY keys beyond the register tier
+  uint64_t rk_reg;  // register tier: one READY key per lane (kKeyMax = empty)
   MemLog log;
   uint64_t* sortk;
   uint8_t* sortd;
@@ -321,7 +322,7 @@ struct Sim {
     kc.ib = g.ib;
     kc.mask = (1ull << g.ib) - 1ull;
     ds = g.ib + 2 + g.tb;
-    lowmask = g.dev_key ? (1ull << ds) - 1ull : kKeyMax;
+    lowmask = kKey ? (1ull << ds) - 1ull : kKeyMax;
   }
 
   __device__ __forceinline__ bool popped(uint32_t x) const { return (bits[x >> 5] >> (x & 31u)) & 1u; }
@@ -366,31 +367,35 @@ struct Sim {
     return hold[p];
   }
 
+  // READY keys go to a free lane's register if there is one, else the heap.
   __device__ __forceinline__ void push_ready(uint64_t key) {
     if (status) return;
-    if (!q.push(key)) status = GMG_SIM_QUEUE;
+    const uint32_t freel = __ballot_sync(kFullMask, rk_reg == kKeyMax);
+    if (freel) {
+      if ((int)lane_id() == __ffs(freel) - 1) rk_reg = key;
+    } else if (!q.push(key)) {
+      status = GMG_SIM_QUEUE;
+    }
   }
   // Every lane with `want` logs (key, dev).  Uniform call.
   __device__ __forceinline__ void log_event(bool want, uint64_t key, int dev) {
     const uint32_t b = __ballot_sync(kFullMask, want);
-    if (b == 0u || status) return;
     const int cnt = __popc(b);
     const int pos = log.n + __popc(b & lanes_below());
-    const uint64_t e = g.dev_key ? (((uint64_t)(dev & 0xff) << ds) | key) : key;
-    if (log.n + cnt <= log.ms) {
-      if (want) {
-        log.sk[pos] = e;
-        if (!g.dev_key) log.sd[pos] = (uint8_t)dev;
-      }
-    } else {
-      if (log.n + cnt > log.cap) {
-        status = GMG_SIM_QUEUE;
-        return;
-      }
-      if (want) {
-        *log.kp(pos) = e;
-        if (!g.dev_key) *log.dp(pos) = (uint8_t)dev;
-      }
+    if (kKey && log.n + 32 <= log.ms) {
+      // fast path: every lane's slot is in shared memory
+      if (want) log.sk[pos] = ((uint64_t)(dev & 0xff) << ds) | key;
+      log.n += cnt;
+      return;
+    }
+    if (cnt == 0 || status) return;
+    if (log.n + cnt > log.cap) {
+      status = GMG_SIM_QUEUE;
+      return;
+    }
+    if (want) {
+      *log.kp(pos) = kKey ? (((uint64_t)(dev & 0xff) << ds) | key) : key;
+      if (!kKey) *log.dp(pos) = (uint8_t)dev;
     }
     log.n += cnt;
   }
@@ -402,6 +407,7 @@ struct Sim {
     for (int r = lane; r < g.R; r += 32) creq[r] = 0;
     dv.reset(g);
     q.size = 0;
+    rk_reg = kKeyMax;
     log.n = 0;
     trig = P.drain_trigger;
     rootptr = 0;
@@ -489,18 +495,27 @@ struct Sim {
         push_ready(__shfl_sync(kFullMask, kc.make(rj, kReady, j), src));
       }
       const bool rem = v && dj != d;
-      local_succ |= __any_sync(kFullMask, v && dj == d);
-      const uint32_t peers = __match_any_sync(kFullMask, rem ? (uint32_t)dj : (256u + lane));
-      bool leader = rem && (__ffs(peers) - 1 == (int)lane);
-      if (leader && c0 > 0) {
-        for (uint32_t u = 0; u < c0; ++u)
-          if (row[__ldg(g.succ + succ_off + u)] == dj) {
-            leader = false;
-            break;
-          }
+      bool leader;
+      if (nsucc == 1) {
+        // one successor, on lane 0
+        leader = rem;
+        local_succ = __shfl_sync(kFullMask, v && dj == d, 0);
+        const int64_t a0 = __shfl_sync(kFullMask, rem ? arr : f, 0);
+        hm = a0 > hm ? a0 : hm;
+      } else {
+        local_succ |= __any_sync(kFullMask, v && dj == d);
+        const uint32_t peers = __match_any_sync(kFullMask, rem ? (uint32_t)dj : (256u + lane));
+        leader = rem && (__ffs(peers) - 1 == (int)lane);
+        if (leader && c0 > 0) {
+          for (uint32_t u = 0; u < c0; ++u)
+            if (row[__ldg(g.succ + succ_off + u)] == dj) {
+              leader = false;
+              break;
+            }
+        }
+        const int64_t hl = (int64_t)warp_max_u64(leader ? (uint64_t)arr : 0ull);
+        hm = hl > hm ? hl : hm;
       }
-      const int64_t hl = (int64_t)warp_max_u64(leader ? (uint64_t)arr : 0ull);
-      hm = hl > hm ? hl : hm;
       // one receive copy per distinct remote accelerator, allocated when the
       // transfer starts
       log_event(leader, kc.make(f, kAlloc, i), dj);
@@ -544,10 +559,11 @@ struct Sim {
       int64_t T = f;
       uint32_t p = 0;
       if (t < npred) {
-        const uint32_t pe = __ldg(g.pred + pred_off + t);
+        const uint2 ps = __ldg(g.predsib + pred_off + t);
+        const uint32_t pe = ps.x;
         p = pe & kIdMask;
         if (pe & kHoldBit) {
-          const uint32_t sb = __ldg(g.psib + pred_off + t);
+          const uint32_t sb = ps.y;
           if (sb == kSibNone) {
             rel = true;
           } else if (sb != kSibMany) {
@@ -603,65 +619,100 @@ struct Sim {
     __syncwarp();
   }
 
-  // Apply events sorted by (accelerator, time, class, op), 32 at a time:
-  // each accelerator's events are contiguous, so a segmented warp scan of
-  // the byte deltas gives the live bytes after every event, a segmented max
-  // scan the peak, and a warp min the first capacity violation.
-  __device__ void apply_segmented(int m) {
+  // Apply 32 consecutive events of the (accelerator, time, class, op) order,
+  // one per lane (v: lane holds an event).  Each accelerator's events are
+  // contiguous, so a segmented warp scan of the byte deltas gives the live
+  // bytes after every event; allocations raise the accelerator's peak; the
+  // smallest (time, op, accelerator) allocation over capacity is kept in
+  // vmin.
+  __device__ __forceinline__ void apply_chunk(uint64_t key, bool v, uint64_t& vmin) {
     const unsigned lane = lane_id();
-    const int ds = g.ib + 2 + g.tb;
     const uint64_t tmask = (1ull << g.tb) - 1ull;
-    uint64_t vmin = kKeyMax;
-    for (int c0 = 0; c0 < m; c0 += 32) {
-      const int idx = c0 + (int)lane;
-      const bool v = idx < m;
-      const uint64_t key = v ? sortk[idx] : 0ull;
-      const int dev = v ? (int)(key >> ds) : -1 - (int)lane;
-      const uint32_t op = (uint32_t)(key & kc.mask);
-      const bool isalloc = v && kc.cls(key) == kAlloc;
-      int64_t delta = 0;
-      if (v) {
-        const int64_t b = op_durbytes(g.ops, op).y;
-        delta = isalloc ? b : -b;
-      }
-      int64_t s = delta;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const int64_t o = __shfl_up_sync(kFullMask, s, off);
-        const int od = __shfl_up_sync(kFullMask, dev, off);
-        if ((int)lane >= off && od == dev) s += o;
-      }
-      const int64_t live = (v ? dv.lv[dev] : 0) + s;
-      int64_t pm = isalloc ? live : INT64_MIN;
-#pragma unroll
-      for (int off = 1; off < 32; off <<= 1) {
-        const int64_t o = __shfl_up_sync(kFullMask, pm, off);
-        const int od = __shfl_up_sync(kFullMask, dev, off);
-        if ((int)lane >= off && od == dev && o > pm) pm = o;
-      }
-      const int nd = __shfl_down_sync(kFullMask, dev, 1);
-      const bool last = v && (lane == 31 || nd != dev);
-      const bool over = isalloc && live > __ldg(g.cap + dev);
-      const uint64_t vk = over ? ((((key >> (g.ib + 2)) & tmask) << (g.ib + 8)) | ((uint64_t)op << 8) |
-                                  (uint64_t)dev)
-                               : kKeyMax;
-      const uint64_t cm = warp_min_u64(vk);
-      vmin = cm < vmin ? cm : vmin;
-      __syncwarp();
-      if (last) {
-        dv.lv[dev] = live;
-        if (pm > dv.pk[dev]) dv.pk[dev] = pm;
-      }
-      __syncwarp();
+    const int dev = v ? (int)(key >> ds) : -1 - (int)lane;
+    const uint32_t op = (uint32_t)(key & kc.mask);
+    const bool isalloc = v && kc.cls(key) == kAlloc;
+    int64_t delta = 0;
+    if (v) {
+      const int64_t b = op_durbytes(g.ops, op).y;
+      delta = isalloc ? b : -b;
     }
-    // every event of this drain is later than every event already applied,
-    // so an earlier violation stands
+    int64_t s = delta;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int64_t o = __shfl_up_sync(kFullMask, s, off);
+      const int od = __shfl_up_sync(kFullMask, dev, off);
+      if ((int)lane >= off && od == dev) s += o;
+    }
+    const int64_t live = (v ? dv.lv[dev] : 0) + s;
+    const int nd = __shfl_down_sync(kFullMask, dev, 1);
+    const bool last = v && (lane == 31 || nd != dev);
+    const bool over = isalloc && live > __ldg(g.cap + dev);
+    const uint64_t vk = over ? ((((key >> (g.ib + 2)) & tmask) << (g.ib + 8)) | ((uint64_t)op << 8) |
+                                (uint64_t)dev)
+                             : kKeyMax;
+    const uint64_t cm = warp_min_u64(vk);
+    vmin = cm < vmin ? cm : vmin;
+    __syncwarp();
+    if (isalloc)  // live bytes are never negative
+      atomicMax(reinterpret_cast<unsigned long long*>(dv.pk + dev), (unsigned long long)live);
+    if (last) dv.lv[dev] = live;
+    __syncwarp();
+  }
+
+  // every event of a drain is later than every event already applied, so
+  // an earlier violation stands
+  __device__ __forceinline__ void settle_violation(uint64_t vmin) {
     if (!vflag && vmin != kKeyMax) {
       vflag = 1;
       vt = (int64_t)(vmin >> (g.ib + 8));
       vop = (int32_t)((vmin >> 8) & kc.mask);
       vdev = (int32_t)(vmin & 0xffu);
     }
+  }
+
+  __device__ void apply_segmented(int m) {
+    uint64_t vmin = kKeyMax;
+    for (int c0 = 0; c0 < m; c0 += 32) {
+      const int idx = c0 + (int)lane_id();
+      const bool v = idx < m;
+      apply_chunk(v ? sortk[idx] : 0ull, v, vmin);
+    }
+    settle_violation(vmin);
+  }
+
+  // Sort and apply m <= 64 extracted events in registers: lane l holds
+  // elements l and 32 + l of a bitonic network.
+  __device__ void sort_apply_regs(int m) {
+    const unsigned lane = lane_id();
+    uint64_t a0 = (int)lane < m ? sortk[lane] : kKeyMax;
+    uint64_t a1 = (int)lane + 32 < m ? sortk[lane + 32] : kKeyMax;
+    const bool two = m > 32;
+    const int p2 = two ? 64 : 32;
+    for (int k = 2; k <= p2; k <<= 1) {
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        if (j == 32) {
+          const uint64_t lo = a0 < a1 ? a0 : a1;
+          a1 = a0 < a1 ? a1 : a0;
+          a0 = lo;
+          continue;
+        }
+        const bool lower = (lane & j) == 0;
+        {
+          const uint64_t o = __shfl_xor_sync(kFullMask, a0, j);
+          const bool keep_min = lower == ((lane & k) == 0);
+          a0 = keep_min ? (o < a0 ? o : a0) : (o > a0 ? o : a0);
+        }
+        if (two) {
+          const uint64_t o = __shfl_xor_sync(kFullMask, a1, j);
+          const bool keep_min = lower == (((lane + 32) & k) == 0);
+          a1 = keep_min ? (o < a1 ? o : a1) : (o > a1 ? o : a1);
+        }
+      }
+    }
+    uint64_t vmin = kKeyMax;
+    apply_chunk(a0, (int)lane < m, vmin);
+    if (two) apply_chunk(a1, (int)lane + 32 < m, vmin);
+    settle_violation(vmin);
   }
 
   __device__ int count_below(uint64_t kmax) const {
@@ -678,7 +729,7 @@ struct Sim {
   // number is known to fit) and compact the rest; returns their number.
   __device__ int extract(uint64_t kmax) {
     const unsigned lane = lane_id();
-    const bool side = !g.dev_key;
+    const bool side = !kKey;
     int m = 0, keep = 0;
     const int n = log.n;
     for (int c0 = 0; c0 < n; c0 += 32) {
@@ -719,7 +770,7 @@ struct Sim {
   // power of two >= 32.
   __device__ void sort_area(int m) {
     const unsigned lane = lane_id();
-    const bool side = !g.dev_key;
+    const bool side = !kKey;
     int p2 = 32;
     while (p2 < m) p2 <<= 1;
     for (int x = m + (int)lane; x < p2; x += 32) sortk[x] = kKeyMax;
@@ -776,9 +827,13 @@ struct Sim {
       }
       const int m = extract(kmax);
       if (m == 0) break;
-      sort_area(m);
-      if (g.dev_key) apply_segmented(m);
-      else apply_serial(m);
+      if (kKey && m <= 64) {
+        sort_apply_regs(m);
+      } else {
+        sort_area(m);
+        if (kKey) apply_segmented(m);
+        else apply_serial(m);
+      }
       if (kmax == lim) break;
     }
     trig = log.n + P.drain_trigger;
@@ -791,12 +846,16 @@ struct Sim {
     if (status) return;
     while (true) {
       const uint64_t top = q.top();
+      const uint64_t rm = warp_min_u64(rk_reg);
       const uint64_t rk = rootptr < g.nroots ? __ldg(g.root_keys + rootptr) : kKeyMax;
-      const uint64_t nk = rk < top ? rk : top;
+      uint64_t nk = rk < top ? rk : top;
+      nk = rm < nk ? rm : nk;
       if (kMode == kBase) maybe_checkpoint(nk);
       if (nk == kKeyMax) break;
       if (log.n >= trig) drain(kc.time(nk));
-      if (rk < top) {
+      if (nk == rm) {
+        if (rk_reg == rm) rk_reg = kKeyMax;  // keys are unique
+      } else if (nk == rk) {
         ++rootptr;
       } else {
         __syncwarp();
@@ -910,19 +969,23 @@ struct Sim {
 // handled yet), save the complete simulator state -- simulated-op bitmap,
 // accelerator state, READY heap, event log, partial results.  An
 // incremental candidate whose resume time T0 is >= that time restarts there.
-template <bool kReg, int kMode>
-__device__ void Sim<kReg, kMode>::maybe_checkpoint(uint64_t next_key) {
+template <bool kReg, int kMode, bool kKey>
+__device__ void Sim<kReg, kMode, kKey>::maybe_checkpoint(uint64_t next_key) {
   if (kMode != kBase) return;
   const DevBase& B = P.base;
   if (next_key == kKeyMax || ck >= B.nck || readypops < next_ck) return;
   const int64_t tn = kc.time(next_key);
   if (tn <= last_t) return;
   const unsigned lane = lane_id();
-  if (q.size <= B.ckq && log.n <= B.ckm) {
+  const bool hasreg = rk_reg != kKeyMax;
+  const uint32_t regm = __ballot_sync(kFullMask, hasreg);
+  const int nready = q.size + __popc(regm);
+  if (nready <= B.ckq && log.n <= B.ckm) {
     int64_t* sc = B.ck_scalars + (int64_t)ck * 8;
+    if (hasreg) B.ck_qkey[(int64_t)ck * B.ckq + q.size + __popc(regm & lanes_below())] = rk_reg;
     if (lane == 0) {
       B.ck_time[ck] = tn;
-      sc[0] = q.size;
+      sc[0] = nready;
       sc[1] = rootptr;
       sc[2] = score;
       sc[3] = makespan;
@@ -948,8 +1011,8 @@ __device__ void Sim<kReg, kMode>::maybe_checkpoint(uint64_t next_key) {
   __syncwarp();
 }
 
-template <bool kReg, int kMode>
-__device__ void setup_slot(Sim<kReg, kMode>& S, const SimParams& P, unsigned wib, int64_t slot,
+template <bool kReg, int kMode, bool kKey>
+__device__ void setup_slot(Sim<kReg, kMode, kKey>& S, const SimParams& P, unsigned wib, int64_t slot,
                            uint8_t* smem) {
   uint8_t* sl = P.scratch + slot * P.slot_bytes;
   const WarpSmem w = carve_smem(smem, P, wib);
@@ -980,13 +1043,13 @@ __device__ void setup_slot(Sim<kReg, kMode>& S, const SimParams& P, unsigned wib
 // ---------------------------------------------------------------------------
 // sim_batch: K full placements.
 // ---------------------------------------------------------------------------
-template <bool kReg>
+template <bool kReg, bool kKey>
 __global__ void __launch_bounds__(128, 7) sim_full_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
   const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
-  Sim<kReg, kFull> S(P);
+  Sim<kReg, kFull, kKey> S(P);
   setup_slot(S, P, wib, slot, smem);
   for (int64_t k = slot; k < P.K; k += nslots) {
     S.row = P.place + k * P.ld;
@@ -1003,10 +1066,10 @@ __global__ void __launch_bounds__(128, 7) sim_full_kernel(const __grid_constant_
 // ---------------------------------------------------------------------------
 // base_create: simulate the base placement once, recording resume points.
 // ---------------------------------------------------------------------------
-template <bool kReg>
+template <bool kReg, bool kKey>
 __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
-  Sim<kReg, kBase> S(P);
+  Sim<kReg, kBase, kKey> S(P);
   setup_slot(S, P, 0, 0, smem);
   const DevBase& B = P.base;
   const unsigned lane = lane_id();
@@ -1054,11 +1117,11 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
 // ---------------------------------------------------------------------------
 // sim_incremental: K move lists against the base.
 // ---------------------------------------------------------------------------
-template <bool kReg>
-__device__ void regen(Sim<kReg, kInc>& S, uint32_t p);
+template <bool kReg, bool kKey>
+__device__ void regen(Sim<kReg, kInc, kKey>& S, uint32_t p);
 
-template <bool kReg>
-__device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k, uint8_t* crow) {
+template <bool kReg, bool kKey>
+__device__ void inc_candidate(Sim<kReg, kInc, kKey>& S, const SimParams& P, int64_t k, uint8_t* crow) {
   const DevGmg& g = S.g;
   const DevBase& B = P.base;
   const unsigned lane = lane_id();
@@ -1171,6 +1234,7 @@ __device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k,
   S.last_t = -1;
   S.status = GMG_SIM_OK;
   S.trig = P.drain_trigger;
+  S.rk_reg = kKeyMax;
   S.dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
   for (int r = lane; r < g.R; r += 32) S.creq[r] = B.ck_creq[(int64_t)c * g.R + r];
   for (int w = lane; w < words; w += 32) S.bits[w] = B.ck_bits[(int64_t)c * B.ck_words + w];
@@ -1211,7 +1275,7 @@ __device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k,
       dv8 = B.ck_mdev[(int64_t)c * B.ckm + idx];
       keep = true;
       const uint32_t cls = S.kc.cls(e), op = S.kc.op(e);
-      const int dev = g.dev_key ? (int)(e >> S.ds) : (int)dv8;
+      const int dev = kKey ? (int)(e >> S.ds) : (int)dv8;
       const uint4 ls = op_lists(g.ops, op);
       bool moved_succ = false;
       for (uint32_t u = 0; u < ls.y && !moved_succ; ++u) {
@@ -1280,8 +1344,8 @@ __device__ void inc_candidate(Sim<kReg, kInc>& S, const SimParams& P, int64_t k,
 // placement: receive copies on every remote accelerator of its successors
 // (allocated at f_p), and the releases that are already determined because
 // every listed consumer on that accelerator has finished.
-template <bool kReg>
-__device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
+template <bool kReg, bool kKey>
+__device__ void regen(Sim<kReg, kInc, kKey>& S, uint32_t p) {
   const DevGmg& g = S.g;
   const unsigned lane = lane_id();
   const int64_t fp = S.fb[p];
@@ -1352,13 +1416,13 @@ __device__ void regen(Sim<kReg, kInc>& S, uint32_t p) {
   S.log_event(lane == 0, S.kc.make(m > hm ? m : hm, kFree, p), dp);
 }
 
-template <bool kReg>
+template <bool kReg, bool kKey>
 __global__ void __launch_bounds__(128, 7) sim_inc_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
   const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
-  Sim<kReg, kInc> S(P);
+  Sim<kReg, kInc, kKey> S(P);
   setup_slot(S, P, wib, slot, smem);
   S.rb = P.base.rb;
   S.fb = P.base.fb;
@@ -1442,39 +1506,66 @@ __global__ void __launch_bounds__(256) select_final_kernel(const Rank* part, int
 // ---------------------------------------------------------------------------
 size_t select_rank_bytes() { return sizeof(Rank); }
 
-const void* full_kernel_ptr(bool reg) {
-  return reg ? (const void*)sim_full_kernel<true> : (const void*)sim_full_kernel<false>;
-}
-const void* inc_kernel_ptr(bool reg) {
-  return reg ? (const void*)sim_inc_kernel<true> : (const void*)sim_inc_kernel<false>;
-}
+// Kernel instances by (accelerator state in registers, accelerator id in
+// the event key).
+#define GSIM_KERNEL_TABLE(name)                                                          \
+  const void* name##_ptr(bool reg, bool key) {                                           \
+    if (reg) return key ? (const void*)name<true, true> : (const void*)name<true, false>;  \
+    return key ? (const void*)name<false, true> : (const void*)name<false, false>;         \
+  }
+GSIM_KERNEL_TABLE(sim_full_kernel)
+GSIM_KERNEL_TABLE(sim_inc_kernel)
+GSIM_KERNEL_TABLE(sim_base_kernel)
+#undef GSIM_KERNEL_TABLE
+
+const void* full_kernel_ptr(bool reg, bool key) { return sim_full_kernel_ptr(reg, key); }
+const void* inc_kernel_ptr(bool reg, bool key) { return sim_inc_kernel_ptr(reg, key); }
 
 cudaError_t set_smem_limits(int smem) {
-  const void* fns[] = {(const void*)sim_full_kernel<true>, (const void*)sim_full_kernel<false>,
-                       (const void*)sim_inc_kernel<true>,  (const void*)sim_inc_kernel<false>,
-                       (const void*)sim_base_kernel<true>, (const void*)sim_base_kernel<false>};
-  for (const void* f : fns) {
-    const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-  }
+  for (int r = 0; r < 2; ++r)
+    for (int k = 0; k < 2; ++k) {
+      const void* fns[] = {sim_full_kernel_ptr(r, k), sim_inc_kernel_ptr(r, k), sim_base_kernel_ptr(r, k)};
+      for (const void* f : fns) {
+        const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+      }
+    }
   return cudaSuccess;
 }
 
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
-  if (reg) sim_full_kernel<true><<<grid, block, smem, st>>>(P);
-  else sim_full_kernel<false><<<grid, block, smem, st>>>(P);
+  const bool key = P.g.dev_key != 0;
+  if (reg) {
+    if (key) sim_full_kernel<true, true><<<grid, block, smem, st>>>(P);
+    else sim_full_kernel<true, false><<<grid, block, smem, st>>>(P);
+  } else {
+    if (key) sim_full_kernel<false, true><<<grid, block, smem, st>>>(P);
+    else sim_full_kernel<false, false><<<grid, block, smem, st>>>(P);
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
-  if (reg) sim_inc_kernel<true><<<grid, block, smem, st>>>(P);
-  else sim_inc_kernel<false><<<grid, block, smem, st>>>(P);
+  const bool key = P.g.dev_key != 0;
+  if (reg) {
+    if (key) sim_inc_kernel<true, true><<<grid, block, smem, st>>>(P);
+    else sim_inc_kernel<true, false><<<grid, block, smem, st>>>(P);
+  } else {
+    if (key) sim_inc_kernel<false, true><<<grid, block, smem, st>>>(P);
+    else sim_inc_kernel<false, false><<<grid, block, smem, st>>>(P);
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st) {
-  if (reg) sim_base_kernel<true><<<1, 32, smem, st>>>(P);
-  else sim_base_kernel<false><<<1, 32, smem, st>>>(P);
+  const bool key = P.g.dev_key != 0;
+  if (reg) {
+    if (key) sim_base_kernel<true, true><<<1, 32, smem, st>>>(P);
+    else sim_base_kernel<true, false><<<1, 32, smem, st>>>(P);
+  } else {
+    if (key) sim_base_kernel<false, true><<<1, 32, smem, st>>>(P);
+    else sim_base_kernel<false, false><<<1, 32, smem, st>>>(P);
+  }
   return cudaGetLastError();
 }
 

@@ -107,16 +107,22 @@ def test_golden_examples_on_gpu():
 
 
 def test_queue_capacity_status():
-    d, rows = _random_case(13, 120, 4)
+    # one op feeding 120 successors: 120 ready keys at once, beyond the
+    # 32-key register tier plus a 3-slot heap
+    n = 121
+    d = mk([[]] + [[0]] * 120, [5] * n, [1] * n, n_dev=4, bw=1, lat=1)
     g = G.gmg_create(d)
+    rows = np.zeros((8, 128), np.uint8)
+    rows[:, :n] = np.random.default_rng(0).integers(0, 4, (8, n))
     out = G.sim_batch(g, torch_place(rows), queue_cap=3)
+    ok = G.sim_batch(g, torch_place(rows))
     torch.cuda.synchronize()
     st = out.status.cpu().numpy()
-    assert (st == G.SIM_QUEUE).any()
-    sc = out.score.cpu().numpy()
-    assert (sc[st == G.SIM_QUEUE] == np.iinfo(np.int64).max).all()
-    best = G.select_best(out).cpu().tolist()
-    assert best[0] == -1 or st[best[0]] == 0
+    assert (st == G.SIM_QUEUE).all()
+    assert (out.score.cpu().numpy() == np.iinfo(np.int64).max).all()
+    assert G.select_best(out).cpu().tolist()[0] == -1
+    s, pk, rq = oracle_rows(d, rows)
+    compare(ok.to_numpy(), s, pk, rq)
 
 
 @pytest.mark.parametrize("wpb", [1, 2, 3, 4])
