@@ -33,6 +33,7 @@ constexpr uint32_t kAllCons = 4u;  // consumers = successors
 constexpr uint32_t kHoldBit = 0x80000000u;
 constexpr uint32_t kSibNone = 0xffffffffu;  // the only listed consumer
 constexpr uint32_t kSibMany = 0xfffffffeu;  // three or more listed consumers
+constexpr uint32_t kSibLater = 0x40000000u; // flag: the other consumer is a descendant
 constexpr uint32_t kIdMask = 0x7fffffffu;
 
 // Exact ceil(n / bw) by multiply-shift (Granlund & Montgomery 1994,

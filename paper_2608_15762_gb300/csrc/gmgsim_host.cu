@@ -217,14 +217,48 @@ int build(const gmg_desc_t* d, Built& b) {
   // For every (predecessor p -> holding consumer c) entry: the other listed
   // consumer of p, so that c can tell whether it is p's last one there.
   b.sib.assign(b.E, kSibNone);
+  // Bounded reachability along successors (ids are topological, so a search
+  // never needs to pass the target id); "unknown" simply keeps the run-time
+  // check.
+  std::vector<uint32_t> stack;
+  std::vector<int32_t> seen_at(n, -1);
+  int stamp = 0;
+  auto reaches = [&](uint32_t from, uint32_t to) {
+    ++stamp;
+    stack.assign(1, from);
+    int visited = 0;
+    while (!stack.empty() && visited < 256) {
+      const uint32_t x = stack.back();
+      stack.pop_back();
+      ++visited;
+      const OpRec& rx = b.ops[x];
+      for (uint32_t k = 0; k < rx.nsucc; ++k) {
+        const uint32_t y = b.succ[rx.succ_off + k];
+        if (y == to) return true;
+        if (y < to && seen_at[y] != stamp) {
+          seen_at[y] = stamp;
+          stack.push_back(y);
+        }
+      }
+    }
+    return false;
+  };
   for (int p = 0; p < n; ++p) {
     const OpRec& r = b.ops[p];
     const uint32_t* lst = (r.flags & kAllCons) ? b.succ.data() + r.succ_off : b.cons.data() + r.cons_off;
     for (uint32_t u = 0; u < r.ncons; ++u) {
       const uint32_t c = lst[u];
       uint32_t v = kSibNone;
-      if (r.ncons == 2) v = lst[1 - u];
-      else if (r.ncons > 2) v = kSibMany;
+      if (r.ncons == 2) {
+        const uint32_t o = lst[1 - u];
+        // A fixed finishing order between the two consumers (one depends on
+        // the other) settles the release without a run-time check.
+        if (o < c && reaches(o, c)) v = kSibNone;           // c always finishes last
+        else if (o > c && reaches(c, o)) v = o | kSibLater;  // o always finishes later
+        else v = o;
+      } else if (r.ncons > 2) {
+        v = kSibMany;
+      }
       for (uint32_t k = b.ops[c].pred_off; k < b.ops[c].pred_off + b.ops[c].npred; ++k)
         if ((b.pred[k] & kIdMask) == (uint32_t)p) b.sib[k] = v;
     }

@@ -369,7 +369,6 @@ struct Sim {
 
   // READY keys go to a free lane's register if there is one, else the heap.
   __device__ __forceinline__ void push_ready(uint64_t key) {
-    if (status) return;
     const uint32_t freel = __ballot_sync(kFullMask, rk_reg == kKeyMax);
     if (freel) {
       if ((int)lane_id() == __ffs(freel) - 1) rk_reg = key;
@@ -566,6 +565,9 @@ struct Sim {
           const uint32_t sb = ps.y;
           if (sb == kSibNone) {
             rel = true;
+          } else if (sb != kSibMany && (sb & kSibLater)) {
+            // the other consumer depends on this one: it finishes later
+            rel = row[sb & ~kSibLater] != d;
           } else if (sb != kSibMany) {
             rel = !(row[sb] == d && !popped(sb));
           } else {
@@ -680,38 +682,51 @@ struct Sim {
     settle_violation(vmin);
   }
 
+  // One compare-exchange stage of a bitonic network held in registers: the
+  // element of lane l (index l + 32 h) meets the one of lane l ^ j.
+  template <int K, int J, int H>
+  static __device__ __forceinline__ uint64_t bitonic_lane_stage(uint64_t a) {
+    const unsigned lane = lane_id();
+    const uint64_t o = __shfl_xor_sync(kFullMask, a, J);
+    const bool keep_min = ((lane & J) == 0) == (((lane + 32u * H) & K) == 0);
+    const bool lt = o < a;
+    return keep_min == lt ? o : a;
+  }
+
+  template <int K, int J>
+  static __device__ __forceinline__ void bitonic_stages(uint64_t& a0, uint64_t& a1, bool two) {
+    if (J == 32) {
+      const uint64_t lo = a0 < a1 ? a0 : a1;
+      a1 = a0 < a1 ? a1 : a0;
+      a0 = lo;
+    } else if (J > 0) {
+      a0 = bitonic_lane_stage<K, (J > 0 ? J : 1), 0>(a0);
+      if (two) a1 = bitonic_lane_stage<K, (J > 0 ? J : 1), 1>(a1);
+    }
+    if (J > 1) bitonic_stages<K, (J > 1 ? J / 2 : 0)>(a0, a1, two);
+  }
+
+  template <int K>
+  static __device__ __forceinline__ void bitonic_upto(uint64_t& a0, uint64_t& a1, bool two) {
+    if (K > 2) bitonic_upto<(K > 2 ? K / 2 : 2)>(a0, a1, two);
+    bitonic_stages<K, K / 2>(a0, a1, two);
+  }
+
   // Sort and apply m <= 64 extracted events in registers: lane l holds
   // elements l and 32 + l of a bitonic network.
   __device__ void sort_apply_regs(int m) {
     const unsigned lane = lane_id();
     uint64_t a0 = (int)lane < m ? sortk[lane] : kKeyMax;
     uint64_t a1 = (int)lane + 32 < m ? sortk[lane + 32] : kKeyMax;
-    const bool two = m > 32;
-    const int p2 = two ? 64 : 32;
-    for (int k = 2; k <= p2; k <<= 1) {
-      for (int j = k >> 1; j > 0; j >>= 1) {
-        if (j == 32) {
-          const uint64_t lo = a0 < a1 ? a0 : a1;
-          a1 = a0 < a1 ? a1 : a0;
-          a0 = lo;
-          continue;
-        }
-        const bool lower = (lane & j) == 0;
-        {
-          const uint64_t o = __shfl_xor_sync(kFullMask, a0, j);
-          const bool keep_min = lower == ((lane & k) == 0);
-          a0 = keep_min ? (o < a0 ? o : a0) : (o > a0 ? o : a0);
-        }
-        if (two) {
-          const uint64_t o = __shfl_xor_sync(kFullMask, a1, j);
-          const bool keep_min = lower == (((lane + 32) & k) == 0);
-          a1 = keep_min ? (o < a1 ? o : a1) : (o > a1 ? o : a1);
-        }
-      }
-    }
     uint64_t vmin = kKeyMax;
-    apply_chunk(a0, (int)lane < m, vmin);
-    if (two) apply_chunk(a1, (int)lane + 32 < m, vmin);
+    if (m > 32) {
+      bitonic_upto<64>(a0, a1, true);
+      apply_chunk(a0, true, vmin);
+      apply_chunk(a1, (int)lane + 32 < m, vmin);
+    } else {
+      bitonic_upto<32>(a0, a1, false);
+      apply_chunk(a0, (int)lane < m, vmin);
+    }
     settle_violation(vmin);
   }
 
