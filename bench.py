@@ -149,8 +149,7 @@ def prepare(config: int, rank: int, device):
     p.K = p.n_full + p.n_inc
     p.host_place = None
     if p.n_full:
-        ks = range(rank * p.n_full, (rank + 1) * p.n_full)
-        rows = wl.full_rows(ks)
+        rows = wl.full_rows(G.shard_range(rank, p.n_full))
         p.host_place = torch.from_numpy(rows).pin_memory()
         p.place = p.host_place.to(device)
     if p.n_inc:
@@ -362,7 +361,11 @@ def main():
 
     wl = p.wl
     K, N, D = p.K, wl.desc.n_ops, wl.desc.n_dev
-    best = p.best.cpu().tolist()
+    if world > 1:
+        from paper_2608_15762_gb300 import gmgsim as G
+        best = list(G.select_best_across_ranks(p.best, rank * p.n_full))
+    else:
+        best = p.best.cpu().tolist()
     value = world * K / (ms / 1000)
     kms = statistics.mean(kern_ms)
     # Roofline of the dominant kernel (the candidate simulation).

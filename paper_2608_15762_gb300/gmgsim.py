@@ -389,6 +389,33 @@ def select_best(out: SimOut, K: Optional[int] = None, score_mode: int = 0, best=
     return best
 
 
+def shard_range(rank: int, per_rank: int):
+    """Global candidate indices of one rank when every rank simulates its own
+    block of per_rank candidates (candidates are independent: no exchange)."""
+    return range(rank * per_rank, (rank + 1) * per_rank)
+
+
+def select_best_across_ranks(best, k_offset: int, group=None):
+    """Combine the ranks' select_best results into the best over all ranks'
+    candidates (lowest global index on ties; (-1, INT64_MAX) if none).
+
+    best: int64[2] (local index or -1, score) on this rank's device.  One
+    all_gather of 16 bytes per rank; call outside any timed region."""
+    import torch
+    import torch.distributed as dist
+    loc = best.detach().to(torch.int64).reshape(2).clone()
+    if int(loc[0]) >= 0:
+        loc[0] += k_offset
+    world = dist.get_world_size(group)
+    bufs = [torch.empty_like(loc) for _ in range(world)]
+    dist.all_gather(bufs, loc, group=group)
+    cands = [(int(b[1]), int(b[0])) for b in bufs if int(b[0]) >= 0]
+    if not cands:
+        return -1, int(np.iinfo(np.int64).max)
+    sc, k = min(cands)
+    return k, sc
+
+
 def ceil_div_host(n: int, d: int) -> int:
     return int(lib().gmg_ceil_div_host(n, d))
 

@@ -126,6 +126,19 @@ class Moves:
     def n_cand(self) -> int:
         return int(self.off.shape[0] - 1)
 
+    def subset(self, ks: Sequence[int]) -> "Moves":
+        """The move lists of candidates ks, in that order."""
+        off = [0]
+        ops, devs = [], []
+        for k in ks:
+            a, b = int(self.off[k]), int(self.off[k + 1])
+            ops.append(self.op[a:b])
+            devs.append(self.dev[a:b])
+            off.append(off[-1] + b - a)
+        return Moves(np.array(off, np.int32),
+                     np.concatenate(ops).astype(np.int32) if ops else np.zeros(0, np.int32),
+                     np.concatenate(devs).astype(np.uint8) if devs else np.zeros(0, np.uint8))
+
 
 @dataclass
 class Workload:

@@ -91,15 +91,7 @@ def test_workload_incremental_sampled():
     got = out.to_numpy()
     ks = np.random.default_rng(33).choice(mv.n_cand, 512, replace=False)
     ks.sort()
-    sub = W.Moves(np.zeros(len(ks) + 1, np.int32), None, None)
-    ops, devs = [], []
-    for i, k in enumerate(ks):
-        ops.extend(mv.op[mv.off[k]:mv.off[k + 1]].tolist())
-        devs.extend(mv.dev[mv.off[k]:mv.off[k + 1]].tolist())
-        sub.off[i + 1] = len(ops)
-    sub.op = np.array(ops, np.int32)
-    sub.dev = np.array(devs, np.uint8)
-    s, pk, rq = O.incremental_batch(wl.desc, wl.base_place, sub)
+    s, pk, rq = O.incremental_batch(wl.desc, wl.base_place, mv.subset(ks))
     compare(got, s, pk, rq, ks=ks)
     assert (got["status"] == 0).all()
     assert (got["events"] <= wl.desc.n_ops).all() and (got["events"] > 0).all()

@@ -183,13 +183,25 @@ def test_workload_memory_tight_sampled():
     assert (got["status"] == 0).all() and (got["events"] == wl.desc.n_ops).all()
 
 
-def test_workload_large_full_half_sampled():
+def test_workload_large_full_size_sampled():
+    """The 256-accelerator workload exactly as the benchmark runs it: every
+    full placement and every incremental candidate on the GPU, sampled
+    candidates of both halves checked against the oracle."""
     wl = W.config5()
-    ks = np.random.default_rng(55).choice(wl.n_full, 8, replace=False)
-    ks.sort()
     g = G.gmg_create(wl.desc)
-    rows = wl.full_rows(ks)
-    out = G.sim_batch(g, torch_place(rows), req_done=True)
+    out = G.sim_batch(g, torch_place(wl.all_full_rows()), req_done=True)
+    b = G.base_create(g, torch.from_numpy(wl.base_place).cuda())
+    off, op, dv = G.moves_to_device(wl.moves, "cuda")
+    inc = G.sim_incremental(g, b, off, op, dv, req_done=True)
+    best = G.select_best(out)
     torch.cuda.synchronize()
-    s, pk, rq = oracle_rows(wl.desc, rows)
-    compare(out.to_numpy(), s, pk, rq)
+    got, goti = out.to_numpy(), inc.to_numpy()
+    assert (got["status"] == 0).all() and (goti["status"] == 0).all()
+    rng = np.random.default_rng(55)
+    ks = np.sort(rng.choice(wl.n_full, 6, replace=False))
+    s, pk, rq = oracle_rows(wl.desc, wl.full_rows(ks))
+    compare(got, s, pk, rq, ks=ks)
+    ki = np.sort(rng.choice(wl.moves.n_cand, 6, replace=False))
+    si, pki, rqi = O.incremental_batch(wl.desc, wl.base_place, wl.moves.subset(ki))
+    compare(goti, si, pki, rqi, ks=ki)
+    assert best.cpu().tolist()[1] == int(got["score"].min())
