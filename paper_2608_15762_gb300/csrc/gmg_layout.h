@@ -159,7 +159,8 @@ struct SimParams {
   int32_t ms;            // HBM event log slots in shared memory per warp
   int32_t mcap;          // HBM event log slots per warp
   int32_t sortcap;       // sort area entries per warp (power of two, >= max(32, n_dev))
-  int32_t drain_trigger; // drain the log after this many new events
+  int32_t drain_trigger; // (unused by the drain schedule; kept for layout stability)
+  int32_t opcap;         // ops started between HBM-event generations (<= 32)
   int32_t n_trace;
   const int32_t* trace_k;
   const int32_t* move_off;

@@ -35,10 +35,11 @@ constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
 constexpr int kDefaultWarpsPerBlock = 4;
 constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
 constexpr int64_t kDefaultQueueCap = 1 << 16;
-constexpr int kSharedLogEntries = 160;
+constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
 constexpr int kSortCap = 128;             // power of two; raised to n_dev's power of two
 constexpr int kDrainTrigger = 48;
+constexpr int kOpsPerGeneration = 24;     // ~100 HBM events: one 128-key register sort
 constexpr int kCheckpoints = 256;
 constexpr int kCheckpointQueue = 4096;
 constexpr int kCheckpointLog = 8192;
@@ -400,7 +401,8 @@ int log_cap(const gmg* g, const sim_opts_t* o) {
 }
 
 size_t smem_per_warp(const SimParams& P) {
-  return align_up((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9, 16) + (size_t)P.g.D * 24;
+  return align_up((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 + (size_t)P.opcap * 4, 16) +
+         (size_t)P.g.D * 24;
 }
 
 bool g_smem_set = false;
@@ -421,6 +423,7 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   P.sortcap = kSortCap;
   while (P.sortcap < G.D) P.sortcap <<= 1;
   P.drain_trigger = kDrainTrigger;
+  P.opcap = kOpsPerGeneration;
   L.smem = (size_t)L.wpb * smem_per_warp(P);
   size_t o2 = 0;
   auto take = [&](size_t bytes) {

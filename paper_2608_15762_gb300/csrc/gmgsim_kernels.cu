@@ -260,6 +260,7 @@ struct Devices {
 // Shared-memory carve-up per warp: READY heap head, event-log head, sort
 // area, accelerator state.
 struct WarpSmem {
+  uint32_t* oplog;  // [opcap]
   uint64_t* heap;   // [qs]
   uint64_t* logk;   // [ms]
   uint64_t* sortk;  // [sortcap]
@@ -271,7 +272,8 @@ struct WarpSmem {
 __device__ __forceinline__ size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P, unsigned wib) {
-  const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9);
+  const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 +
+                              (size_t)P.opcap * 4);
   const size_t per = head + (size_t)P.g.D * 24;
   uint8_t* b = smem + per * wib;
   WarpSmem w;
@@ -280,6 +282,7 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
   w.sortk = w.logk + P.ms;
   w.logd = reinterpret_cast<uint8_t*>(w.sortk + P.sortcap);
   w.sortd = w.logd + P.ms;
+  w.oplog = reinterpret_cast<uint32_t*>(w.sortd + P.sortcap);
   w.dev = reinterpret_cast<int64_t*>(b + head);
   return w;
 }
@@ -298,6 +301,8 @@ struct Sim {
   uint64_t* sortk;
   uint8_t* sortd;
   int sortcap;
+  uint32_t* oplog;  // ops started since the last HBM-event generation
+  int opn;
   int ds;           // accelerator shift of a log entry
   uint64_t lowmask; // key part of a log entry
   Devices<kReg> dv;
@@ -362,10 +367,7 @@ struct Sim {
     }
     return h;
   }
-  __device__ __forceinline__ int64_t hold_of(uint32_t p, int dp) const {
-    if (kMode == kInc && rb[p] < Tc) return lane_hold(p, fb[p], dp);
-    return hold[p];
-  }
+
 
   // READY keys go to a free lane's register if there is one, else the heap.
   __device__ __forceinline__ void push_ready(uint64_t key) {
@@ -408,6 +410,7 @@ struct Sim {
     q.size = 0;
     rk_reg = kKeyMax;
     log.n = 0;
+    opn = 0;
     trig = P.drain_trigger;
     rootptr = 0;
     score = makespan = 0;
@@ -421,7 +424,8 @@ struct Sim {
   }
 
   // -------------------------------------------------------------------------
-  // READY(r, i): start op i (Sec. 3.3.2/3.3.3) and emit what follows from it.
+  // READY(r, i): start op i (Sec. 3.3.2/3.3.3), record it for HBM-event
+  // generation, and push the successors it makes ready.
   // -------------------------------------------------------------------------
   __device__ void start_op(uint32_t i, int64_t r) {
     const unsigned lane = lane_id();
@@ -430,7 +434,7 @@ struct Sim {
     const uint4 ls = op_lists(g.ops, i);
     const uint4 cs = op_cons(g.ops, i);
     const int64_t dur = db.x, bytes = db.y, xq = rx.y;
-    const uint32_t succ_off = ls.x, nsucc = ls.y, pred_off = ls.z, npred = ls.w;
+    const uint32_t succ_off = ls.x, nsucc = ls.y;
     const uint32_t flags = cs.w;
     const int d = row[i];
     const int64_t fd = dv.get_free(d);
@@ -443,35 +447,31 @@ struct Sim {
       if (flags & kReqSink)
         atomicMax(reinterpret_cast<unsigned long long*>(creq + (int32_t)cs.z), (unsigned long long)f);
       if (kMode == kBase) P.base.rb[i] = r;
+      oplog[opn] = i;
     }
+    ++opn;
     if (flags & kScored) score += f;
     makespan = f > makespan ? f : makespan;
     if (kMode != kInc || r >= T0) ++nev;
-    ++readypops;
-    // the op's own output is allocated when it starts
-    log_event(lane == 0, kc.make(s, kAlloc, i), d);
+    if (kMode == kBase) ++readypops;
     __syncwarp();
 
-    // Successors: transfers, readiness, receive copies.
-    int64_t hm = f;  // latest arrival of an outgoing transfer (or f)
-    bool local_succ = false;
+    // Successors: a successor is ready once every predecessor has finished;
+    // its ready time is the latest arrival over all of them.
     for (uint32_t c0 = 0; c0 < nsucc; c0 += 32) {
       const uint32_t t = c0 + lane;
-      const bool v = t < nsucc;
       uint32_t j = 0;
-      int dj = -1;
-      int64_t arr = f, rj = 0;
+      int64_t rj = 0;
       bool rdy = false;
-      if (v) {
+      if (t < nsucc) {
         j = __ldg(g.succ + succ_off + t);
-        dj = row[j];
+        const int dj = row[j];
+        int64_t arr = f;
         if (dj != d) arr = f + xfer(d, dj, bytes, xq);
         const longlong2 jrx = op_relxq(g.ops, j);
         const uint4 jls = op_lists(g.ops, j);
         rj = jrx.x > arr ? jrx.x : arr;
         rdy = true;
-        // ready once every other predecessor has finished; its ready time is
-        // the latest arrival over all of them
         if (jls.w > 1) {
           for (uint32_t k = 0; k < jls.w; ++k) {
             const uint32_t p = __ldg(g.pred + jls.z + k) & kIdMask;
@@ -493,109 +493,132 @@ struct Sim {
         m &= m - 1;
         push_ready(__shfl_sync(kFullMask, kc.make(rj, kReady, j), src));
       }
-      const bool rem = v && dj != d;
-      bool leader;
-      if (nsucc == 1) {
-        // one successor, on lane 0
-        leader = rem;
-        local_succ = __shfl_sync(kFullMask, v && dj == d, 0);
-        const int64_t a0 = __shfl_sync(kFullMask, rem ? arr : f, 0);
-        hm = a0 > hm ? a0 : hm;
-      } else {
-        local_succ |= __any_sync(kFullMask, v && dj == d);
-        const uint32_t peers = __match_any_sync(kFullMask, rem ? (uint32_t)dj : (256u + lane));
-        leader = rem && (__ffs(peers) - 1 == (int)lane);
-        if (leader && c0 > 0) {
-          for (uint32_t u = 0; u < c0; ++u)
-            if (row[__ldg(g.succ + succ_off + u)] == dj) {
-              leader = false;
-              break;
-            }
-        }
-        const int64_t hl = (int64_t)warp_max_u64(leader ? (uint64_t)arr : 0ull);
-        hm = hl > hm ? hl : hm;
-      }
-      // one receive copy per distinct remote accelerator, allocated when the
-      // transfer starts
-      log_event(leader, kc.make(f, kAlloc, i), dj);
-      if (!(flags & kAllCons)) {
-        // a receive copy with no listed consumer there is released on arrival
-        bool nocons = false;
-        if (leader) {
-          nocons = true;
-          for (uint32_t u = 0; u < cs.y; ++u)
-            if (row[__ldg(g.cons + cs.x + u)] == dj) {
-              nocons = false;
-              break;
-            }
-        }
-        log_event(nocons, kc.make(arr, kFree, i), dj);
-      }
     }
-    // The source copy: released now-known if no listed consumer is local,
-    // else by its last local consumer (which reads hold[i]).
-    bool local_cons = local_succ;
-    if (!(flags & kAllCons)) {
-      bool lc = false;
-      for (uint32_t c0 = 0; c0 < cs.y; c0 += 32) {
-        const uint32_t t = c0 + lane;
-        if (t < cs.y && row[__ldg(g.cons + cs.x + t)] == d) lc = true;
-      }
-      local_cons = __any_sync(kFullMask, lc);
-    }
-    if (local_cons) {
-      if (lane == 0) hold[i] = hm;
-    } else {
-      log_event(lane == 0, kc.make(hm, kFree, i), d);
-    }
+  }
 
-    // Inputs held by this op: if it is the last listed consumer of a
-    // predecessor's output on this accelerator, that copy is released at f
-    // (the source copy not before the predecessor's transfers arrived).
-    for (uint32_t c0 = 0; c0 < npred; c0 += 32) {
-      const uint32_t t = c0 + lane;
-      bool rel = false;
-      int64_t T = f;
-      uint32_t p = 0;
-      if (t < npred) {
-        const uint2 ps = __ldg(g.predsib + pred_off + t);
-        const uint32_t pe = ps.x;
-        p = pe & kIdMask;
-        if (pe & kHoldBit) {
-          const uint32_t sb = ps.y;
-          if (sb == kSibNone) {
-            rel = true;
-          } else if (sb != kSibMany && (sb & kSibLater)) {
-            // the other consumer depends on this one: it finishes later
-            rel = row[sb & ~kSibLater] != d;
-          } else if (sb != kSibMany) {
-            rel = !(row[sb] == d && !popped(sb));
+  // -------------------------------------------------------------------------
+  // HBM events of the ops started since the last generation, one op per lane
+  // (Sec. 3.3.2 residency, Recv before Send of Sec. 3.5.2): the op's own
+  // output allocated at s; a receive copy on every other accelerator of a
+  // successor allocated at f (released on arrival if no listed consumer is
+  // there); the own copy released at the latest outgoing arrival if no
+  // listed consumer is local; and for every held input whose last local
+  // consumer this op is, that copy released at f (an own copy not before its
+  // producer's outgoing arrivals).  Ops on one accelerator finish in the
+  // order they start, so "last consumer here" compares finish times and can
+  // be decided any time after the op started.
+  // -------------------------------------------------------------------------
+  __device__ void generate() {
+    const unsigned lane = lane_id();
+    for (int c0 = 0; c0 < opn; c0 += 32) {
+      const int idx = c0 + (int)lane;
+      const bool v = idx < opn;
+      const uint32_t x = v ? oplog[idx] : 0u;
+      longlong2 db = make_longlong2(0, 0), rx = make_longlong2(0, 0);
+      uint4 ls = make_uint4(0, 0, 0, 0), cs = make_uint4(0, 0, 0, 0);
+      int d = 0;
+      int64_t f = 0;
+      if (v) {
+        db = op_durbytes(g.ops, x);
+        rx = op_relxq(g.ops, x);
+        ls = op_lists(g.ops, x);
+        cs = op_cons(g.ops, x);
+        d = row[x];
+        f = fbuf[x];
+      }
+      const int64_t bytes = db.y, xq = rx.y;
+      const bool allcons = (cs.w & kAllCons) != 0;
+      log_event(v, kc.make(f - db.x, kAlloc, x), d);
+      // receive copies, one per distinct remote accelerator
+      int64_t hold = f;
+      bool localc = false;
+      const uint32_t nsx = ls.y;
+      const uint32_t maxs = __reduce_max_sync(kFullMask, nsx);
+      const bool anyexp = __any_sync(kFullMask, v && !allcons);
+      for (uint32_t u = 0; u < maxs; ++u) {
+        bool want = false, nocons = false;
+        int du = 0;
+        int64_t arr = f;
+        if (u < nsx) {
+          du = row[__ldg(g.succ + ls.x + u)];
+          if (du == d) {
+            localc = true;
           } else {
-            const uint4 pls = op_lists(g.ops, p);
-            const uint4 pcs = op_cons(g.ops, p);
-            const bool all = (pcs.w & kAllCons) != 0;
-            const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
-            const uint32_t nl = all ? pls.y : pcs.y;
-            rel = true;
-            for (uint32_t u = 0; u < nl; ++u) {
-              const uint32_t c = __ldg(lst + u);
-              if (c != i && row[c] == d && !popped(c)) {
-                rel = false;
+            want = true;
+            for (uint32_t w = 0; w < u; ++w)
+              if (row[__ldg(g.succ + ls.x + w)] == du) {
+                want = false;
                 break;
+              }
+            if (want) {
+              arr = f + xfer(d, du, bytes, xq);
+              hold = arr > hold ? arr : hold;
+              if (!allcons) {
+                nocons = true;
+                for (uint32_t w = 0; w < cs.y; ++w)
+                  if (row[__ldg(g.cons + cs.x + w)] == du) {
+                    nocons = false;
+                    break;
+                  }
               }
             }
           }
-          if (rel) {
-            const int dp = row[p];
-            if (dp == d) {
-              const int64_t h = hold_of(p, dp);
+        }
+        log_event(want, kc.make(f, kAlloc, x), du);
+        if (anyexp) log_event(nocons, kc.make(arr, kFree, x), du);
+      }
+      if (v && !allcons) {
+        localc = false;
+        for (uint32_t w = 0; w < cs.y; ++w)
+          if (row[__ldg(g.cons + cs.x + w)] == d) {
+            localc = true;
+            break;
+          }
+      }
+      log_event(v && !localc, kc.make(hold, kFree, x), d);
+      // releases of the inputs this op holds
+      const uint32_t npx = ls.w;
+      const uint32_t maxp = __reduce_max_sync(kFullMask, npx);
+      for (uint32_t u = 0; u < maxp; ++u) {
+        bool rel = false;
+        int64_t T = f;
+        uint32_t p = 0;
+        if (u < npx) {
+          const uint2 ps = __ldg(g.predsib + ls.z + u);
+          p = ps.x & kIdMask;
+          if (ps.x & kHoldBit) {
+            const uint32_t sb = ps.y;
+            if (sb == kSibNone) {
+              rel = true;
+            } else if (sb != kSibMany && (sb & kSibLater)) {
+              rel = row[sb & ~kSibLater] != d;  // the other consumer finishes later
+            } else if (sb != kSibMany) {
+              rel = !(row[sb] == d && !(popped(sb) && fin(sb) < f));
+            } else {
+              const uint4 pls = op_lists(g.ops, p);
+              const uint4 pcs = op_cons(g.ops, p);
+              const bool all = (pcs.w & kAllCons) != 0;
+              const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
+              const uint32_t nl = all ? pls.y : pcs.y;
+              rel = true;
+              for (uint32_t w = 0; w < nl; ++w) {
+                const uint32_t c = __ldg(lst + w);
+                if (c != x && row[c] == d && !(popped(c) && fin(c) < f)) {
+                  rel = false;
+                  break;
+                }
+              }
+            }
+            if (rel && row[p] == d) {
+              const int64_t h = lane_hold(p, fin(p), d);
               T = h > T ? h : T;
             }
           }
         }
+        log_event(rel, kc.make(T, kFree, p), d);
       }
-      log_event(rel, kc.make(T, kFree, p), d);
     }
+    opn = 0;
     __syncwarp();
   }
 
@@ -682,52 +705,58 @@ struct Sim {
     settle_violation(vmin);
   }
 
-  // One compare-exchange stage of a bitonic network held in registers: the
-  // element of lane l (index l + 32 h) meets the one of lane l ^ j.
-  template <int K, int J, int H>
-  static __device__ __forceinline__ uint64_t bitonic_lane_stage(uint64_t a) {
-    const unsigned lane = lane_id();
-    const uint64_t o = __shfl_xor_sync(kFullMask, a, J);
-    const bool keep_min = ((lane & J) == 0) == (((lane + 32u * H) & K) == 0);
-    const bool lt = o < a;
-    return keep_min == lt ? o : a;
-  }
-
-  template <int K, int J>
-  static __device__ __forceinline__ void bitonic_stages(uint64_t& a0, uint64_t& a1, bool two) {
-    if (J == 32) {
-      const uint64_t lo = a0 < a1 ? a0 : a1;
-      a1 = a0 < a1 ? a1 : a0;
-      a0 = lo;
-    } else if (J > 0) {
-      a0 = bitonic_lane_stage<K, (J > 0 ? J : 1), 0>(a0);
-      if (two) a1 = bitonic_lane_stage<K, (J > 0 ? J : 1), 1>(a1);
+  // Bitonic sort of 32*E keys held in registers: lane l holds elements
+  // l + 32 e.  Pairs 32 or more apart meet inside a lane, closer pairs via
+  // shfl_xor.  Fully unrolled.
+  template <int E>
+  static __device__ __forceinline__ void reg_bitonic(uint64_t (&a)[E]) {
+    const int lane = (int)lane_id();
+#pragma unroll
+    for (int k = 2; k <= 32 * E; k <<= 1) {
+#pragma unroll
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        if (j >= 32) {
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const int e2 = e ^ (j >> 5);
+            if (e2 > e) {
+              const bool asc = ((lane + 32 * e) & k) == 0;
+              const uint64_t x = a[e], y = a[e2];
+              const bool sw = asc ? (x > y) : (x < y);
+              a[e] = sw ? y : x;
+              a[e2] = sw ? x : y;
+            }
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const uint64_t o = __shfl_xor_sync(kFullMask, a[e], j);
+            const bool keep_min = ((lane & j) == 0) == (((lane + 32 * e) & k) == 0);
+            a[e] = (keep_min == (o < a[e])) ? o : a[e];
+          }
+        }
+      }
     }
-    if (J > 1) bitonic_stages<K, (J > 1 ? J / 2 : 0)>(a0, a1, two);
   }
 
-  template <int K>
-  static __device__ __forceinline__ void bitonic_upto(uint64_t& a0, uint64_t& a1, bool two) {
-    if (K > 2) bitonic_upto<(K > 2 ? K / 2 : 2)>(a0, a1, two);
-    bitonic_stages<K, K / 2>(a0, a1, two);
-  }
-
-  // Sort and apply m <= 64 extracted events in registers: lane l holds
-  // elements l and 32 + l of a bitonic network.
-  __device__ void sort_apply_regs(int m) {
-    const unsigned lane = lane_id();
-    uint64_t a0 = (int)lane < m ? sortk[lane] : kKeyMax;
-    uint64_t a1 = (int)lane + 32 < m ? sortk[lane + 32] : kKeyMax;
+  template <int E>
+  __device__ __forceinline__ void sort_apply_regs_e(int m) {
+    const int lane = (int)lane_id();
+    uint64_t a[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) a[e] = lane + 32 * e < m ? sortk[lane + 32 * e] : kKeyMax;
+    reg_bitonic<E>(a);
     uint64_t vmin = kKeyMax;
-    if (m > 32) {
-      bitonic_upto<64>(a0, a1, true);
-      apply_chunk(a0, true, vmin);
-      apply_chunk(a1, (int)lane + 32 < m, vmin);
-    } else {
-      bitonic_upto<32>(a0, a1, false);
-      apply_chunk(a0, (int)lane < m, vmin);
-    }
+#pragma unroll
+    for (int e = 0; e < E; ++e) apply_chunk(a[e], lane + 32 * e < m, vmin);
     settle_violation(vmin);
+  }
+
+  // Sort and apply m <= 128 extracted events in registers.
+  __device__ void sort_apply_regs(int m) {
+    if (m <= 32) sort_apply_regs_e<1>(m);
+    else if (m <= 64) sort_apply_regs_e<2>(m);
+    else sort_apply_regs_e<4>(m);
   }
 
   __device__ int count_below(uint64_t kmax) const {
@@ -814,6 +843,7 @@ struct Sim {
 
   // Apply every logged event that can no longer be preceded (time < t_next).
   __device__ void drain(int64_t t_next) {
+    generate();
     const uint64_t lim = t_next == kI64Max ? kKeyMax : kc.time_floor(t_next);
     while (log.n > 0) {
       uint64_t kmax = lim;
@@ -842,7 +872,7 @@ struct Sim {
       }
       const int m = extract(kmax);
       if (m == 0) break;
-      if (kKey && m <= 64) {
+      if (kKey && m <= 128) {
         sort_apply_regs(m);
       } else {
         sort_area(m);
@@ -867,7 +897,7 @@ struct Sim {
       nk = rm < nk ? rm : nk;
       if (kMode == kBase) maybe_checkpoint(nk);
       if (nk == kKeyMax) break;
-      if (log.n >= trig) drain(kc.time(nk));
+      if (opn >= P.opcap) drain(kc.time(nk));
       if (nk == rm) {
         if (rk_reg == rm) rk_reg = kKeyMax;  // keys are unique
       } else if (nk == rk) {
@@ -992,6 +1022,7 @@ __device__ void Sim<kReg, kMode, kKey>::maybe_checkpoint(uint64_t next_key) {
   const int64_t tn = kc.time(next_key);
   if (tn <= last_t) return;
   const unsigned lane = lane_id();
+  generate();
   const bool hasreg = rk_reg != kKeyMax;
   const uint32_t regm = __ballot_sync(kFullMask, hasreg);
   const int nready = q.size + __popc(regm);
@@ -1045,6 +1076,8 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey>& S, const SimParams& P, unsign
   S.log.n = 0;
   S.sortk = w.sortk;
   S.sortd = w.sortd;
+  S.oplog = w.oplog;
+  S.opn = 0;
   S.sortcap = P.sortcap;
   S.fbuf = reinterpret_cast<int64_t*>(sl + P.off_f);
   S.hold = reinterpret_cast<int64_t*>(sl + P.off_hold);
@@ -1250,6 +1283,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey>& S, const SimParams& P, int6
   S.status = GMG_SIM_OK;
   S.trig = P.drain_trigger;
   S.rk_reg = kKeyMax;
+  S.opn = 0;
   S.dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
   for (int r = lane; r < g.R; r += 32) S.creq[r] = B.ck_creq[(int64_t)c * g.R + r];
   for (int w = lane; w < words; w += 32) S.bits[w] = B.ck_bits[(int64_t)c * B.ck_words + w];
