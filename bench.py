@@ -33,7 +33,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "candidate placements simulated/sec (and op-events/sec) vs HBM/issue roofline"
 UNIT = "candidates/s"
-PROFILE = os.path.join(ROOT, "profiles", "sim_full_kernel_prefill_N3088_K4096.txt")
+PROFILE_DIR = os.path.join(ROOT, "profiles")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2608_15762_gb300", "csrc", f)
                   for f in ("gmgsim_kernels.cu", "gmg_layout.h")]
 
@@ -46,13 +46,19 @@ def kernel_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def read_profile():
-    """Instruction and DRAM counts per launch of the dominant kernel from the
-    committed ncu summary, if it was taken on the current kernel source."""
-    if not os.path.exists(PROFILE):
+def profile_path(kernel: str, workload: str) -> str:
+    return os.path.join(PROFILE_DIR, "%s_%s.txt" % (kernel, workload))
+
+
+def read_profile(path: str):
+    """Instruction and DRAM counts per candidate of the dominant kernel from
+    the committed ncu summary of that kernel on this workload (captured on
+    `candidates_per_launch` candidates), if it was taken on the current kernel
+    source."""
+    if not os.path.exists(path):
         return None
     vals = {}
-    with open(PROFILE) as f:
+    with open(path) as f:
         for line in f:
             if ":" in line:
                 k, v = line.split(":", 1)
@@ -60,9 +66,10 @@ def read_profile():
     if vals.get("kernel_source_sha256") != kernel_hash():
         return None
     try:
-        return {"inst": float(vals["inst_executed_per_launch"]),
-                "dram": float(vals["dram_bytes_per_launch"])}
-    except (KeyError, ValueError):
+        c = float(vals["candidates_per_launch"])
+        return {"inst_per_cand": float(vals["inst_executed_per_launch"]) / c,
+                "dram_per_cand": float(vals["dram_bytes_per_launch"]) / c, "captured": int(c)}
+    except (KeyError, ValueError, ZeroDivisionError):
         return None
 
 
@@ -135,7 +142,7 @@ class Prepared:
     pass
 
 
-def prepare(config: int, rank: int, device):
+def prepare(config: int, rank: int, device, cap=None):
     import numpy as np
     import torch
     from paper_2608_15762_gb300 import gmgsim as G
@@ -146,17 +153,24 @@ def prepare(config: int, rank: int, device):
     p.g = G.gmg_create(wl.desc, device=device)
     p.n_full = wl.n_full
     p.n_inc = 0 if wl.moves is None else wl.moves.n_cand
+    moves = wl.moves
+    if cap is not None:
+        # profiling captures: the first `cap` candidates of each half
+        p.n_full = min(p.n_full, cap)
+        if p.n_inc > cap:
+            moves = moves.subset(np.arange(cap))
+            p.n_inc = cap
     p.K = p.n_full + p.n_inc
     p.host_place = None
     if p.n_full:
-        rows = wl.full_rows(G.shard_range(rank, p.n_full))
+        rows = wl.full_rows(range(p.n_full)) if cap is not None else wl.full_rows(G.shard_range(rank, p.n_full))
         p.host_place = torch.from_numpy(rows).pin_memory()
         p.place = p.host_place.to(device)
     if p.n_inc:
         p.host_base = torch.from_numpy(np.ascontiguousarray(wl.base_place)).pin_memory()
         p.base_place = p.host_base.to(device)
         p.host_moves = [torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
-                        for a in (wl.moves.off, wl.moves.op, wl.moves.dev)]
+                        for a in (moves.off, moves.op, moves.dev)]
         p.moves = [t.to(device) for t in p.host_moves]
     p.out = G.SimOut.empty(p.K, wl.desc.n_dev, wl.desc.n_req, device)
     p.scratch = G.Scratch(device)
@@ -292,6 +306,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--candidates", type=int, default=None,
+                    help="profiling aid: simulate only the first N candidates of each half "
+                         "(the line then describes that smaller batch)")
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -310,7 +327,7 @@ def main():
 
     from paper_2608_15762_gb300 import build as lib_build
     lib_build.build()
-    p = prepare(args.config, rank, device)
+    p = prepare(args.config, rank, device, cap=args.candidates)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
 
     def barrier():
@@ -370,26 +387,35 @@ def main():
     kms = statistics.mean(kern_ms)
     # Roofline of the dominant kernel (the candidate simulation).
     pk = peaks()
+    # the timed kernel: the full-placement simulation if the batch has one,
+    # else the incremental one
+    kern = "sim_full_kernel" if p.n_full else "sim_inc_kernel"
+    kcand = p.n_full if p.n_full else p.n_inc
     out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
-    alg_bytes = (p.n_full * W_ld(N) if p.n_full else 0) + K * out_bytes_per_cand
+    if p.n_full:
+        alg_bytes = p.n_full * (W_ld(N) + out_bytes_per_cand)
+    else:
+        alg_bytes = sum(t.numel() * t.element_size() for t in p.host_moves) + p.n_inc * out_bytes_per_cand
     hbm_gbs = alg_bytes / (kms / 1000) / 1e9
     props = torch.cuda.get_device_properties(device)
     issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
-    prof = read_profile() if args.config == 2 else None
+    ppath = profile_path(kern, wl.name)
+    prof = read_profile(ppath)
     roof = {"bound": "alu", "unit": "Ginst/s", "peak": issue_peak,
             "peak_src": "%d SMs x 4 issue slots x %.0f MHz (%s sm_max_mhz)" % (
                 props.multi_processor_count, pk["sm_max_mhz"], pk["src"]),
-            "achieved": None, "frac": None, "traffic": None,
-            "kernel": "sim_full_kernel" if p.n_full else "sim_inc_kernel",
-            "kernel_ms": kms}
+            "achieved": None, "frac": None, "traffic": None, "kernel": kern, "kernel_ms": kms}
     if prof:
-        ach = prof["inst"] / (kms / 1000) / 1e9
-        roof.update(achieved=ach, frac=ach / issue_peak, traffic=prof["dram"],
-                    inst_per_launch=prof["inst"], inst_src=os.path.relpath(PROFILE, ROOT))
+        inst = prof["inst_per_cand"] * kcand
+        ach = inst / (kms / 1000) / 1e9
+        roof.update(achieved=ach, frac=ach / issue_peak, traffic=prof["dram_per_cand"] * kcand,
+                    inst_per_launch=inst, inst_src="%s (ncu on %d candidates, scaled to %d)" % (
+                        os.path.relpath(ppath, ROOT), prof["captured"], kcand))
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+        "ms_per_step_best": min(step_ms), "ms_per_step_median": statistics.median(step_ms),
         "config": {"workload": wl.name, "candidates": K, "n_ops": N, "n_dev": D,
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
                    "parallelism": "dp%d over candidates" % world},

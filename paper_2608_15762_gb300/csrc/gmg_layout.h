@@ -124,7 +124,6 @@ struct DevBase {
   uint8_t* row;          // [ld] base placement
   int64_t* rb;           // [N] base ready time
   int64_t* fb;           // [N] base finish time
-  int64_t* hb;           // [N] base hold time (latest outgoing arrival)
   int32_t* status;       // [1]
   // base results (outputs of the base placement)
   int64_t* res_scalars;  // [8]: makespan, score, viol_flag, viol_op, viol_dev, viol_time, sla_miss, n_ck
@@ -169,7 +168,7 @@ struct SimParams {
   uint8_t* scratch;
   int64_t slot_bytes;    // scratch bytes per warp slot
   // byte offsets inside a slot
-  int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row;
+  int64_t off_f, off_bits, off_creq, off_qk, off_mk, off_md, off_row;
 };
 
 }  // namespace gsim

@@ -434,7 +434,6 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   const int64_t qspill = std::max<int64_t>(P.qcap - P.qs, 0);
   const int64_t mspill = std::max<int64_t>(P.mcap - P.ms, 0);
   P.off_f = take(8 * (size_t)G.n);
-  P.off_hold = take(8 * (size_t)G.n);
   P.off_bits = take(4 * (size_t)((G.n + 31) / 32) + 16);
   P.off_creq = take(8 * (size_t)G.R);
   P.off_qk = take(8 * (size_t)qspill);
@@ -498,7 +497,7 @@ void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
 }
 
 struct BasePlan {
-  size_t off_row, off_rb, off_fb, off_hb, off_status, off_res, off_peak, off_creq, off_cktime,
+  size_t off_row, off_rb, off_fb, off_status, off_res, off_peak, off_creq, off_cktime,
       off_cksc, off_ckdev, off_ckcreq, off_ckqk, off_ckmk, off_ckmd, off_ckbits, off_slot, total;
   int nck, ckq, ckm, ckw, ld, stride;
   Launch L;
@@ -526,7 +525,6 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   B.off_row = take(B.ld);
   B.off_rb = take(8 * (size_t)G.n);
   B.off_fb = take(8 * (size_t)G.n);
-  B.off_hb = take(8 * (size_t)G.n);
   B.off_status = take(16);
   B.off_res = take(64);
   B.off_peak = take(8 * (size_t)G.D);
@@ -774,7 +772,6 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   D.row = w + B.off_row;
   D.rb = reinterpret_cast<int64_t*>(w + B.off_rb);
   D.fb = reinterpret_cast<int64_t*>(w + B.off_fb);
-  D.hb = reinterpret_cast<int64_t*>(w + B.off_hb);
   D.status = reinterpret_cast<int32_t*>(w + B.off_status);
   D.res_scalars = reinterpret_cast<int64_t*>(w + B.off_res);
   D.res_peak = reinterpret_cast<int64_t*>(w + B.off_peak);

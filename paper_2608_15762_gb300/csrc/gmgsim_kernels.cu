@@ -308,7 +308,6 @@ struct Sim {
   Devices<kReg> dv;
   const uint8_t* row;
   int64_t* fbuf;
-  int64_t* hold;
   uint32_t* bits;
   int64_t* creq;
   // incremental resume
@@ -1080,7 +1079,6 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey>& S, const SimParams& P, unsign
   S.opn = 0;
   S.sortcap = P.sortcap;
   S.fbuf = reinterpret_cast<int64_t*>(sl + P.off_f);
-  S.hold = reinterpret_cast<int64_t*>(sl + P.off_hold);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
   S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
   S.dv.setup(P.g, w.dev);
@@ -1126,7 +1124,6 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
     *reinterpret_cast<uint4*>(B.row + c) = *reinterpret_cast<const uint4*>(P.place + c);
   for (int c = lane; c < B.nck; c += 32) B.ck_time[c] = kI64Max;
   S.fbuf = B.fb;
-  S.hold = B.hb;
   S.row = P.place;
   __syncwarp();
   if (S.row_has_bad_device(P.place)) {

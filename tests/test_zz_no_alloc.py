@@ -52,8 +52,17 @@ def test_same_results_as_sim_batch_on_two_calls(which):
             assert np.array_equal(a[f], b[f]), f
 
 
+def _noalloc_bytes():
+    """GMG_NOALLOC_SCRATCH_BYTES as include/gmgsim.h defines it."""
+    import os
+    import re
+    hdr = os.path.join(os.path.dirname(__file__), "..", "include", "gmgsim.h")
+    m = re.search(r"#define GMG_NOALLOC_SCRATCH_BYTES \(\(size_t\)(\d+) << (\d+)\)", open(hdr).read())
+    return int(m.group(1)) << int(m.group(2))
+
+
 def test_refuses_a_graph_whose_scratch_does_not_fit():
-    n = 3 << 20   # one warp's scratch alone is ~16 bytes per op: > 32 MiB
+    n = 5 << 20   # a chain whose one-warp scratch (a finish time per op, ...) exceeds 32 MiB
     pred_off = np.arange(n + 1, dtype=np.int32) - 1
     pred_off[0] = 0
     desc = W.GmgDesc(n_dev=2, pred_off=pred_off, pred_idx=np.arange(n - 1, dtype=np.int32),
@@ -64,6 +73,7 @@ def test_refuses_a_graph_whose_scratch_does_not_fit():
                      avail0=np.zeros(2, np.int64), bw=np.ones(4, np.int64),
                      lat=np.zeros(4, np.int64)).normalized()
     g = G.gmg_create(desc)
+    assert G.sim_scratch_bytes(g, 1) > _noalloc_bytes()
     place = torch.zeros((1, W.placement_ld(n)), dtype=torch.uint8, device="cuda")
     out = G.SimOut.empty(1, 2, 0, place.device)
     co = out._c()
