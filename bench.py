@@ -378,6 +378,7 @@ def main():
 
     wl = p.wl
     K, N, D = p.K, wl.desc.n_ops, wl.desc.n_dev
+    inc_events = int(p.out.events[p.n_full:].sum().item()) if p.n_inc else 0
     if world > 1:
         from paper_2608_15762_gb300 import gmgsim as G
         best = list(G.select_best_across_ranks(p.best, rank * p.n_full))
@@ -419,7 +420,9 @@ def main():
         "config": {"workload": wl.name, "candidates": K, "n_ops": N, "n_dev": D,
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
                    "parallelism": "dp%d over candidates" % world},
-        "op_events_per_s": world * (p.n_full * N) / (ms / 1000) if p.n_full else None,
+        # full placements simulate every op; an incremental candidate re-simulates
+        # the ops its `events` output counts (read after the timed region)
+        "op_events_per_s": world * (p.n_full * N + inc_events) / (ms / 1000),
         "roofline": roof,
         "hbm": {"achieved": hbm_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
                 "frac": hbm_gbs / pk["hbm_gbs"], "algorithmic_bytes_per_launch": alg_bytes,
