@@ -92,6 +92,7 @@ struct DevGmg {
   int32_t ib;                 // op-id bits of a packed key
   int32_t tb;                 // time bits needed (every time < 2^tb)
   int32_t dev_key;            // 1 if an accelerator id fits above (time, class, op) in 64 bits
+  int32_t t32;                // 1 if every time is below 2^31 (the kernels then use int32 times)
   int32_t uniform;
 };
 

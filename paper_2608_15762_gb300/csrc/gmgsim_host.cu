@@ -15,8 +15,8 @@
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
 size_t select_rank_bytes();
-const void* full_kernel_ptr(bool reg, bool key);
-const void* inc_kernel_ptr(bool reg, bool key);
+const void* full_kernel_ptr(bool reg, bool key, bool t32);
+const void* inc_kernel_ptr(bool reg, bool key, bool t32);
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
@@ -452,7 +452,8 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     g_smem_set = true;
   }
   int bps = 0;
-  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0) : full_kernel_ptr(L.reg, G.dev_key != 0);
+  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0)
+                       : full_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0);
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
     return GMG_ECUDA;
   bps = std::max(bps, 1);
@@ -616,6 +617,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.tb = 1;
   while (G.tb < 62 && (int64_t(1) << G.tb) <= b.time_bound) ++G.tb;
   G.dev_key = (G.tb + G.ib + 2 + 8 <= 63) ? 1 : 0;
+  G.t32 = G.tb <= 31 ? 1 : 0;  // every time < 2^tb fits int32
   G.uniform = b.uniform ? 1 : 0;
   gmg_info_t& I = g->info;
   std::memset(&I, 0, sizeof(I));

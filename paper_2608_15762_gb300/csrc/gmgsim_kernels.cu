@@ -42,6 +42,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <type_traits>
+
 #include "gmg_layout.h"
 
 namespace gsim {
@@ -85,8 +87,10 @@ __device__ __forceinline__ uint4 op_cons(const OpRec* ops, uint32_t i) {
 struct KeyCodec {
   int ib;
   uint64_t mask;
-  __device__ __forceinline__ uint64_t make(int64_t t, uint32_t cls, uint32_t op) const {
-    return ((uint64_t)t << (ib + 2)) | ((uint64_t)cls << ib) | (uint64_t)op;
+  template <typename TM>
+  __device__ __forceinline__ uint64_t make(TM t, uint32_t cls, uint32_t op) const {
+    using U = typename std::make_unsigned<TM>::type;
+    return ((uint64_t)(U)t << (ib + 2)) | ((uint64_t)cls << ib) | (uint64_t)op;
   }
   __device__ __forceinline__ int64_t time(uint64_t k) const { return (int64_t)(k >> (ib + 2)); }
   __device__ __forceinline__ uint64_t time_floor(int64_t t) const { return (uint64_t)t << (ib + 2); }
@@ -180,9 +184,9 @@ struct MemLog {
 // holds accelerator d's in a register, else a shared array.  Live and peak
 // bytes: shared arrays (the drain updates them a batch at a time).
 // ---------------------------------------------------------------------------
-template <bool kReg>
+template <bool kReg, typename TM>
 struct Devices {
-  int64_t fr_reg;
+  TM fr_reg;
   int64_t* fr;  // shared [D] (when !kReg)
   int64_t* lv;  // shared [D]
   int64_t* pk;  // shared [D]
@@ -200,14 +204,14 @@ struct Devices {
       pk[d] = g.base[d];
       if (!kReg) fr[d] = g.avail0[d];
     }
-    if (kReg) fr_reg = l < (unsigned)D ? g.avail0[l] : 0;
+    if (kReg) fr_reg = l < (unsigned)D ? (TM)g.avail0[l] : (TM)0;
     __syncwarp();
   }
-  __device__ __forceinline__ int64_t get_free(int d) const {
+  __device__ __forceinline__ TM get_free(int d) const {
     if (kReg) return __shfl_sync(kFullMask, fr_reg, d);
-    return fr[d];
+    return (TM)fr[d];
   }
-  __device__ __forceinline__ void set_free(int d, int64_t v) {
+  __device__ __forceinline__ void set_free(int d, TM v) {
     if (kReg) {
       if ((int)lane_id() == d) fr_reg = v;
     } else {
@@ -240,7 +244,7 @@ struct Devices {
       dst[D + d] = lv[d];
       dst[2 * D + d] = pk[d];
     }
-    if (kReg && l < (unsigned)D) dst[l] = fr_reg;
+    if (kReg && l < (unsigned)D) dst[l] = (int64_t)fr_reg;
   }
   __device__ void load(const int64_t* src) {
     const unsigned l = lane_id();
@@ -249,7 +253,7 @@ struct Devices {
       lv[d] = src[D + d];
       pk[d] = src[2 * D + d];
     }
-    if (kReg) fr_reg = l < (unsigned)D ? src[l] : 0;
+    if (kReg) fr_reg = l < (unsigned)D ? (TM)src[l] : (TM)0;
     __syncwarp();
   }
   __device__ void write_peak(int64_t* dst) const {
@@ -290,8 +294,13 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
 // ---------------------------------------------------------------------------
 // One warp's simulator.
 // ---------------------------------------------------------------------------
-template <bool kReg, int kMode, bool kKey>
+// kT32: every time of the graph is below 2^31 (the host's bound), so ready,
+// start, finish, free and arrival times are carried as int32 (bytes, scores
+// and outputs stay int64).
+template <bool kReg, int kMode, bool kKey, bool kT32 = false>
 struct Sim {
+  static_assert(!(kT32 && kMode == kBase), "the base snapshot keeps 64-bit times");
+  using tm_t = typename std::conditional<kT32, int32_t, int64_t>::type;
   const SimParams& P;
   const DevGmg& g;
   KeyCodec kc;
@@ -305,18 +314,19 @@ struct Sim {
   int opn;
   int ds;           // accelerator shift of a log entry
   uint64_t lowmask; // key part of a log entry
-  Devices<kReg> dv;
+  Devices<kReg, tm_t> dv;
   const uint8_t* row;
-  int64_t* fbuf;
+  tm_t* fbuf;       // finish times (scratch; the base's own array in kBase)
   uint32_t* bits;
   int64_t* creq;
   // incremental resume
   const int64_t* rb;
   const int64_t* fb;
-  int64_t Tc, T0;
+  tm_t Tc, T0;
   // running results
   int rootptr, trig;
-  int64_t score, makespan, iters, nev, readypops, last_t;
+  int64_t score, iters, nev, readypops;
+  tm_t makespan, last_t;
   int32_t vflag, vop, vdev, status;
   int64_t vt;
   // base checkpoints
@@ -332,14 +342,19 @@ struct Sim {
   __device__ __forceinline__ bool popped(uint32_t x) const { return (bits[x >> 5] >> (x & 31u)) & 1u; }
   // Finish time of a simulated op (incremental: ops before the resume point
   // keep their base finish).
-  __device__ __forceinline__ int64_t fin(uint32_t x) const {
-    if (kMode == kInc && rb[x] < Tc) return fb[x];
+  // The low 32 bits of a base-snapshot time (little-endian int64).
+  static __device__ __forceinline__ tm_t base_time(const int64_t* a, uint32_t x) {
+    if (kT32) return (tm_t)__ldg(reinterpret_cast<const int32_t*>(a) + 2 * (size_t)x);
+    return (tm_t)__ldg(a + x);
+  }
+  __device__ __forceinline__ tm_t fin(uint32_t x) const {
+    if (kMode == kInc && base_time(rb, x) < Tc) return base_time(fb, x);
     return fbuf[x];
   }
 
   // Transfer estimator of one output over link d -> e (d != e), Sec. 3.3.1.
-  __device__ __forceinline__ int64_t xfer(int d, int e, int64_t bytes, int64_t xq) const {
-    if (g.uniform) return xq + g.lat0;
+  __device__ __forceinline__ tm_t xfer(int d, int e, int64_t bytes, int64_t xq) const {
+    if (g.uniform) return (tm_t)xq + (tm_t)g.lat0;
     const longlong2* L = reinterpret_cast<const longlong2*>(g.links + (d * g.D + e));
     const longlong2 a = __ldg(L), b = __ldg(L + 1);
     LinkRec l;
@@ -347,20 +362,20 @@ struct Sim {
     l.bw = a.y;
     l.lat = b.x;
     l.shift = (int32_t)(b.y & 0xffffffff);
-    return ceil_div_link(bytes, l) + l.lat;
+    return (tm_t)(ceil_div_link(bytes, l) + l.lat);
   }
 
   // Latest arrival of p's output at another accelerator (or f_p): the
   // earliest its source copy may be released.  Per lane.
-  __device__ int64_t lane_hold(uint32_t p, int64_t fp, int dp) const {
+  __device__ tm_t lane_hold(uint32_t p, tm_t fp, int dp) const {
     const int64_t pb = op_durbytes(g.ops, p).y;
     const int64_t pxq = op_relxq(g.ops, p).y;
     const uint4 ls = op_lists(g.ops, p);
-    int64_t h = fp;
+    tm_t h = fp;
     for (uint32_t u = 0; u < ls.y; ++u) {
       const int du = row[__ldg(g.succ + ls.x + u)];
       if (du != dp) {
-        const int64_t a = fp + xfer(dp, du, pb, pxq);
+        const tm_t a = fp + xfer(dp, du, pb, pxq);
         h = a > h ? a : h;
       }
     }
@@ -426,19 +441,20 @@ struct Sim {
   // READY(r, i): start op i (Sec. 3.3.2/3.3.3), record it for HBM-event
   // generation, and push the successors it makes ready.
   // -------------------------------------------------------------------------
-  __device__ void start_op(uint32_t i, int64_t r) {
+  __device__ void start_op(uint32_t i, tm_t r) {
     const unsigned lane = lane_id();
     const longlong2 db = op_durbytes(g.ops, i);
     const longlong2 rx = op_relxq(g.ops, i);
     const uint4 ls = op_lists(g.ops, i);
     const uint4 cs = op_cons(g.ops, i);
-    const int64_t dur = db.x, bytes = db.y, xq = rx.y;
+    const tm_t dur = (tm_t)db.x;
+    const int64_t bytes = db.y, xq = rx.y;
     const uint32_t succ_off = ls.x, nsucc = ls.y;
     const uint32_t flags = cs.w;
     const int d = row[i];
-    const int64_t fd = dv.get_free(d);
-    const int64_t s = r > fd ? r : fd;
-    const int64_t f = s + dur;
+    const tm_t fd = dv.get_free(d);
+    const tm_t s = r > fd ? r : fd;
+    const tm_t f = s + dur;
     dv.set_free(d, f);
     if (lane == 0) {
       fbuf[i] = f;
@@ -449,7 +465,7 @@ struct Sim {
       oplog[opn] = i;
     }
     ++opn;
-    if (flags & kScored) score += f;
+    if (flags & kScored) score += (int64_t)f;
     makespan = f > makespan ? f : makespan;
     if (kMode != kInc || r >= T0) ++nev;
     if (kMode == kBase) ++readypops;
@@ -460,16 +476,17 @@ struct Sim {
     for (uint32_t c0 = 0; c0 < nsucc; c0 += 32) {
       const uint32_t t = c0 + lane;
       uint32_t j = 0;
-      int64_t rj = 0;
+      tm_t rj = 0;
       bool rdy = false;
       if (t < nsucc) {
         j = __ldg(g.succ + succ_off + t);
         const int dj = row[j];
-        int64_t arr = f;
+        tm_t arr = f;
         if (dj != d) arr = f + xfer(d, dj, bytes, xq);
         const longlong2 jrx = op_relxq(g.ops, j);
         const uint4 jls = op_lists(g.ops, j);
-        rj = jrx.x > arr ? jrx.x : arr;
+        const tm_t rel = (tm_t)jrx.x;
+        rj = rel > arr ? rel : arr;
         rdy = true;
         if (jls.w > 1) {
           for (uint32_t k = 0; k < jls.w; ++k) {
@@ -480,7 +497,7 @@ struct Sim {
               break;
             }
             const int dp = row[p];
-            int64_t a = fin(p);
+            tm_t a = fin(p);
             if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
             rj = a > rj ? a : rj;
           }
@@ -516,7 +533,7 @@ struct Sim {
       longlong2 db = make_longlong2(0, 0), rx = make_longlong2(0, 0);
       uint4 ls = make_uint4(0, 0, 0, 0), cs = make_uint4(0, 0, 0, 0);
       int d = 0;
-      int64_t f = 0;
+      tm_t f = 0;
       if (v) {
         db = op_durbytes(g.ops, x);
         rx = op_relxq(g.ops, x);
@@ -527,9 +544,9 @@ struct Sim {
       }
       const int64_t bytes = db.y, xq = rx.y;
       const bool allcons = (cs.w & kAllCons) != 0;
-      log_event(v, kc.make(f - db.x, kAlloc, x), d);
+      log_event(v, kc.make(f - (tm_t)db.x, kAlloc, x), d);
       // receive copies, one per distinct remote accelerator
-      int64_t hold = f;
+      tm_t hold = f;
       bool localc = false;
       const uint32_t nsx = ls.y;
       const uint32_t maxs = __reduce_max_sync(kFullMask, nsx);
@@ -537,7 +554,7 @@ struct Sim {
       for (uint32_t u = 0; u < maxs; ++u) {
         bool want = false, nocons = false;
         int du = 0;
-        int64_t arr = f;
+        tm_t arr = f;
         if (u < nsx) {
           du = row[__ldg(g.succ + ls.x + u)];
           if (du == d) {
@@ -580,7 +597,7 @@ struct Sim {
       const uint32_t maxp = __reduce_max_sync(kFullMask, npx);
       for (uint32_t u = 0; u < maxp; ++u) {
         bool rel = false;
-        int64_t T = f;
+        tm_t T = f;
         uint32_t p = 0;
         if (u < npx) {
           const uint2 ps = __ldg(g.predsib + ls.z + u);
@@ -609,7 +626,7 @@ struct Sim {
               }
             }
             if (rel && row[p] == d) {
-              const int64_t h = lane_hold(p, fin(p), d);
+              const tm_t h = lane_hold(p, fin(p), d);
               T = h > T ? h : T;
             }
           }
@@ -909,7 +926,7 @@ struct Sim {
         status = GMG_SIM_LOOP;
         break;
       }
-      const int64_t t = kc.time(nk);
+      const tm_t t = (tm_t)kc.time(nk);
       last_t = t;
       start_op(kc.op(nk), t);
       if (status) break;
@@ -979,7 +996,7 @@ struct Sim {
     const int ts = trace_slot(k);
     if (ts >= 0)
       for (int x = lane; x < g.n; x += 32) {
-        const int64_t fx = fin((uint32_t)x);
+        const int64_t fx = (int64_t)fin((uint32_t)x);
         o.trace_finish[(int64_t)ts * g.n + x] = fx;
         o.trace_start[(int64_t)ts * g.n + x] = fx - op_durbytes(g.ops, (uint32_t)x).x;
       }
@@ -1013,8 +1030,8 @@ struct Sim {
 // handled yet), save the complete simulator state -- simulated-op bitmap,
 // accelerator state, READY heap, event log, partial results.  An
 // incremental candidate whose resume time T0 is >= that time restarts there.
-template <bool kReg, int kMode, bool kKey>
-__device__ void Sim<kReg, kMode, kKey>::maybe_checkpoint(uint64_t next_key) {
+template <bool kReg, int kMode, bool kKey, bool kT32>
+__device__ void Sim<kReg, kMode, kKey, kT32>::maybe_checkpoint(uint64_t next_key) {
   if (kMode != kBase) return;
   const DevBase& B = P.base;
   if (next_key == kKeyMax || ck >= B.nck || readypops < next_ck) return;
@@ -1056,8 +1073,8 @@ __device__ void Sim<kReg, kMode, kKey>::maybe_checkpoint(uint64_t next_key) {
   __syncwarp();
 }
 
-template <bool kReg, int kMode, bool kKey>
-__device__ void setup_slot(Sim<kReg, kMode, kKey>& S, const SimParams& P, unsigned wib, int64_t slot,
+template <bool kReg, int kMode, bool kKey, bool kT32>
+__device__ void setup_slot(Sim<kReg, kMode, kKey, kT32>& S, const SimParams& P, unsigned wib, int64_t slot,
                            uint8_t* smem) {
   uint8_t* sl = P.scratch + slot * P.slot_bytes;
   const WarpSmem w = carve_smem(smem, P, wib);
@@ -1078,7 +1095,7 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey>& S, const SimParams& P, unsign
   S.oplog = w.oplog;
   S.opn = 0;
   S.sortcap = P.sortcap;
-  S.fbuf = reinterpret_cast<int64_t*>(sl + P.off_f);
+  S.fbuf = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32>::tm_t*>(sl + P.off_f);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
   S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
   S.dv.setup(P.g, w.dev);
@@ -1089,13 +1106,13 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey>& S, const SimParams& P, unsign
 // ---------------------------------------------------------------------------
 // sim_batch: K full placements.
 // ---------------------------------------------------------------------------
-template <bool kReg, bool kKey>
+template <bool kReg, bool kKey, bool kT32>
 __global__ void __launch_bounds__(128, 7) sim_full_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
   const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
-  Sim<kReg, kFull, kKey> S(P);
+  Sim<kReg, kFull, kKey, kT32> S(P);
   setup_slot(S, P, wib, slot, smem);
   for (int64_t k = slot; k < P.K; k += nslots) {
     S.row = P.place + k * P.ld;
@@ -1162,11 +1179,12 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
 // ---------------------------------------------------------------------------
 // sim_incremental: K move lists against the base.
 // ---------------------------------------------------------------------------
-template <bool kReg, bool kKey>
-__device__ void regen(Sim<kReg, kInc, kKey>& S, uint32_t p);
+template <bool kReg, bool kKey, bool kT32>
+__device__ void regen(Sim<kReg, kInc, kKey, kT32>& S, uint32_t p);
 
-template <bool kReg, bool kKey>
-__device__ void inc_candidate(Sim<kReg, kInc, kKey>& S, const SimParams& P, int64_t k, uint8_t* crow) {
+template <bool kReg, bool kKey, bool kT32>
+__device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32>& S, const SimParams& P, int64_t k, uint8_t* crow) {
+  using tm_t = typename Sim<kReg, kInc, kKey, kT32>::tm_t;
   const DevGmg& g = S.g;
   const DevBase& B = P.base;
   const unsigned lane = lane_id();
@@ -1251,7 +1269,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey>& S, const SimParams& P, int6
       }
     return;
   }
-  S.T0 = (int64_t)t0;
+  S.T0 = (tm_t)t0;
   // Latest recorded resume point at or before T0.
   int best = -1;
   for (int c = lane; c < B.nck; c += 32)
@@ -1265,10 +1283,10 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey>& S, const SimParams& P, int6
     return;
   }
   // Restore the simulator state of checkpoint c.
-  S.Tc = B.ck_time[c];
+  S.Tc = (tm_t)B.ck_time[c];
   S.rootptr = (int)sc[1];
   S.score = sc[2];
-  S.makespan = sc[3];
+  S.makespan = (tm_t)sc[3];
   S.vflag = (int32_t)sc[4];
   S.vt = sc[5];
   S.vop = (int32_t)(sc[6] >> 32);
@@ -1390,8 +1408,8 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey>& S, const SimParams& P, int6
 // placement: receive copies on every remote accelerator of its successors
 // (allocated at f_p), and the releases that are already determined because
 // every listed consumer on that accelerator has finished.
-template <bool kReg, bool kKey>
-__device__ void regen(Sim<kReg, kInc, kKey>& S, uint32_t p) {
+template <bool kReg, bool kKey, bool kT32>
+__device__ void regen(Sim<kReg, kInc, kKey, kT32>& S, uint32_t p) {
   const DevGmg& g = S.g;
   const unsigned lane = lane_id();
   const int64_t fp = S.fb[p];
@@ -1462,13 +1480,13 @@ __device__ void regen(Sim<kReg, kInc, kKey>& S, uint32_t p) {
   S.log_event(lane == 0, S.kc.make(m > hm ? m : hm, kFree, p), dp);
 }
 
-template <bool kReg, bool kKey>
+template <bool kReg, bool kKey, bool kT32>
 __global__ void __launch_bounds__(128, 7) sim_inc_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
   const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
-  Sim<kReg, kInc, kKey> S(P);
+  Sim<kReg, kInc, kKey, kT32> S(P);
   setup_slot(S, P, wib, slot, smem);
   S.rb = P.base.rb;
   S.fb = P.base.fb;
@@ -1553,66 +1571,59 @@ __global__ void __launch_bounds__(256) select_final_kernel(const Rank* part, int
 size_t select_rank_bytes() { return sizeof(Rank); }
 
 // Kernel instances by (accelerator state in registers, accelerator id in
-// the event key).
-#define GSIM_KERNEL_TABLE(name)                                                          \
-  const void* name##_ptr(bool reg, bool key) {                                           \
-    if (reg) return key ? (const void*)name<true, true> : (const void*)name<true, false>;  \
-    return key ? (const void*)name<false, true> : (const void*)name<false, false>;         \
-  }
-GSIM_KERNEL_TABLE(sim_full_kernel)
-GSIM_KERNEL_TABLE(sim_inc_kernel)
-GSIM_KERNEL_TABLE(sim_base_kernel)
-#undef GSIM_KERNEL_TABLE
-
-const void* full_kernel_ptr(bool reg, bool key) { return sim_full_kernel_ptr(reg, key); }
-const void* inc_kernel_ptr(bool reg, bool key) { return sim_inc_kernel_ptr(reg, key); }
+// the event key, 32-bit times).
+template <bool R, bool K>
+const void* full_ptr3(bool t32) {
+  return t32 ? (const void*)sim_full_kernel<R, K, true> : (const void*)sim_full_kernel<R, K, false>;
+}
+template <bool R, bool K>
+const void* inc_ptr3(bool t32) {
+  return t32 ? (const void*)sim_inc_kernel<R, K, true> : (const void*)sim_inc_kernel<R, K, false>;
+}
+const void* full_kernel_ptr(bool reg, bool key, bool t32) {
+  if (reg) return key ? full_ptr3<true, true>(t32) : full_ptr3<true, false>(t32);
+  return key ? full_ptr3<false, true>(t32) : full_ptr3<false, false>(t32);
+}
+const void* inc_kernel_ptr(bool reg, bool key, bool t32) {
+  if (reg) return key ? inc_ptr3<true, true>(t32) : inc_ptr3<true, false>(t32);
+  return key ? inc_ptr3<false, true>(t32) : inc_ptr3<false, false>(t32);
+}
+const void* base_kernel_ptr(bool reg, bool key) {
+  if (reg) return key ? (const void*)sim_base_kernel<true, true> : (const void*)sim_base_kernel<true, false>;
+  return key ? (const void*)sim_base_kernel<false, true> : (const void*)sim_base_kernel<false, false>;
+}
 
 cudaError_t set_smem_limits(int smem) {
   for (int r = 0; r < 2; ++r)
-    for (int k = 0; k < 2; ++k) {
-      const void* fns[] = {sim_full_kernel_ptr(r, k), sim_inc_kernel_ptr(r, k), sim_base_kernel_ptr(r, k)};
-      for (const void* f : fns) {
-        const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-        if (e != cudaSuccess) return e;
+    for (int k = 0; k < 2; ++k)
+      for (int t = 0; t < 2; ++t) {
+        const void* fns[] = {full_kernel_ptr(r, k, t), inc_kernel_ptr(r, k, t), base_kernel_ptr(r, k)};
+        for (const void* f : fns) {
+          const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+          if (e != cudaSuccess) return e;
+        }
       }
-    }
   return cudaSuccess;
 }
 
+// A kernel instance's launch through its pointer (the instance is chosen by
+// the graph's flags).
+static cudaError_t launch_ptr(const void* fn, const SimParams& P, int grid, int block, size_t smem,
+                              cudaStream_t st) {
+  void* args[] = {const_cast<SimParams*>(&P)};
+  return cudaLaunchKernel(fn, dim3(grid), dim3(block), args, smem, st);
+}
+
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
-  const bool key = P.g.dev_key != 0;
-  if (reg) {
-    if (key) sim_full_kernel<true, true><<<grid, block, smem, st>>>(P);
-    else sim_full_kernel<true, false><<<grid, block, smem, st>>>(P);
-  } else {
-    if (key) sim_full_kernel<false, true><<<grid, block, smem, st>>>(P);
-    else sim_full_kernel<false, false><<<grid, block, smem, st>>>(P);
-  }
-  return cudaGetLastError();
+  return launch_ptr(full_kernel_ptr(reg, P.g.dev_key != 0, P.g.t32 != 0), P, grid, block, smem, st);
 }
 
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
-  const bool key = P.g.dev_key != 0;
-  if (reg) {
-    if (key) sim_inc_kernel<true, true><<<grid, block, smem, st>>>(P);
-    else sim_inc_kernel<true, false><<<grid, block, smem, st>>>(P);
-  } else {
-    if (key) sim_inc_kernel<false, true><<<grid, block, smem, st>>>(P);
-    else sim_inc_kernel<false, false><<<grid, block, smem, st>>>(P);
-  }
-  return cudaGetLastError();
+  return launch_ptr(inc_kernel_ptr(reg, P.g.dev_key != 0, P.g.t32 != 0), P, grid, block, smem, st);
 }
 
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st) {
-  const bool key = P.g.dev_key != 0;
-  if (reg) {
-    if (key) sim_base_kernel<true, true><<<1, 32, smem, st>>>(P);
-    else sim_base_kernel<true, false><<<1, 32, smem, st>>>(P);
-  } else {
-    if (key) sim_base_kernel<false, true><<<1, 32, smem, st>>>(P);
-    else sim_base_kernel<false, false><<<1, 32, smem, st>>>(P);
-  }
-  return cudaGetLastError();
+  return launch_ptr(base_kernel_ptr(reg, P.g.dev_key != 0), P, 1, 32, smem, st);
 }
 
 cudaError_t launch_select(const int32_t* status, const int32_t* viol, const int64_t* score,

@@ -37,9 +37,13 @@ def _run(desc, base, moves, **kw):
     (5, 600, 33, {}),
     (6, 400, 256, dict(explicit_cons=True)),
     (7, 1500, 16, dict(edge_p=0.8, max_pred=4, dur_hi=3000)),
+    (8, 300, 8, dict(dur_hi=1 << 32)),             # times beyond 2^31: 64-bit instances
+    (9, 300, 40, dict(dur_hi=1 << 31, explicit_cons=True)),
 ])
 def test_random_incremental_bit_exact(seed, n, D, kw):
     d = W.random_desc(5000 + seed, n, D, **kw)
+    if kw.get("dur_hi", 0) >= 1 << 31:
+        assert G.gmg_create(d).info["time_bound"] >= 1 << 31
     g0 = np.random.default_rng(seed)
     base = g0.integers(0, D, n).astype(np.uint8)
     mv = W.random_moves(seed, 300, base, D, max_moves=12)
@@ -84,14 +88,13 @@ def test_incremental_equals_full_batch_of_applied_moves():
         assert np.array_equal(a[key], f[key]), key
 
 
-def test_workload_incremental_sampled():
+def test_workload_incremental_all_candidates():
+    """Every one of the 16,384 move lists of the incremental workload."""
     wl = W.config3()
     mv = wl.moves
     g, b, out = _run(wl.desc, wl.base_place, mv)
     got = out.to_numpy()
-    ks = np.random.default_rng(33).choice(mv.n_cand, 512, replace=False)
-    ks.sort()
-    s, pk, rq = O.incremental_batch(wl.desc, wl.base_place, mv.subset(ks))
-    compare(got, s, pk, rq, ks=ks)
+    s, pk, rq = O.incremental_batch(wl.desc, wl.base_place, mv)
+    compare(got, s, pk, rq)
     assert (got["status"] == 0).all()
     assert (got["events"] <= wl.desc.n_ops).all() and (got["events"] > 0).all()

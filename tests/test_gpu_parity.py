@@ -43,10 +43,15 @@ def _random_case(seed, n, D, **kw):
     (9, 500, 256, dict(explicit_cons=True, bytes_hi=1 << 30)),
     (10, 1000, 16, dict(edge_p=0.9, max_pred=4)),
     (11, 90, 6, dict(with_release=False, with_avail0=False, cap=1 << 40)),
+    (15, 300, 8, dict(dur_hi=1 << 32)),               # times beyond 2^31: 64-bit instances
+    (16, 200, 40, dict(dur_hi=1 << 31, explicit_cons=True)),
+    (17, 150, 4, dict(dur_hi=1 << 40, link_hetero=False)),
 ])
 def test_random_dags_bit_exact(seed, n, D, kw):
     d, rows = _random_case(seed, n, D, **kw)
     g = G.gmg_create(d)
+    if kw.get("dur_hi", 0) >= 1 << 31:
+        assert g.info["time_bound"] >= 1 << 31
     K = rows.shape[0]
     tk = torch.tensor([0, 5, K - 1], dtype=torch.int32, device="cuda")
     out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk)
@@ -166,18 +171,16 @@ def test_workload_prefill_all_candidates():
     assert (s["sla_miss"] > 0).any()
 
 
-def test_workload_memory_tight_sampled():
+def test_workload_memory_tight_all_candidates():
+    """Every one of the 8,192 placements of the memory-tight decode workload."""
     wl = W.config4()
-    K = wl.n_full
-    ks = np.random.default_rng(44).choice(K, 24, replace=False)
-    ks.sort()
+    rows = wl.all_full_rows()
     g = G.gmg_create(wl.desc)
-    place = torch_place(wl.all_full_rows())
-    out = G.sim_batch(g, place, req_done=True)
+    out = G.sim_batch(g, torch_place(rows), req_done=True)
     torch.cuda.synchronize()
     got = out.to_numpy()
-    s, pk, rq = oracle_rows(wl.desc, wl.full_rows(ks))
-    compare(got, s, pk, rq, ks=ks)
+    s, pk, rq = oracle_rows(wl.desc, rows)
+    compare(got, s, pk, rq)
     frac = float(got["viol_flag"].mean())
     assert 0.25 < frac < 0.35, frac
     assert (got["status"] == 0).all() and (got["events"] == wl.desc.n_ops).all()
@@ -198,10 +201,10 @@ def test_workload_large_full_size_sampled():
     got, goti = out.to_numpy(), inc.to_numpy()
     assert (got["status"] == 0).all() and (goti["status"] == 0).all()
     rng = np.random.default_rng(55)
-    ks = np.sort(rng.choice(wl.n_full, 6, replace=False))
+    ks = np.sort(rng.choice(wl.n_full, 256, replace=False))
     s, pk, rq = oracle_rows(wl.desc, wl.full_rows(ks))
     compare(got, s, pk, rq, ks=ks)
-    ki = np.sort(rng.choice(wl.moves.n_cand, 6, replace=False))
+    ki = np.sort(rng.choice(wl.moves.n_cand, 256, replace=False))
     si, pki, rqi = O.incremental_batch(wl.desc, wl.base_place, wl.moves.subset(ki))
     compare(goti, si, pki, rqi, ks=ki)
     assert best.cpu().tolist()[1] == int(got["score"].min())
