@@ -169,7 +169,7 @@ struct SimParams {
   uint8_t* scratch;
   int64_t slot_bytes;    // scratch bytes per warp slot
   // byte offsets inside a slot
-  int64_t off_f, off_bits, off_creq, off_qk, off_mk, off_md, off_row;
+  int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row;
 };
 
 }  // namespace gsim

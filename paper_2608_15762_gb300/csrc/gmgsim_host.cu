@@ -39,7 +39,7 @@ constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
 constexpr int kSortCap = 128;             // power of two; raised to n_dev's power of two
 constexpr int kDrainTrigger = 48;
-constexpr int kOpsPerGeneration = 24;     // ~100 HBM events: one 128-key register sort
+constexpr int kOpsPerGeneration = 24;     // ~85 HBM events per generation (prefill graphs)
 constexpr int kCheckpoints = 256;
 constexpr int kCheckpointQueue = 4096;
 constexpr int kCheckpointLog = 8192;
@@ -434,6 +434,7 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   const int64_t qspill = std::max<int64_t>(P.qcap - P.qs, 0);
   const int64_t mspill = std::max<int64_t>(P.mcap - P.ms, 0);
   P.off_f = take(8 * (size_t)G.n);
+  P.off_hold = take(8 * (size_t)G.n);
   P.off_bits = take(4 * (size_t)((G.n + 31) / 32) + 16);
   P.off_creq = take(8 * (size_t)G.R);
   P.off_qk = take(8 * (size_t)qspill);

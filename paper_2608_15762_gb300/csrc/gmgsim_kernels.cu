@@ -317,6 +317,7 @@ struct Sim {
   Devices<kReg, tm_t> dv;
   const uint8_t* row;
   tm_t* fbuf;       // finish times (scratch; the base's own array in kBase)
+  tm_t* holdb;      // latest outgoing arrival of each op's output (scratch)
   uint32_t* bits;
   int64_t* creq;
   // incremental resume
@@ -324,7 +325,8 @@ struct Sim {
   const int64_t* fb;
   tm_t Tc, T0;
   // running results
-  int rootptr, trig;
+  int rootptr;
+  uint64_t rkey;    // root_keys[rootptr], kKeyMax past the end
   int64_t score, iters, nev, readypops;
   tm_t makespan, last_t;
   int32_t vflag, vop, vdev, status;
@@ -383,6 +385,10 @@ struct Sim {
   }
 
 
+  __device__ __forceinline__ void load_root() {
+    rkey = rootptr < g.nroots ? __ldg(g.root_keys + rootptr) : kKeyMax;
+  }
+
   // READY keys go to a free lane's register if there is one, else the heap.
   __device__ __forceinline__ void push_ready(uint64_t key) {
     const uint32_t freel = __ballot_sync(kFullMask, rk_reg == kKeyMax);
@@ -425,8 +431,8 @@ struct Sim {
     rk_reg = kKeyMax;
     log.n = 0;
     opn = 0;
-    trig = P.drain_trigger;
     rootptr = 0;
+    load_root();
     score = makespan = 0;
     iters = nev = readypops = 0;
     last_t = -1;
@@ -566,17 +572,17 @@ struct Sim {
                 want = false;
                 break;
               }
-            if (want) {
-              arr = f + xfer(d, du, bytes, xq);
-              hold = arr > hold ? arr : hold;
-              if (!allcons) {
-                nocons = true;
-                for (uint32_t w = 0; w < cs.y; ++w)
-                  if (row[__ldg(g.cons + cs.x + w)] == du) {
-                    nocons = false;
-                    break;
-                  }
-              }
+          }
+          if (want) {
+            arr = f + xfer(d, du, bytes, xq);
+            hold = arr > hold ? arr : hold;
+            if (!allcons) {
+              nocons = true;
+              for (uint32_t w = 0; w < cs.y; ++w)
+                if (row[__ldg(g.cons + cs.x + w)] == du) {
+                  nocons = false;
+                  break;
+                }
             }
           }
         }
@@ -592,6 +598,8 @@ struct Sim {
           }
       }
       log_event(v && !localc, kc.make(hold, kFree, x), d);
+      if (v) holdb[x] = hold;
+      __syncwarp();
       // releases of the inputs this op holds
       const uint32_t npx = ls.w;
       const uint32_t maxp = __reduce_max_sync(kFullMask, npx);
@@ -626,7 +634,9 @@ struct Sim {
               }
             }
             if (rel && row[p] == d) {
-              const tm_t h = lane_hold(p, fin(p), d);
+              // p's own copy: not before its outgoing arrivals (recorded when
+              // p's events were generated; p started before this op)
+              const tm_t h = (kMode == kInc && base_time(rb, p) < Tc) ? lane_hold(p, fin(p), d) : holdb[p];
               T = h > T ? h : T;
             }
           }
@@ -768,12 +778,11 @@ struct Sim {
     settle_violation(vmin);
   }
 
-  // Sort and apply m <= 128 extracted events in registers.
-  __device__ void sort_apply_regs(int m) {
-    if (m <= 32) sort_apply_regs_e<1>(m);
-    else if (m <= 64) sort_apply_regs_e<2>(m);
-    else sort_apply_regs_e<4>(m);
-  }
+  // Sort and apply m <= 32 extracted events in registers.  (Wider register
+  // networks sort faster but their unrolled code -- each inlining its own
+  // copies of the segmented apply -- overflowed the instruction cache: larger
+  // drains go through the shared-memory sort.)
+  __device__ void sort_apply_regs(int m) { sort_apply_regs_e<1>(m); }
 
   __device__ int count_below(uint64_t kmax) const {
     int c = 0;
@@ -888,7 +897,7 @@ struct Sim {
       }
       const int m = extract(kmax);
       if (m == 0) break;
-      if (kKey && m <= 128) {
+      if (kKey && m <= 32) {
         sort_apply_regs(m);
       } else {
         sort_area(m);
@@ -897,7 +906,6 @@ struct Sim {
       }
       if (kmax == lim) break;
     }
-    trig = log.n + P.drain_trigger;
   }
 
   __device__ void maybe_checkpoint(uint64_t next_key);
@@ -908,7 +916,7 @@ struct Sim {
     while (true) {
       const uint64_t top = q.top();
       const uint64_t rm = warp_min_u64(rk_reg);
-      const uint64_t rk = rootptr < g.nroots ? __ldg(g.root_keys + rootptr) : kKeyMax;
+      const uint64_t rk = rkey;
       uint64_t nk = rk < top ? rk : top;
       nk = rm < nk ? rm : nk;
       if (kMode == kBase) maybe_checkpoint(nk);
@@ -918,6 +926,7 @@ struct Sim {
         if (rk_reg == rm) rk_reg = kKeyMax;  // keys are unique
       } else if (nk == rk) {
         ++rootptr;
+        load_root();
       } else {
         __syncwarp();
         q.pop();
@@ -1096,6 +1105,7 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey, kT32>& S, const SimParams& P, 
   S.opn = 0;
   S.sortcap = P.sortcap;
   S.fbuf = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32>::tm_t*>(sl + P.off_f);
+  S.holdb = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32>::tm_t*>(sl + P.off_hold);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
   S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
   S.dv.setup(P.g, w.dev);
@@ -1285,6 +1295,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32>& S, const SimParams& P
   // Restore the simulator state of checkpoint c.
   S.Tc = (tm_t)B.ck_time[c];
   S.rootptr = (int)sc[1];
+  S.load_root();
   S.score = sc[2];
   S.makespan = (tm_t)sc[3];
   S.vflag = (int32_t)sc[4];
@@ -1296,7 +1307,6 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32>& S, const SimParams& P
   S.readypops = 0;
   S.last_t = -1;
   S.status = GMG_SIM_OK;
-  S.trig = P.drain_trigger;
   S.rk_reg = kKeyMax;
   S.opn = 0;
   S.dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
