@@ -35,7 +35,8 @@ METRIC = "candidate placements simulated/sec (and op-events/sec) vs HBM/issue ro
 UNIT = "candidates/s"
 PROFILE_DIR = os.path.join(ROOT, "profiles")
 KERNEL_SOURCES = [os.path.join(ROOT, "paper_2608_15762_gb300", "csrc", f)
-                  for f in ("gmgsim_kernels.cu", "gmg_layout.h")]
+                  for f in ("gmgsim_sim.cuh", "gmgsim_full.cu", "gmgsim_inc.cu", "gmgsim_kernels.cu",
+                            "gmg_layout.h")]
 
 
 def kernel_hash() -> str:
@@ -304,7 +305,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5])
+    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--candidates", type=int, default=None,
                     help="profiling aid: simulate only the first N candidates of each half "

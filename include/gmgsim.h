@@ -87,7 +87,7 @@ typedef struct {
   const int32_t* pred_idx; /* [E] each < i (topological), no duplicates per op */
   const int32_t* cons_off; /* [N+1] optional: consumers whose completion releases op i's output */
   const int32_t* cons_idx; /* each a successor of i, no duplicates; NULL lists = all successors */
-  const int64_t* dur_us;     /* [N] >= 1 */
+  const int64_t* dur_us;     /* [N] >= 1 (ignored, may be NULL, when n_types >= 2) */
   const int64_t* out_bytes;  /* [N] >= 0 */
   const int64_t* release_us; /* [N] >= 0, optional (0) */
   const int32_t* req_id;     /* [N] in [-1, R), optional (-1 = no request) */
@@ -98,6 +98,13 @@ typedef struct {
   const int64_t* avail0_us;   /* [D] >= 0, optional (0): accelerator busy until then */
   const int64_t* bw_B_per_us; /* [D*D] row = source; >= 1 off the diagonal (diagonal ignored) */
   const int64_t* lat_us;      /* [D*D] >= 0 off the diagonal */
+  /* Heterogeneous accelerators: the operator estimator of Sec. 3.3.1 keeps one
+   * estimate per (accelerator type, operator), so an op's duration depends on
+   * the type of the accelerator it is placed on.  n_types <= 1: one type, every
+   * op takes dur_us[i] everywhere and the two arrays below are not read. */
+  int32_t n_types;             /* T in [0, 256] */
+  const uint8_t* dev_type;     /* [D] each < T */
+  const int64_t* dur_by_type;  /* [N*T] row-major by op: dur of op i on type t at [i*T + t], >= 1 */
 } gmg_desc_t;
 
 typedef struct gmg gmg_t;           /* opaque; host metadata + borrowed device workspace */

@@ -37,7 +37,8 @@ class _Graph(C.Structure):
                 ("n_req", C.c_int32)] + [
         (name, C.c_void_p) for name in (
             "pred_off", "pred_idx", "cons_off", "cons_idx", "dur", "out_bytes", "release",
-            "req_id", "scored", "deadline", "cap", "base", "avail0", "bw", "lat")]
+            "req_id", "scored", "deadline", "cap", "base", "avail0", "bw", "lat")] + [
+        ("n_types", C.c_int32), ("dev_type", C.c_void_p), ("dur_type", C.c_void_p)]
 
 
 _LIB = None
@@ -78,7 +79,8 @@ class _GraphHolder:
                         _ptr(d.pred_off), _ptr(d.pred_idx), _ptr(d.cons_off), _ptr(d.cons_idx),
                         _ptr(d.dur), _ptr(d.out_bytes), _ptr(d.release), _ptr(d.req_id),
                         _ptr(d.scored), _ptr(d.deadline), _ptr(d.cap), _ptr(d.base),
-                        _ptr(d.avail0), _ptr(d.bw), _ptr(d.lat))
+                        _ptr(d.avail0), _ptr(d.bw), _ptr(d.lat), d.n_types, _ptr(d.dev_type),
+                        _ptr(d.dur_by_type))
 
     @property
     def ref(self):

@@ -15,7 +15,9 @@
 //  * Transfer estimator (Sec. 3.3.1): t = alpha * size + c per accelerator
 //    pair, here in integer form ceil(size / bw[d][e]) + lat[d][e], 0 on the
 //    same accelerator.  Integer durations stand in for the operator
-//    estimator's output.
+//    estimator's output; the operator estimator is kept per (accelerator
+//    type, operator), so with several accelerator types an operator's
+//    duration is the one of the type it is placed on.
 //  * Queue rule (Sec. 3.3.2 and Sec. 3.5.1): each accelerator queue runs at
 //    most one operator at a time; the operator started is the ready, issued
 //    one with the earliest ready time (ties: lowest op id).
@@ -96,6 +98,9 @@ typedef struct {
   const int64_t* avail0;     // NULL: 0
   const int64_t* bw;         // n_dev*n_dev, row = source
   const int64_t* lat;
+  int32_t n_types;           // >= 2: durations per (op, accelerator type)
+  const uint8_t* dev_type;   // [n_dev]
+  const int64_t* dur_type;   // [n_ops * n_types], op-major
 } orc_graph;
 
 typedef struct {
@@ -122,7 +127,15 @@ struct Graph {
   std::vector<int64_t> dur, bytes, release, deadline, cap, base, avail0, bw, lat;
   std::vector<int> req;
   std::vector<uint8_t> scored;
+  int T = 0;                     // accelerator types (0: one type, dur)
+  std::vector<uint8_t> dev_type;  // [D]
+  std::vector<int64_t> dur_type;  // [n*T]
 };
+
+// Duration of op i on accelerator d.
+int64_t dur_on(const Graph& g, int i, int d) {
+  return g.T ? g.dur_type[size_t(i) * g.T + g.dev_type[d]] : g.dur[i];
+}
 
 int64_t ceil_div(int64_t a, int64_t b) {
   int64_t q = a / b;
@@ -140,7 +153,10 @@ int build(const orc_graph* in, Graph& g) {
   const int n = in->n_ops, D = in->n_dev, R = in->n_req;
   if (n < 0 || in->n_edges < 0 || D < 1 || D > 256 || R < 0) return kEInval;
   if (!in->pred_off || (in->n_edges > 0 && !in->pred_idx)) return kEInval;
-  if (n > 0 && (!in->dur || !in->out_bytes)) return kEInval;
+  if (in->n_types < 0 || in->n_types > 256) return kEInval;
+  g.T = in->n_types >= 2 ? in->n_types : 0;
+  if (g.T && (!in->dev_type || (n > 0 && !in->dur_type))) return kEInval;
+  if (n > 0 && ((!g.T && !in->dur) || !in->out_bytes)) return kEInval;
   if (D > 1 && (!in->bw || !in->lat)) return kEInval;
   g.n = n; g.e = in->n_edges; g.D = D; g.R = R;
   if (in->pred_off[0] != 0 || in->pred_off[n] != in->n_edges) return kEInval;
@@ -183,7 +199,17 @@ int build(const orc_graph* in, Graph& g) {
   }
   g.dur.resize(n); g.bytes.resize(n); g.release.resize(n); g.req.resize(n); g.scored.resize(n);
   for (int i = 0; i < n; ++i) {
-    g.dur[i] = in->dur[i];
+    if (g.T) {
+      // an op's longest duration over the types bounds its times
+      g.dur[i] = 0;
+      for (int t = 0; t < g.T; ++t) {
+        const int64_t v = in->dur_type[size_t(i) * g.T + t];
+        if (v < 1) return kEInval;
+        g.dur[i] = std::max(g.dur[i], v);
+      }
+    } else {
+      g.dur[i] = in->dur[i];
+    }
     g.bytes[i] = in->out_bytes[i];
     g.release[i] = in->release ? in->release[i] : 0;
     g.req[i] = in->req_id ? in->req_id[i] : -1;
@@ -200,6 +226,12 @@ int build(const orc_graph* in, Graph& g) {
     g.base[d] = in->base ? in->base[d] : 0;
     g.avail0[d] = in->avail0 ? in->avail0[d] : 0;
     if (g.cap[d] < 0 || g.base[d] < 0 || g.base[d] > g.cap[d] || g.avail0[d] < 0) return kEInval;
+  }
+  if (g.T) {
+    g.dev_type.assign(in->dev_type, in->dev_type + D);
+    for (int d = 0; d < D; ++d)
+      if (g.dev_type[d] >= g.T) return kEInval;
+    g.dur_type.assign(in->dur_type, in->dur_type + size_t(n) * g.T);
   }
   g.bw.assign(size_t(D) * D, 1);
   g.lat.assign(size_t(D) * D, 0);
@@ -306,7 +338,7 @@ void simulate(const Graph& g, const uint8_t* dev, Result& res) {
       ready_q[d].erase(ready_q[d].begin());
       running[d] = i;
       s[i] = now;
-      f[i] = now + g.dur[i];
+      f[i] = now + dur_on(g, i, d);
       events.push(Ev(f[i], 0, i));
     }
   }

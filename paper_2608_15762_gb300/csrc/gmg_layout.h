@@ -93,6 +93,9 @@ struct DevGmg {
   int32_t tb;                 // time bits needed (every time < 2^tb)
   int32_t dev_key;            // 1 if an accelerator id fits above (time, class, op) in 64 bits
   int32_t t32;                // 1 if every time is below 2^31 (the kernels then use int32 times)
+  int32_t ntypes;             // accelerator types; >= 2: durations from durt by dtype
+  const int64_t* durt;        // [N*ntypes] duration of op i on type t at i*ntypes + t
+  const uint8_t* dtype;       // [D] type of each accelerator
   int32_t uniform;
 };
 

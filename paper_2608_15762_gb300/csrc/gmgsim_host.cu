@@ -15,8 +15,8 @@
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
 size_t select_rank_bytes();
-const void* full_kernel_ptr(bool reg, bool key, bool t32);
-const void* inc_kernel_ptr(bool reg, bool key, bool t32);
+const void* full_kernel_ptr(bool reg, bool key, bool t32, bool types);
+const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types);
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
@@ -48,12 +48,12 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
   size_t off_ops, off_succ, off_pred, off_sib, off_cons, off_roots, off_cap, off_base, off_avail,
-      off_dl, off_links, total;
+      off_dl, off_links, off_durt, off_dtype, total;
 };
 
 // Everything gmg_create derives from a description.
 struct Built {
-  int n = 0, E = 0, D = 0, R = 0, Ec = 0, nroots = 0, ib = 1;
+  int n = 0, E = 0, D = 0, R = 0, Ec = 0, nroots = 0, ib = 1, T = 0;
   bool uniform = true;
   int64_t bw0 = 1, lat0 = 0, time_bound = 0, max_iter = 0, queue_bound = 0, log_bound = 0;
   std::vector<OpRec> ops;
@@ -61,6 +61,8 @@ struct Built {
   std::vector<uint64_t> roots;
   std::vector<int64_t> cap, base, avail0, deadline;
   std::vector<LinkRec> links;
+  std::vector<int64_t> durt;  // [n*T] when T >= 2
+  std::vector<uint8_t> dtype; // [D] when T >= 2
   Layout L{};
 };
 
@@ -102,6 +104,8 @@ void plan(Built& b) {
   L.off_avail = take(8 * (size_t)b.D);
   L.off_dl = take(8 * (size_t)b.R);
   L.off_links = take(b.uniform ? 0 : sizeof(LinkRec) * (size_t)b.D * b.D);
+  L.off_durt = take(8 * b.durt.size());
+  L.off_dtype = take(b.dtype.size());
   L.total = o;
 }
 
@@ -112,7 +116,10 @@ int build(const gmg_desc_t* d, Built& b) {
   if (n < 0 || d->n_edges < 0 || D < 1 || D > 256 || R < 0) return GMG_EINVAL;
   if (n > (1 << kMaxOpsLog2)) return GMG_ERANGE;
   if (!d->pred_off || (d->n_edges > 0 && !d->pred_idx)) return GMG_EINVAL;
-  if (n > 0 && (!d->dur_us || !d->out_bytes)) return GMG_EINVAL;
+  const int T = d->n_types >= 2 ? d->n_types : 0;
+  if (d->n_types < 0 || d->n_types > 256) return GMG_EINVAL;
+  if (T && (!d->dev_type || (n > 0 && !d->dur_by_type))) return GMG_EINVAL;
+  if (n > 0 && ((!T && !d->dur_us) || !d->out_bytes)) return GMG_EINVAL;
   if (D > 1 && (!d->bw_B_per_us || !d->lat_us)) return GMG_EINVAL;
   if (d->pred_off[0] != 0 || d->pred_off[n] != d->n_edges) return GMG_EINVAL;
   for (int i = 0; i < n; ++i)
@@ -121,6 +128,13 @@ int build(const gmg_desc_t* d, Built& b) {
   b.E = d->n_edges;
   b.D = D;
   b.R = R;
+  b.T = T;
+  if (T) {
+    b.dtype.assign(d->dev_type, d->dev_type + D);
+    for (int e = 0; e < D; ++e)
+      if (b.dtype[e] >= T) return GMG_EINVAL;
+    b.durt.assign(d->dur_by_type, d->dur_by_type + (size_t)n * T);
+  }
   b.ib = 1;
   while ((int64_t(1) << b.ib) < n) ++b.ib;
   // predecessors (topological, no duplicates) and successor counts
@@ -154,7 +168,17 @@ int build(const gmg_desc_t* d, Built& b) {
   // per-op scalars
   for (int i = 0; i < n; ++i) {
     OpRec& r = b.ops[i];
-    r.dur = d->dur_us[i];
+    if (T) {
+      // the bounds below take an op's longest duration over the types
+      r.dur = 0;
+      for (int t = 0; t < T; ++t) {
+        const int64_t v = b.durt[(size_t)i * T + t];
+        if (v < 1) return GMG_EINVAL;
+        r.dur = std::max(r.dur, v);
+      }
+    } else {
+      r.dur = d->dur_us[i];
+    }
     r.bytes = d->out_bytes[i];
     r.release = d->release_us ? d->release_us[i] : 0;
     r.req = d->req_id ? d->req_id[i] : -1;
@@ -453,8 +477,9 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     g_smem_set = true;
   }
   int bps = 0;
-  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0)
-                       : full_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0);
+  const bool types = G.ntypes >= 2;
+  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0, types)
+                       : full_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0, types);
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
     return GMG_ECUDA;
   bps = std::max(bps, 1);
@@ -589,6 +614,10 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   put(L.off_avail, b.avail0.data(), 8 * b.avail0.size());
   put(L.off_dl, b.deadline.data(), 8 * b.deadline.size());
   if (!b.uniform) put(L.off_links, b.links.data(), sizeof(LinkRec) * b.links.size());
+  if (b.T) {
+    put(L.off_durt, b.durt.data(), 8 * b.durt.size());
+    put(L.off_dtype, b.dtype.data(), b.dtype.size());
+  }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemcpyAsync(d_ws, host.data(), b.L.total, cudaMemcpyHostToDevice, st) != cudaSuccess)
     return GMG_ECUDA;
@@ -608,6 +637,9 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.avail0 = reinterpret_cast<const int64_t*>(w + L.off_avail);
   G.deadline = reinterpret_cast<const int64_t*>(w + L.off_dl);
   G.links = b.uniform ? nullptr : reinterpret_cast<const LinkRec*>(w + L.off_links);
+  G.ntypes = b.T;
+  G.durt = b.T ? reinterpret_cast<const int64_t*>(w + L.off_durt) : nullptr;
+  G.dtype = b.T ? w + L.off_dtype : nullptr;
   G.lat0 = b.lat0;
   G.max_iter = b.max_iter;
   G.n = b.n;
@@ -618,7 +650,9 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.tb = 1;
   while (G.tb < 62 && (int64_t(1) << G.tb) <= b.time_bound) ++G.tb;
   G.dev_key = (G.tb + G.ib + 2 + 8 <= 63) ? 1 : 0;
-  G.t32 = G.tb <= 31 ? 1 : 0;  // every time < 2^tb fits int32
+  // every time < 2^tb fits int32; the 32-bit instances also take the
+  // accelerator id from the event key
+  G.t32 = (G.tb <= 31 && G.dev_key) ? 1 : 0;
   G.uniform = b.uniform ? 1 : 0;
   gmg_info_t& I = g->info;
   std::memset(&I, 0, sizeof(I));

@@ -1,0 +1,1128 @@
+// Device side of the what-if placement simulator, shared by the kernel
+// translation units (gmgsim_full.cu, gmgsim_inc.cu, gmgsim_kernels.cu).
+//
+// One warp simulates one candidate placement (Algorithm 1 evaluates the
+// candidate partitions "in parallel"; here every warp of a persistent grid
+// takes candidates k = warp, warp + W, ...).  Inside a warp the simulation
+// is the event-driven loop of Sec. 3.3.3 restated as one ordered sweep:
+//
+//   READY(r_i, i)  op i's last input has arrived (Sec. 3.3.2 ready time).
+//                  Taking READY keys in (r, id) order and starting each op
+//                  at s_i = max(r_i, accelerator free time) makes every queue
+//                  run its ops in (ready time, id) order, one at a time
+//                  (Sec. 3.3.2, Sec. 3.5.1) -- exactly "an idle queue starts
+//                  the ready op with the earliest ready time".
+//   FREE / ALLOC   HBM events of the copies of an op's output: the op's own
+//                  buffer at s_i, a receive buffer on every other accelerator
+//                  of a successor at f_i (Recv before Send, Sec. 3.5.2), each
+//                  released by its last listed consumer there (Sec. 3.3.2).
+//
+// READY keys live in a warp-cooperative 32-ary min-heap: the 32 children of
+// a node are compared by the 32 lanes at once (one coalesced load, two
+// redux.sync), so a pop costs log32(size) warp steps.  Ops without
+// predecessors never enter it: their keys are pre-sorted on the host.
+//
+// HBM events are appended to a per-warp log in O(1).  Every event produced
+// while handling READY(r, .) happens at a time >= r, so once the next READY
+// key has time T, every logged event with time < T is final and no later
+// event can precede it.  Such events are drained in batches: extracted into
+// shared memory, bitonic-sorted by (time, frees before allocs, op), and
+// applied in order to the per-accelerator live bytes, which gives the peaks
+// and the first capacity violation (Sec. 3.4.2 OOM discard) exactly.
+//
+// Lanes also fan out over successor lists (readiness, transfer arrivals,
+// distinct receiving accelerators via __match_any_sync) and predecessor
+// lists (ready-time maxima, last-consumer releases).  With at most 32
+// accelerators, lane d keeps accelerator d's free time, live bytes and peak
+// in registers.
+//
+// No wait in these kernels depends on another warp or block; the only loop
+// whose trip count is not bounded by the data is the event loop, capped at
+// g.max_iter iterations (status GMG_SIM_LOOP).
+
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <type_traits>
+
+#include "gmg_layout.h"
+
+namespace gsim {
+namespace {
+
+constexpr unsigned kFullMask = 0xffffffffu;
+constexpr uint64_t kKeyMax = ~0ull;
+constexpr int64_t kI64Max = 0x7fffffffffffffffll;
+
+__device__ __forceinline__ uint64_t warp_min_u64(uint64_t v) {
+  const uint32_t hi = (uint32_t)(v >> 32), lo = (uint32_t)v;
+  const uint32_t mh = __reduce_min_sync(kFullMask, hi);
+  const uint32_t ml = __reduce_min_sync(kFullMask, hi == mh ? lo : 0xffffffffu);
+  return ((uint64_t)mh << 32) | ml;
+}
+
+__device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
+  const uint32_t hi = (uint32_t)(v >> 32), lo = (uint32_t)v;
+  const uint32_t mh = __reduce_max_sync(kFullMask, hi);
+  const uint32_t ml = __reduce_max_sync(kFullMask, hi == mh ? lo : 0u);
+  return ((uint64_t)mh << 32) | ml;
+}
+
+__device__ __forceinline__ unsigned lane_id() { return threadIdx.x & 31u; }
+__device__ __forceinline__ uint32_t lanes_below() { return (1u << lane_id()) - 1u; }
+
+// 16-byte pieces of an OpRec, loaded through the read-only path.
+__device__ __forceinline__ longlong2 op_durbytes(const OpRec* ops, uint32_t i) {
+  return __ldg(reinterpret_cast<const longlong2*>(ops + i));
+}
+__device__ __forceinline__ longlong2 op_relxq(const OpRec* ops, uint32_t i) {
+  return __ldg(reinterpret_cast<const longlong2*>(ops + i) + 1);
+}
+__device__ __forceinline__ uint4 op_lists(const OpRec* ops, uint32_t i) {
+  return __ldg(reinterpret_cast<const uint4*>(ops + i) + 2);  // succ_off, nsucc, pred_off, npred
+}
+__device__ __forceinline__ uint4 op_cons(const OpRec* ops, uint32_t i) {
+  return __ldg(reinterpret_cast<const uint4*>(ops + i) + 3);  // cons_off, ncons, req, flags
+}
+
+struct KeyCodec {
+  int ib;
+  uint64_t mask;
+  template <typename TM>
+  __device__ __forceinline__ uint64_t make(TM t, uint32_t cls, uint32_t op) const {
+    using U = typename std::make_unsigned<TM>::type;
+    return ((uint64_t)(U)t << (ib + 2)) | ((uint64_t)cls << ib) | (uint64_t)op;
+  }
+  __device__ __forceinline__ int64_t time(uint64_t k) const { return (int64_t)(k >> (ib + 2)); }
+  __device__ __forceinline__ uint64_t time_floor(int64_t t) const { return (uint64_t)t << (ib + 2); }
+  __device__ __forceinline__ uint32_t cls(uint64_t k) const { return (uint32_t)(k >> ib) & 3u; }
+  __device__ __forceinline__ uint32_t op(uint64_t k) const { return (uint32_t)(k & mask); }
+};
+
+// ---------------------------------------------------------------------------
+// READY keys: warp-cooperative 32-ary min-heap.  Slots [0, qs) are in shared
+// memory (qs >= 33, so the root and its children always are), the rest in
+// the warp's global scratch.  All lanes call every method with the same
+// arguments; lane 0 performs the stores.
+// ---------------------------------------------------------------------------
+struct ReadyHeap {
+  uint64_t* sk;
+  uint64_t* gk;
+  int qs, cap, size;
+
+  __device__ __forceinline__ uint64_t* kp(int i) const { return i < qs ? sk + i : gk + (i - qs); }
+  __device__ __forceinline__ uint64_t top() const { return size > 0 ? sk[0] : kKeyMax; }
+
+  __device__ void sift_down(int pos, uint64_t x) {
+    const unsigned lane = lane_id();
+    while (true) {
+      const int c0 = pos * 32 + 1;
+      if (c0 >= size) break;
+      const int idx = c0 + (int)lane;
+      uint64_t ck = kKeyMax;
+      if (idx < size) ck = c0 == 1 ? sk[idx] : *kp(idx);
+      const uint64_t m = warp_min_u64(ck);
+      if (m >= x) break;
+      const int src = __ffs(__ballot_sync(kFullMask, ck == m)) - 1;
+      if (lane == 0) *kp(pos) = m;
+      pos = c0 + src;
+    }
+    if (lane == 0) *kp(pos) = x;
+    __syncwarp();
+  }
+
+  __device__ void pop() {
+    const int n = --size;
+    if (n == 0) return;
+    const uint64_t x = *kp(n);
+    sift_down(0, x);
+  }
+
+  __device__ bool push(uint64_t key) {
+    if (size >= cap) return false;
+    int pos = size++;
+    while (pos > 0) {
+      const int par = (pos - 1) >> 5;
+      const uint64_t pk = *kp(par);
+      if (pk <= key) break;
+      if (lane_id() == 0) *kp(pos) = pk;
+      pos = par;
+    }
+    if (lane_id() == 0) *kp(pos) = key;
+    __syncwarp();
+    return true;
+  }
+
+  __device__ void heapify() {
+    if (size < 2) return;
+    for (int pos = (size - 2) / 32; pos >= 0; --pos) {
+      const uint64_t x = *kp(pos);
+      __syncwarp();
+      sift_down(pos, x);
+    }
+  }
+};
+
+// ---------------------------------------------------------------------------
+// HBM event log: unordered 8-byte entries -- (accelerator << ds) | key when
+// the accelerator id fits above the key, else the key with the accelerator
+// in a side byte array.  Slots [0, ms) are in shared memory, the rest in
+// global scratch.
+// ---------------------------------------------------------------------------
+struct MemLog {
+  uint64_t* sk;
+  uint8_t* sd;
+  uint64_t* gk;
+  uint8_t* gd;
+  int ms, cap, n;
+
+  __device__ __forceinline__ uint64_t* kp(int i) const { return i < ms ? sk + i : gk + (i - ms); }
+  __device__ __forceinline__ uint8_t* dp(int i) const { return i < ms ? sd + i : gd + (i - ms); }
+};
+
+// ---------------------------------------------------------------------------
+// Per-accelerator state.  Free times: with at most 32 accelerators lane d
+// holds accelerator d's in a register, else a shared array.  Live and peak
+// bytes: shared arrays (the drain updates them a batch at a time).
+// ---------------------------------------------------------------------------
+template <bool kReg, typename TM>
+struct Devices {
+  TM fr_reg;
+  int64_t* fr;  // shared [D] (when !kReg)
+  int64_t* lv;  // shared [D]
+  int64_t* pk;  // shared [D]
+  int D;
+  __device__ void setup(const DevGmg& g, int64_t* sm) {
+    D = g.D;
+    fr = sm;
+    lv = sm + (kReg ? 0 : D);
+    pk = lv + D;
+  }
+  __device__ void reset(const DevGmg& g) {
+    const unsigned l = lane_id();
+    for (int d = l; d < D; d += 32) {
+      lv[d] = g.base[d];
+      pk[d] = g.base[d];
+      if (!kReg) fr[d] = g.avail0[d];
+    }
+    if (kReg) fr_reg = l < (unsigned)D ? (TM)g.avail0[l] : (TM)0;
+    __syncwarp();
+  }
+  __device__ __forceinline__ TM get_free(int d) const {
+    if (kReg) return __shfl_sync(kFullMask, fr_reg, d);
+    return (TM)fr[d];
+  }
+  __device__ __forceinline__ void set_free(int d, TM v) {
+    if (kReg) {
+      if ((int)lane_id() == d) fr_reg = v;
+    } else {
+      __syncwarp();
+      if (lane_id() == 0) fr[d] = v;
+    }
+  }
+  // One event at a time (used when accelerator ids do not fit in the sort key).
+  __device__ __forceinline__ bool alloc(int d, int64_t b, int64_t cap) {
+    const int64_t v = lv[d] + b;
+    const int64_t p = pk[d];
+    __syncwarp();
+    if (lane_id() == 0) {
+      lv[d] = v;
+      if (v > p) pk[d] = v;
+    }
+    __syncwarp();
+    return v > cap;
+  }
+  __device__ __forceinline__ void release(int d, int64_t b) {
+    const int64_t v = lv[d] - b;
+    __syncwarp();
+    if (lane_id() == 0) lv[d] = v;
+    __syncwarp();
+  }
+  __device__ void save(int64_t* dst) const {
+    const unsigned l = lane_id();
+    for (int d = l; d < D; d += 32) {
+      if (!kReg) dst[d] = fr[d];
+      dst[D + d] = lv[d];
+      dst[2 * D + d] = pk[d];
+    }
+    if (kReg && l < (unsigned)D) dst[l] = (int64_t)fr_reg;
+  }
+  __device__ void load(const int64_t* src) {
+    const unsigned l = lane_id();
+    for (int d = l; d < D; d += 32) {
+      if (!kReg) fr[d] = src[d];
+      lv[d] = src[D + d];
+      pk[d] = src[2 * D + d];
+    }
+    if (kReg) fr_reg = l < (unsigned)D ? (TM)src[l] : (TM)0;
+    __syncwarp();
+  }
+  __device__ void write_peak(int64_t* dst) const {
+    for (int d = lane_id(); d < D; d += 32) dst[d] = pk[d];
+  }
+};
+
+// Shared-memory carve-up per warp: READY heap head, event-log head, sort
+// area, accelerator state.
+struct WarpSmem {
+  uint32_t* oplog;  // [opcap]
+  uint64_t* heap;   // [qs]
+  uint64_t* logk;   // [ms]
+  uint64_t* sortk;  // [sortcap]
+  uint8_t* logd;    // [ms]
+  uint8_t* sortd;   // [sortcap]
+  int64_t* dev;     // [3*D] (2*D used when free times are in registers)
+};
+
+__device__ __forceinline__ size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
+
+__device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P, unsigned wib) {
+  const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 +
+                              (size_t)P.opcap * 4);
+  const size_t per = head + (size_t)P.g.D * 24;
+  uint8_t* b = smem + per * wib;
+  WarpSmem w;
+  w.heap = reinterpret_cast<uint64_t*>(b);
+  w.logk = w.heap + P.qs;
+  w.sortk = w.logk + P.ms;
+  w.logd = reinterpret_cast<uint8_t*>(w.sortk + P.sortcap);
+  w.sortd = w.logd + P.ms;
+  w.oplog = reinterpret_cast<uint32_t*>(w.sortd + P.sortcap);
+  w.dev = reinterpret_cast<int64_t*>(b + head);
+  return w;
+}
+
+// ---------------------------------------------------------------------------
+// One warp's simulator.
+// ---------------------------------------------------------------------------
+// kT32: every time of the graph is below 2^31 (the host's bound), so ready,
+// start, finish, free and arrival times are carried as int32 (bytes, scores
+// and outputs stay int64).
+// kTypes: the graph has several accelerator types (durations per (type, op)).
+template <bool kReg, int kMode, bool kKey, bool kT32 = false, bool kTypes = false>
+struct Sim {
+  static_assert(!(kT32 && kMode == kBase), "the base snapshot keeps 64-bit times");
+  using tm_t = typename std::conditional<kT32, int32_t, int64_t>::type;
+  const SimParams& P;
+  const DevGmg& g;
+  KeyCodec kc;
+  ReadyHeap q;      // READY keys beyond the register tier
+  uint64_t rk_reg;  // register tier: one READY key per lane (kKeyMax = empty)
+  MemLog log;
+  uint64_t* sortk;
+  uint8_t* sortd;
+  int sortcap;
+  uint32_t* oplog;  // ops started since the last HBM-event generation
+  int opn;
+  int ds;           // accelerator shift of a log entry
+  uint64_t lowmask; // key part of a log entry
+  Devices<kReg, tm_t> dv;
+  const uint8_t* row;
+  tm_t* fbuf;       // finish times (scratch; the base's own array in kBase)
+  tm_t* holdb;      // latest outgoing arrival of each op's output (scratch)
+  uint32_t* bits;
+  int64_t* creq;
+  // incremental resume
+  const int64_t* rb;
+  const int64_t* fb;
+  tm_t Tc, T0;
+  // running results
+  int rootptr;
+  uint64_t rkey;    // root_keys[rootptr], kKeyMax past the end
+  int64_t score, iters, nev, readypops;
+  tm_t makespan, last_t;
+  int32_t vflag, vop, vdev, status;
+  int64_t vt;
+  // base checkpoints
+  int ck, next_ck;
+
+  __device__ Sim(const SimParams& p) : P(p), g(p.g) {
+    kc.ib = g.ib;
+    kc.mask = (1ull << g.ib) - 1ull;
+    ds = g.ib + 2 + g.tb;
+    lowmask = kKey ? (1ull << ds) - 1ull : kKeyMax;
+  }
+
+  __device__ __forceinline__ bool popped(uint32_t x) const { return (bits[x >> 5] >> (x & 31u)) & 1u; }
+  // Finish time of a simulated op (incremental: ops before the resume point
+  // keep their base finish).
+  // The low 32 bits of a base-snapshot time (little-endian int64).
+  static __device__ __forceinline__ tm_t base_time(const int64_t* a, uint32_t x) {
+    if (kT32) return (tm_t)__ldg(reinterpret_cast<const int32_t*>(a) + 2 * (size_t)x);
+    return (tm_t)__ldg(a + x);
+  }
+  // Duration of op i on accelerator d: by the accelerator's type when the
+  // graph has several (Sec. 3.3.1 keeps one operator estimate per (type,
+  // operator)), else the op record's dur (dflt).
+  __device__ __forceinline__ int64_t dur_of(uint32_t i, int d, int64_t dflt) const {
+    if (kTypes) return __ldg(g.durt + (size_t)i * g.ntypes + __ldg(g.dtype + d));
+    return dflt;
+  }
+  __device__ __forceinline__ tm_t fin(uint32_t x) const {
+    if (kMode == kInc && base_time(rb, x) < Tc) return base_time(fb, x);
+    return fbuf[x];
+  }
+
+  // Transfer estimator of one output over link d -> e (d != e), Sec. 3.3.1.
+  __device__ __forceinline__ tm_t xfer(int d, int e, int64_t bytes, int64_t xq) const {
+    if (g.uniform) return (tm_t)xq + (tm_t)g.lat0;
+    const longlong2* L = reinterpret_cast<const longlong2*>(g.links + (d * g.D + e));
+    const longlong2 a = __ldg(L), b = __ldg(L + 1);
+    LinkRec l;
+    l.magic = (uint64_t)a.x;
+    l.bw = a.y;
+    l.lat = b.x;
+    l.shift = (int32_t)(b.y & 0xffffffff);
+    return (tm_t)(ceil_div_link(bytes, l) + l.lat);
+  }
+
+  // Latest arrival of p's output at another accelerator (or f_p): the
+  // earliest its source copy may be released.  Per lane.
+  __device__ tm_t lane_hold(uint32_t p, tm_t fp, int dp) const {
+    const int64_t pb = op_durbytes(g.ops, p).y;
+    const int64_t pxq = op_relxq(g.ops, p).y;
+    const uint4 ls = op_lists(g.ops, p);
+    tm_t h = fp;
+    for (uint32_t u = 0; u < ls.y; ++u) {
+      const int du = row[__ldg(g.succ + ls.x + u)];
+      if (du != dp) {
+        const tm_t a = fp + xfer(dp, du, pb, pxq);
+        h = a > h ? a : h;
+      }
+    }
+    return h;
+  }
+
+
+  __device__ __forceinline__ void load_root() {
+    rkey = rootptr < g.nroots ? __ldg(g.root_keys + rootptr) : kKeyMax;
+  }
+
+  // READY keys go to a free lane's register if there is one, else the heap.
+  __device__ __forceinline__ void push_ready(uint64_t key) {
+    const uint32_t freel = __ballot_sync(kFullMask, rk_reg == kKeyMax);
+    if (freel) {
+      if ((int)lane_id() == __ffs(freel) - 1) rk_reg = key;
+    } else if (!q.push(key)) {
+      status = GMG_SIM_QUEUE;
+    }
+  }
+  // Every lane with `want` logs (key, dev).  Uniform call.
+  __device__ __forceinline__ void log_event(bool want, uint64_t key, int dev) {
+    const uint32_t b = __ballot_sync(kFullMask, want);
+    const int cnt = __popc(b);
+    const int pos = log.n + __popc(b & lanes_below());
+    if (kKey && log.n + 32 <= log.ms) {
+      // fast path: every lane's slot is in shared memory
+      if (want) log.sk[pos] = ((uint64_t)(dev & 0xff) << ds) | key;
+      log.n += cnt;
+      return;
+    }
+    if (cnt == 0 || status) return;
+    if (log.n + cnt > log.cap) {
+      status = GMG_SIM_QUEUE;
+      return;
+    }
+    if (want) {
+      *log.kp(pos) = kKey ? (((uint64_t)(dev & 0xff) << ds) | key) : key;
+      if (!kKey) *log.dp(pos) = (uint8_t)dev;
+    }
+    log.n += cnt;
+  }
+
+  __device__ void reset_common() {
+    const unsigned lane = lane_id();
+    const int words = (g.n + 31) >> 5;
+    for (int w = lane; w < words; w += 32) bits[w] = 0u;
+    for (int r = lane; r < g.R; r += 32) creq[r] = 0;
+    dv.reset(g);
+    q.size = 0;
+    rk_reg = kKeyMax;
+    log.n = 0;
+    opn = 0;
+    rootptr = 0;
+    load_root();
+    score = makespan = 0;
+    iters = nev = readypops = 0;
+    last_t = -1;
+    vflag = 0;
+    vop = vdev = -1;
+    vt = -1;
+    status = GMG_SIM_OK;
+    __syncwarp();
+  }
+
+  // -------------------------------------------------------------------------
+  // READY(r, i): start op i (Sec. 3.3.2/3.3.3), record it for HBM-event
+  // generation, and push the successors it makes ready.
+  // -------------------------------------------------------------------------
+  __device__ void start_op(uint32_t i, tm_t r) {
+    const unsigned lane = lane_id();
+    const longlong2 db = op_durbytes(g.ops, i);
+    const longlong2 rx = op_relxq(g.ops, i);
+    const uint4 ls = op_lists(g.ops, i);
+    const uint4 cs = op_cons(g.ops, i);
+    const int64_t bytes = db.y, xq = rx.y;
+    const uint32_t succ_off = ls.x, nsucc = ls.y;
+    const uint32_t flags = cs.w;
+    const int d = row[i];
+    const tm_t dur = (tm_t)dur_of(i, d, db.x);
+    const tm_t fd = dv.get_free(d);
+    const tm_t s = r > fd ? r : fd;
+    const tm_t f = s + dur;
+    dv.set_free(d, f);
+    if (lane == 0) {
+      fbuf[i] = f;
+      atomicOr(&bits[i >> 5], 1u << (i & 31u));
+      if (flags & kReqSink)
+        atomicMax(reinterpret_cast<unsigned long long*>(creq + (int32_t)cs.z), (unsigned long long)f);
+      if (kMode == kBase) P.base.rb[i] = r;
+      oplog[opn] = i;
+    }
+    ++opn;
+    if (flags & kScored) score += (int64_t)f;
+    makespan = f > makespan ? f : makespan;
+    if (kMode != kInc || r >= T0) ++nev;
+    if (kMode == kBase) ++readypops;
+    __syncwarp();
+
+    // Successors: a successor is ready once every predecessor has finished;
+    // its ready time is the latest arrival over all of them.
+    for (uint32_t c0 = 0; c0 < nsucc; c0 += 32) {
+      const uint32_t t = c0 + lane;
+      uint32_t j = 0;
+      tm_t rj = 0;
+      bool rdy = false;
+      if (t < nsucc) {
+        j = __ldg(g.succ + succ_off + t);
+        const int dj = row[j];
+        tm_t arr = f;
+        if (dj != d) arr = f + xfer(d, dj, bytes, xq);
+        const longlong2 jrx = op_relxq(g.ops, j);
+        const uint4 jls = op_lists(g.ops, j);
+        const tm_t rel = (tm_t)jrx.x;
+        rj = rel > arr ? rel : arr;
+        rdy = true;
+        if (jls.w > 1) {
+          for (uint32_t k = 0; k < jls.w; ++k) {
+            const uint32_t p = __ldg(g.pred + jls.z + k) & kIdMask;
+            if (p == i) continue;
+            if (!popped(p)) {
+              rdy = false;
+              break;
+            }
+            const int dp = row[p];
+            tm_t a = fin(p);
+            if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
+            rj = a > rj ? a : rj;
+          }
+        }
+      }
+      uint32_t m = __ballot_sync(kFullMask, rdy);
+      while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        push_ready(__shfl_sync(kFullMask, kc.make(rj, kReady, j), src));
+      }
+    }
+  }
+
+  // -------------------------------------------------------------------------
+  // HBM events of the ops started since the last generation, one op per lane
+  // (Sec. 3.3.2 residency, Recv before Send of Sec. 3.5.2): the op's own
+  // output allocated at s; a receive copy on every other accelerator of a
+  // successor allocated at f (released on arrival if no listed consumer is
+  // there); the own copy released at the latest outgoing arrival if no
+  // listed consumer is local; and for every held input whose last local
+  // consumer this op is, that copy released at f (an own copy not before its
+  // producer's outgoing arrivals).  Ops on one accelerator finish in the
+  // order they start, so "last consumer here" compares finish times and can
+  // be decided any time after the op started.
+  // -------------------------------------------------------------------------
+  __device__ void generate() {
+    const unsigned lane = lane_id();
+    for (int c0 = 0; c0 < opn; c0 += 32) {
+      const int idx = c0 + (int)lane;
+      const bool v = idx < opn;
+      const uint32_t x = v ? oplog[idx] : 0u;
+      longlong2 db = make_longlong2(0, 0), rx = make_longlong2(0, 0);
+      uint4 ls = make_uint4(0, 0, 0, 0), cs = make_uint4(0, 0, 0, 0);
+      int d = 0;
+      tm_t f = 0;
+      if (v) {
+        db = op_durbytes(g.ops, x);
+        rx = op_relxq(g.ops, x);
+        ls = op_lists(g.ops, x);
+        cs = op_cons(g.ops, x);
+        d = row[x];
+        f = fbuf[x];
+      }
+      const int64_t bytes = db.y, xq = rx.y;
+      const bool allcons = (cs.w & kAllCons) != 0;
+      log_event(v, kc.make(f - (tm_t)dur_of(x, d, db.x), kAlloc, x), d);
+      // receive copies, one per distinct remote accelerator
+      tm_t hold = f;
+      bool localc = false;
+      const uint32_t nsx = ls.y;
+      const uint32_t maxs = __reduce_max_sync(kFullMask, nsx);
+      const bool anyexp = __any_sync(kFullMask, v && !allcons);
+      for (uint32_t u = 0; u < maxs; ++u) {
+        bool want = false, nocons = false;
+        int du = 0;
+        tm_t arr = f;
+        if (u < nsx) {
+          du = row[__ldg(g.succ + ls.x + u)];
+          if (du == d) {
+            localc = true;
+          } else {
+            want = true;
+            for (uint32_t w = 0; w < u; ++w)
+              if (row[__ldg(g.succ + ls.x + w)] == du) {
+                want = false;
+                break;
+              }
+          }
+          if (want) {
+            arr = f + xfer(d, du, bytes, xq);
+            hold = arr > hold ? arr : hold;
+            if (!allcons) {
+              nocons = true;
+              for (uint32_t w = 0; w < cs.y; ++w)
+                if (row[__ldg(g.cons + cs.x + w)] == du) {
+                  nocons = false;
+                  break;
+                }
+            }
+          }
+        }
+        log_event(want, kc.make(f, kAlloc, x), du);
+        if (anyexp) log_event(nocons, kc.make(arr, kFree, x), du);
+      }
+      if (v && !allcons) {
+        localc = false;
+        for (uint32_t w = 0; w < cs.y; ++w)
+          if (row[__ldg(g.cons + cs.x + w)] == d) {
+            localc = true;
+            break;
+          }
+      }
+      log_event(v && !localc, kc.make(hold, kFree, x), d);
+      if (v) holdb[x] = hold;
+      __syncwarp();
+      // releases of the inputs this op holds
+      const uint32_t npx = ls.w;
+      const uint32_t maxp = __reduce_max_sync(kFullMask, npx);
+      for (uint32_t u = 0; u < maxp; ++u) {
+        bool rel = false;
+        tm_t T = f;
+        uint32_t p = 0;
+        if (u < npx) {
+          const uint2 ps = __ldg(g.predsib + ls.z + u);
+          p = ps.x & kIdMask;
+          if (ps.x & kHoldBit) {
+            const uint32_t sb = ps.y;
+            if (sb == kSibNone) {
+              rel = true;
+            } else if (sb != kSibMany && (sb & kSibLater)) {
+              rel = row[sb & ~kSibLater] != d;  // the other consumer finishes later
+            } else if (sb != kSibMany) {
+              rel = !(row[sb] == d && !(popped(sb) && fin(sb) < f));
+            } else {
+              const uint4 pls = op_lists(g.ops, p);
+              const uint4 pcs = op_cons(g.ops, p);
+              const bool all = (pcs.w & kAllCons) != 0;
+              const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
+              const uint32_t nl = all ? pls.y : pcs.y;
+              rel = true;
+              for (uint32_t w = 0; w < nl; ++w) {
+                const uint32_t c = __ldg(lst + w);
+                if (c != x && row[c] == d && !(popped(c) && fin(c) < f)) {
+                  rel = false;
+                  break;
+                }
+              }
+            }
+            if (rel && row[p] == d) {
+              // p's own copy: not before its outgoing arrivals (recorded when
+              // p's events were generated; p started before this op)
+              const tm_t h = (kMode == kInc && base_time(rb, p) < Tc) ? lane_hold(p, fin(p), d) : holdb[p];
+              T = h > T ? h : T;
+            }
+          }
+        }
+        log_event(rel, kc.make(T, kFree, p), d);
+      }
+    }
+    opn = 0;
+    __syncwarp();
+  }
+
+  // Apply sorted events one at a time (accelerator ids not in the key).
+  __device__ void apply_serial(int m) {
+    for (int e = 0; e < m; ++e) {
+      const uint64_t k = sortk[e];
+      const int dev = sortd[e];
+      const uint32_t op = kc.op(k);
+      const int64_t b = op_durbytes(g.ops, op).y;
+      if (kc.cls(k) == kFree) {
+        dv.release(dev, b);
+      } else if (dv.alloc(dev, b, __ldg(g.cap + dev))) {
+        const int64_t t = kc.time(k);
+        if (!vflag || (t == vt && (int32_t)op == vop && dev < vdev)) {
+          vflag = 1;
+          vt = t;
+          vop = (int32_t)op;
+          vdev = dev;
+        }
+      }
+    }
+    __syncwarp();
+  }
+
+  // Apply 32 consecutive events of the (accelerator, time, class, op) order,
+  // one per lane (v: lane holds an event).  Each accelerator's events are
+  // contiguous, so a segmented warp scan of the byte deltas gives the live
+  // bytes after every event; allocations raise the accelerator's peak; the
+  // smallest (time, op, accelerator) allocation over capacity is kept in
+  // vmin.
+  __device__ __forceinline__ void apply_chunk(uint64_t key, bool v, uint64_t& vmin) {
+    const unsigned lane = lane_id();
+    const uint64_t tmask = (1ull << g.tb) - 1ull;
+    const int dev = v ? (int)(key >> ds) : -1 - (int)lane;
+    const uint32_t op = (uint32_t)(key & kc.mask);
+    const bool isalloc = v && kc.cls(key) == kAlloc;
+    int64_t delta = 0;
+    if (v) {
+      const int64_t b = op_durbytes(g.ops, op).y;
+      delta = isalloc ? b : -b;
+    }
+    int64_t s = delta;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const int64_t o = __shfl_up_sync(kFullMask, s, off);
+      const int od = __shfl_up_sync(kFullMask, dev, off);
+      if ((int)lane >= off && od == dev) s += o;
+    }
+    const int64_t live = (v ? dv.lv[dev] : 0) + s;
+    const int nd = __shfl_down_sync(kFullMask, dev, 1);
+    const bool last = v && (lane == 31 || nd != dev);
+    const bool over = isalloc && live > __ldg(g.cap + dev);
+    const uint64_t vk = over ? ((((key >> (g.ib + 2)) & tmask) << (g.ib + 8)) | ((uint64_t)op << 8) |
+                                (uint64_t)dev)
+                             : kKeyMax;
+    const uint64_t cm = warp_min_u64(vk);
+    vmin = cm < vmin ? cm : vmin;
+    __syncwarp();
+    if (isalloc)  // live bytes are never negative
+      atomicMax(reinterpret_cast<unsigned long long*>(dv.pk + dev), (unsigned long long)live);
+    if (last) dv.lv[dev] = live;
+    __syncwarp();
+  }
+
+  // every event of a drain is later than every event already applied, so
+  // an earlier violation stands
+  __device__ __forceinline__ void settle_violation(uint64_t vmin) {
+    if (!vflag && vmin != kKeyMax) {
+      vflag = 1;
+      vt = (int64_t)(vmin >> (g.ib + 8));
+      vop = (int32_t)((vmin >> 8) & kc.mask);
+      vdev = (int32_t)(vmin & 0xffu);
+    }
+  }
+
+  __device__ void apply_segmented(int m) {
+    uint64_t vmin = kKeyMax;
+    for (int c0 = 0; c0 < m; c0 += 32) {
+      const int idx = c0 + (int)lane_id();
+      const bool v = idx < m;
+      apply_chunk(v ? sortk[idx] : 0ull, v, vmin);
+    }
+    settle_violation(vmin);
+  }
+
+  // Bitonic sort of 32*E keys held in registers: lane l holds elements
+  // l + 32 e.  Pairs 32 or more apart meet inside a lane, closer pairs via
+  // shfl_xor.  Fully unrolled.
+  template <int E>
+  static __device__ __forceinline__ void reg_bitonic(uint64_t (&a)[E]) {
+    const int lane = (int)lane_id();
+#pragma unroll
+    for (int k = 2; k <= 32 * E; k <<= 1) {
+#pragma unroll
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        if (j >= 32) {
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const int e2 = e ^ (j >> 5);
+            if (e2 > e) {
+              const bool asc = ((lane + 32 * e) & k) == 0;
+              const uint64_t x = a[e], y = a[e2];
+              const bool sw = asc ? (x > y) : (x < y);
+              a[e] = sw ? y : x;
+              a[e2] = sw ? x : y;
+            }
+          }
+        } else {
+#pragma unroll
+          for (int e = 0; e < E; ++e) {
+            const uint64_t o = __shfl_xor_sync(kFullMask, a[e], j);
+            const bool keep_min = ((lane & j) == 0) == (((lane + 32 * e) & k) == 0);
+            a[e] = (keep_min == (o < a[e])) ? o : a[e];
+          }
+        }
+      }
+    }
+  }
+
+  template <int E>
+  __device__ __forceinline__ void sort_apply_regs_e(int m) {
+    const int lane = (int)lane_id();
+    uint64_t a[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) a[e] = lane + 32 * e < m ? sortk[lane + 32 * e] : kKeyMax;
+    reg_bitonic<E>(a);
+    uint64_t vmin = kKeyMax;
+#pragma unroll
+    for (int e = 0; e < E; ++e) apply_chunk(a[e], lane + 32 * e < m, vmin);
+    settle_violation(vmin);
+  }
+
+  // Sort and apply m <= 32 extracted events in registers.  (Wider register
+  // networks sort faster but their unrolled code -- each inlining its own
+  // copies of the segmented apply -- overflowed the instruction cache: larger
+  // drains go through the shared-memory sort.)
+  __device__ void sort_apply_regs(int m) { sort_apply_regs_e<1>(m); }
+
+  __device__ int count_below(uint64_t kmax) const {
+    int c = 0;
+    for (int c0 = 0; c0 < log.n; c0 += 32) {
+      const int idx = c0 + (int)lane_id();
+      const bool take = idx < log.n && (*log.kp(idx) & lowmask) < kmax;
+      c += __popc(__ballot_sync(kFullMask, take));
+    }
+    return c;
+  }
+
+  // Move the logged events whose key part is < kmax to the sort area (their
+  // number is known to fit) and compact the rest; returns their number.
+  __device__ int extract(uint64_t kmax) {
+    const unsigned lane = lane_id();
+    const bool side = !kKey;
+    int m = 0, keep = 0;
+    const int n = log.n;
+    for (int c0 = 0; c0 < n; c0 += 32) {
+      const int idx = c0 + (int)lane;
+      const bool v = idx < n;
+      uint64_t e = kKeyMax;
+      uint8_t dv8 = 0;
+      if (v) {
+        if (idx < log.ms) {
+          e = log.sk[idx];
+          if (side) dv8 = log.sd[idx];
+        } else {
+          e = *log.kp(idx);
+          if (side) dv8 = *log.dp(idx);
+        }
+      }
+      const bool take = v && (e & lowmask) < kmax;
+      const uint32_t bt = __ballot_sync(kFullMask, take);
+      const uint32_t bk = __ballot_sync(kFullMask, v && !take);
+      if (take) {
+        const int pos = m + __popc(bt & lanes_below());
+        sortk[pos] = e;
+        if (side) sortd[pos] = dv8;
+      } else if (v) {
+        const int pos = keep + __popc(bk & lanes_below());  // pos <= idx: in place
+        *log.kp(pos) = e;
+        if (side) *log.dp(pos) = dv8;
+      }
+      m += __popc(bt);
+      keep += __popc(bk);
+      __syncwarp();
+    }
+    log.n = keep;
+    return m;
+  }
+
+  // Bitonic sort of sortk[0, m) (and the side bytes alongside), padded to a
+  // power of two >= 32.
+  __device__ void sort_area(int m) {
+    const unsigned lane = lane_id();
+    const bool side = !kKey;
+    int p2 = 32;
+    while (p2 < m) p2 <<= 1;
+    for (int x = m + (int)lane; x < p2; x += 32) sortk[x] = kKeyMax;
+    __syncwarp();
+    for (int k = 2; k <= p2; k <<= 1) {
+      for (int j = k >> 1; j > 0; j >>= 1) {
+        for (int t = lane; t < (p2 >> 1); t += 32) {
+          const int i = ((t & ~(j - 1)) << 1) | (t & (j - 1));
+          const int l = i + j;
+          const uint64_t a = sortk[i], b = sortk[l];
+          const bool asc = (i & k) == 0;
+          if ((a > b) == asc) {
+            sortk[i] = b;
+            sortk[l] = a;
+            if (side) {
+              const uint8_t da = sortd[i], db = sortd[l];
+              sortd[i] = db;
+              sortd[l] = da;
+            }
+          }
+        }
+        __syncwarp();
+      }
+    }
+  }
+
+  // Apply every logged event that can no longer be preceded (time < t_next).
+  __device__ void drain(int64_t t_next) {
+    generate();
+    const uint64_t lim = t_next == kI64Max ? kKeyMax : kc.time_floor(t_next);
+    while (log.n > 0) {
+      uint64_t kmax = lim;
+      if (log.n > sortcap) {
+        const int due = count_below(lim);
+        if (due == 0) break;
+        if (due > sortcap) {
+          // Rare: more due events than the sort area.  Bisect a key bound
+          // with at most sortcap events below it (at most n_dev <= sortcap
+          // events share a key part).
+          uint64_t lo = kKeyMax;
+          for (int c0 = 0; c0 < log.n; c0 += 32) {
+            const int idx = c0 + (int)lane_id();
+            const uint64_t kk = idx < log.n ? (*log.kp(idx) & lowmask) : kKeyMax;
+            lo = kk < lo ? kk : lo;
+          }
+          lo = warp_min_u64(lo) + 1;  // 1 <= count_below(lo) <= sortcap
+          uint64_t hi = lim;          // count_below(hi) > sortcap
+          while (hi - lo > 1) {
+            const uint64_t mid = lo + (hi - lo) / 2;
+            if (count_below(mid) <= sortcap) lo = mid;
+            else hi = mid;
+          }
+          kmax = lo;
+        }
+      }
+      const int m = extract(kmax);
+      if (m == 0) break;
+      if (kKey && m <= 32) {
+        sort_apply_regs(m);
+      } else {
+        sort_area(m);
+        if (kKey) apply_segmented(m);
+        else apply_serial(m);
+      }
+      if (kmax == lim) break;
+    }
+  }
+
+  __device__ void maybe_checkpoint(uint64_t next_key);
+
+  // The event loop (Sec. 3.3.3).
+  __device__ void run() {
+    if (status) return;
+    while (true) {
+      const uint64_t top = q.top();
+      const uint64_t rm = warp_min_u64(rk_reg);
+      const uint64_t rk = rkey;
+      uint64_t nk = rk < top ? rk : top;
+      nk = rm < nk ? rm : nk;
+      if (kMode == kBase) maybe_checkpoint(nk);
+      if (nk == kKeyMax) break;
+      if (opn >= P.opcap) drain(kc.time(nk));
+      if (nk == rm) {
+        if (rk_reg == rm) rk_reg = kKeyMax;  // keys are unique
+      } else if (nk == rk) {
+        ++rootptr;
+        load_root();
+      } else {
+        __syncwarp();
+        q.pop();
+      }
+      if (++iters > g.max_iter) {
+        status = GMG_SIM_LOOP;
+        break;
+      }
+      const tm_t t = (tm_t)kc.time(nk);
+      last_t = t;
+      start_op(kc.op(nk), t);
+      if (status) break;
+    }
+    if (!status) drain(kI64Max);
+  }
+
+  __device__ void write_invalid(int64_t k, int32_t st) {
+    const DevOut& o = P.out;
+    const unsigned lane = lane_id();
+    if (lane == 0) {
+      o.makespan[k] = 0;
+      o.score[k] = kI64Max;
+      o.status[k] = st;
+      o.viol_flag[k] = 0;
+      o.viol_op[k] = -1;
+      o.viol_dev[k] = -1;
+      o.viol_time[k] = -1;
+      o.sla_miss[k] = 0;
+      o.events[k] = 0;
+    }
+    for (int d = lane; d < g.D; d += 32) o.peak[k * g.D + d] = 0;
+    if (o.req_done)
+      for (int r = lane; r < g.R; r += 32) o.req_done[k * g.R + r] = 0;
+    const int ts = trace_slot(k);
+    if (ts >= 0)
+      for (int x = lane; x < g.n; x += 32) {
+        o.trace_start[(int64_t)ts * g.n + x] = 0;
+        o.trace_finish[(int64_t)ts * g.n + x] = 0;
+      }
+  }
+
+  __device__ int trace_slot(int64_t k) const {
+    if (P.n_trace == 0) return -1;
+    int ts = -1;
+    for (int t = lane_id(); t < P.n_trace; t += 32)
+      if (P.trace_k[t] == k) ts = t;
+    return __reduce_max_sync(kFullMask, ts);
+  }
+
+  __device__ void finish(int64_t k) {
+    if (status != GMG_SIM_OK) {
+      write_invalid(k, status);
+      return;
+    }
+    const DevOut& o = P.out;
+    const unsigned lane = lane_id();
+    int32_t miss = 0;
+    for (int r = lane; r < g.R; r += 32) {
+      const int64_t c = creq[r];
+      miss += c > __ldg(g.deadline + r) ? 1 : 0;
+      if (o.req_done) o.req_done[k * g.R + r] = c;
+    }
+    miss = (int32_t)__reduce_add_sync(kFullMask, (unsigned)miss);
+    dv.write_peak(o.peak + k * g.D);
+    if (lane == 0) {
+      o.makespan[k] = makespan;
+      o.score[k] = vflag ? kI64Max : score;
+      o.status[k] = GMG_SIM_OK;
+      o.viol_flag[k] = vflag;
+      o.viol_op[k] = vop;
+      o.viol_dev[k] = vdev;
+      o.viol_time[k] = vt;
+      o.sla_miss[k] = miss;
+      o.events[k] = nev;
+    }
+    const int ts = trace_slot(k);
+    if (ts >= 0)
+      for (int x = lane; x < g.n; x += 32) {
+        const int64_t fx = (int64_t)fin((uint32_t)x);
+        o.trace_finish[(int64_t)ts * g.n + x] = fx;
+        o.trace_start[(int64_t)ts * g.n + x] = fx - dur_of((uint32_t)x, row[x], op_durbytes(g.ops, (uint32_t)x).x);
+      }
+  }
+
+  // Any placement byte >= D?  (16-byte coalesced loads of the row.)
+  __device__ bool row_has_bad_device(const uint8_t* rw) const {
+    if (g.D >= 256) return false;
+    const unsigned lane = lane_id();
+    const uint32_t dd = (uint32_t)g.D * 0x01010101u;
+    bool bad = false;
+    for (int c = lane * 16; c < g.n; c += 512) {
+      const uint4 v = *reinterpret_cast<const uint4*>(rw + c);
+      const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        uint32_t ge = __vcmpgeu4(w[h], dd);
+        const int first = c + 4 * h;
+        if (first + 4 > g.n) {
+          const int keep = g.n - first;  // bytes of this word inside the row
+          ge = keep <= 0 ? 0u : (ge & (0xffffffffu >> (8 * (4 - keep))));
+        }
+        bad |= ge != 0u;
+      }
+    }
+    return __any_sync(kFullMask, bad);
+  }
+};
+
+// Base-mode checkpoint: at a time boundary (nothing at the next key's time
+// handled yet), save the complete simulator state -- simulated-op bitmap,
+// accelerator state, READY heap, event log, partial results.  An
+// incremental candidate whose resume time T0 is >= that time restarts there.
+template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes>
+__device__ void Sim<kReg, kMode, kKey, kT32, kTypes>::maybe_checkpoint(uint64_t next_key) {
+  if (kMode != kBase) return;
+  const DevBase& B = P.base;
+  if (next_key == kKeyMax || ck >= B.nck || readypops < next_ck) return;
+  const int64_t tn = kc.time(next_key);
+  if (tn <= last_t) return;
+  const unsigned lane = lane_id();
+  generate();
+  const bool hasreg = rk_reg != kKeyMax;
+  const uint32_t regm = __ballot_sync(kFullMask, hasreg);
+  const int nready = q.size + __popc(regm);
+  if (nready <= B.ckq && log.n <= B.ckm) {
+    int64_t* sc = B.ck_scalars + (int64_t)ck * 8;
+    if (hasreg) B.ck_qkey[(int64_t)ck * B.ckq + q.size + __popc(regm & lanes_below())] = rk_reg;
+    if (lane == 0) {
+      B.ck_time[ck] = tn;
+      sc[0] = nready;
+      sc[1] = rootptr;
+      sc[2] = score;
+      sc[3] = makespan;
+      sc[4] = vflag;
+      sc[5] = vt;
+      sc[6] = ((int64_t)vop << 32) | (uint32_t)vdev;
+      sc[7] = log.n;
+    }
+    dv.save(B.ck_dev + (int64_t)ck * 3 * g.D);
+    for (int r = lane; r < g.R; r += 32) B.ck_creq[(int64_t)ck * g.R + r] = creq[r];
+    for (int x = lane; x < q.size; x += 32) B.ck_qkey[(int64_t)ck * B.ckq + x] = *q.kp(x);
+    for (int x = lane; x < log.n; x += 32) {
+      B.ck_mkey[(int64_t)ck * B.ckm + x] = *log.kp(x);
+      B.ck_mdev[(int64_t)ck * B.ckm + x] = *log.dp(x);
+    }
+    const int words = (g.n + 31) >> 5;
+    for (int w = lane; w < words; w += 32) B.ck_bits[(int64_t)ck * B.ck_words + w] = bits[w];
+  } else if (lane == 0) {
+    B.ck_time[ck] = kI64Max;
+  }
+  ++ck;
+  next_ck += B.stride_pops;
+  __syncwarp();
+}
+
+template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes>
+__device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes>& S, const SimParams& P, unsigned wib, int64_t slot,
+                           uint8_t* smem) {
+  uint8_t* sl = P.scratch + slot * P.slot_bytes;
+  const WarpSmem w = carve_smem(smem, P, wib);
+  S.q.sk = w.heap;
+  S.q.gk = reinterpret_cast<uint64_t*>(sl + P.off_qk);
+  S.q.qs = P.qs;
+  S.q.cap = P.qcap;
+  S.q.size = 0;
+  S.log.sk = w.logk;
+  S.log.sd = w.logd;
+  S.log.gk = reinterpret_cast<uint64_t*>(sl + P.off_mk);
+  S.log.gd = sl + P.off_md;
+  S.log.ms = P.ms;
+  S.log.cap = P.mcap;
+  S.log.n = 0;
+  S.sortk = w.sortk;
+  S.sortd = w.sortd;
+  S.oplog = w.oplog;
+  S.opn = 0;
+  S.sortcap = P.sortcap;
+  S.fbuf = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32, kTypes>::tm_t*>(sl + P.off_f);
+  S.holdb = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32, kTypes>::tm_t*>(sl + P.off_hold);
+  S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
+  S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
+  S.dv.setup(P.g, w.dev);
+  S.T0 = -1;
+  S.Tc = 0;
+}
+
+}  // namespace
+}  // namespace gsim

@@ -39,7 +39,8 @@ class _Desc(C.Structure):
                 ("n_req", C.c_int32)] + [(n, C.c_void_p) for n in (
                     "pred_off", "pred_idx", "cons_off", "cons_idx", "dur_us", "out_bytes",
                     "release_us", "req_id", "scored", "deadline_us", "cap_bytes", "base_bytes",
-                    "avail0_us", "bw_B_per_us", "lat_us")]
+                    "avail0_us", "bw_B_per_us", "lat_us")] + [
+        ("n_types", C.c_int32), ("dev_type", C.c_void_p), ("dur_by_type", C.c_void_p)]
 
 
 class _Opts(C.Structure):
@@ -119,7 +120,8 @@ class _DescHolder:
         self.c = _Desc(d.n_ops, d.n_edges, d.n_dev, d.n_req, _np_ptr(d.pred_off), _np_ptr(d.pred_idx),
                        _np_ptr(d.cons_off), _np_ptr(d.cons_idx), _np_ptr(d.dur), _np_ptr(d.out_bytes),
                        _np_ptr(d.release), _np_ptr(d.req_id), _np_ptr(d.scored), _np_ptr(d.deadline),
-                       _np_ptr(d.cap), _np_ptr(d.base), _np_ptr(d.avail0), _np_ptr(d.bw), _np_ptr(d.lat))
+                       _np_ptr(d.cap), _np_ptr(d.base), _np_ptr(d.avail0), _np_ptr(d.bw), _np_ptr(d.lat),
+                       d.n_types, _np_ptr(d.dev_type), _np_ptr(d.dur_by_type))
 
 
 def gmg_workspace_bytes(desc) -> int:

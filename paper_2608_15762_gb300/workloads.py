@@ -46,6 +46,7 @@ from __future__ import annotations
 
 import json
 import os
+import dataclasses
 from dataclasses import dataclass
 from typing import List, Optional, Sequence
 
@@ -86,6 +87,20 @@ class GmgDesc:
     lat: np.ndarray
     cons_off: Optional[np.ndarray] = None
     cons_idx: Optional[np.ndarray] = None
+    # heterogeneous accelerators: the type of each accelerator and every op's
+    # duration on every type ([N, T]); None = one type, `dur` everywhere
+    dev_type: Optional[np.ndarray] = None
+    dur_by_type: Optional[np.ndarray] = None
+
+    @property
+    def n_types(self) -> int:
+        return 0 if self.dur_by_type is None else int(np.asarray(self.dur_by_type).shape[1])
+
+    def dur_on(self, i: int, d: int) -> int:
+        """Duration of op i on accelerator d."""
+        if self.dur_by_type is None:
+            return int(self.dur[i])
+        return int(self.dur_by_type[i][int(self.dev_type[d])])
 
     @property
     def n_ops(self) -> int:
@@ -112,7 +127,8 @@ class GmgDesc:
             cap=c(self.cap, np.int64), base=c(self.base, np.int64),
             avail0=c(self.avail0, np.int64), bw=c(self.bw, np.int64),
             lat=c(self.lat, np.int64), cons_off=c(self.cons_off, np.int32),
-            cons_idx=c(self.cons_idx, np.int32))
+            cons_idx=c(self.cons_idx, np.int32), dev_type=c(self.dev_type, np.uint8),
+            dur_by_type=c(self.dur_by_type, np.int64))
 
 
 @dataclass
@@ -571,8 +587,35 @@ def config5(seed: int = 5, n_cand: int = 65536) -> Workload:
                     place_seed=seed, base_place=base, moves=moves)
 
 
+def config6(seed: int = 6) -> Workload:
+    """The prefill workload on two accelerator types: accelerators 0-3 of
+    type 0, 4-7 of type 1, slower by a factor drawn per operator kind (the
+    operator estimator is per (accelerator type, template operator),
+    Sec. 3.3.1) from U[1.3, 2.5]; deadlines from type-0 critical paths."""
+    t = prefill_template(32)
+    reqs = [t] * 8
+    pred_off, pred_idx, offs = _concat(reqs)
+    n = int(offs[-1])
+    g = _rng(seed, 1)
+    dur = lognormal_durations(g, n)
+    out_bytes = uniform_bytes(g, n, 1 * MiB, 256 * MiB)
+    kinds = np.tile(t.kind, 8)
+    uk = np.unique(kinds)
+    factor = dict(zip(uk.tolist(), _rng(seed, 2).uniform(1.3, 2.5, size=uk.shape[0]).tolist()))
+    slow = np.maximum(1, np.rint(dur * np.array([factor[k] for k in kinds.tolist()]))).astype(np.int64)
+    req_id = np.repeat(np.arange(8), np.diff(offs)).astype(np.int32)
+    release = np.zeros(n, np.int64)
+    dl = deadlines_from_critical_path(pred_off, pred_idx, dur, release, req_id, 8,
+                                      np.zeros(8, np.int64), 3, 2)
+    bw, lat = uniform_links(8, 400_000, 10)
+    d = _desc(8, pred_off, pred_idx, dur, out_bytes, release, req_id, dl, 80 * GiB, bw, lat)
+    d = dataclasses.replace(d, dev_type=np.array([0, 0, 0, 0, 1, 1, 1, 1], np.uint8),
+                            dur_by_type=np.stack([dur, slow], axis=1)).normalized()
+    return Workload("hetero-prefill-8x32L-N3088-D8-T2-K4096", 6, d, n_full=4096, place_seed=seed)
+
+
 def make_workload(config: int, **kw) -> Workload:
-    return {1: config1, 2: config2, 3: config3, 4: config4, 5: config5}[config](**kw)
+    return {1: config1, 2: config2, 3: config3, 4: config4, 5: config5, 6: config6}[config](**kw)
 
 
 # ----------------------------------------------------------------------------
@@ -583,8 +626,10 @@ def random_desc(seed: int, n_ops: int, n_dev: int, n_req: int = 2, max_pred: int
                 edge_p: float = 0.3, dur_hi: int = 50, bytes_hi: int = 1 << 12,
                 cap=None, explicit_cons: bool = False, with_release: bool = True,
                 with_avail0: bool = True, link_hetero: bool = True,
-                deadline: bool = True) -> GmgDesc:
-    """A random topologically numbered DAG with small integer values."""
+                deadline: bool = True, n_types: int = 0) -> GmgDesc:
+    """A random topologically numbered DAG with small integer values (with
+    n_types >= 2: accelerator types and per-type durations, drawn from a
+    stream of their own so the other fields match the one-type graph)."""
     g = _rng(seed, 77)
     preds = []
     for i in range(n_ops):
@@ -636,10 +681,16 @@ def random_desc(seed: int, n_ops: int, n_dev: int, n_req: int = 2, max_pred: int
             co.append(len(ci))
         cons_off = np.array(co, np.int64)
         cons_idx = np.array(ci, np.int64)
+    dev_type = dur_by_type = None
+    if n_types >= 2:
+        gt = _rng(seed, 78)
+        dev_type = gt.integers(0, n_types, size=n_dev).astype(np.uint8)
+        dur_by_type = gt.integers(1, dur_hi + 1, size=(n_ops, n_types), dtype=np.int64)
     return GmgDesc(n_dev=n_dev, pred_off=pred_off, pred_idx=pred_idx, dur=dur,
                    out_bytes=out_bytes, release=release, req_id=req_id, scored=scored,
                    deadline=dl, cap=capv, base=base, avail0=avail0, bw=bw, lat=lat,
-                   cons_off=cons_off, cons_idx=cons_idx).normalized()
+                   cons_off=cons_off, cons_idx=cons_idx, dev_type=dev_type,
+                   dur_by_type=dur_by_type).normalized()
 
 
 def random_moves(seed: int, n_cand: int, base: np.ndarray, n_dev: int, max_moves: int,

@@ -84,7 +84,7 @@ def tick_sim(desc, place, t_max=100000):
             if cands:
                 _, i = min(cands)
                 start[i] = t
-                finish[i] = t + int(desc.dur[i])
+                finish[i] = t + desc.dur_on(i, d)
                 running[d] = i
         t += 1
     return ready, start, finish
@@ -111,7 +111,7 @@ def sweep_sim(desc, place):
         last_key = (r, i)
         d = dev[i]
         start[i] = max(r, free[d])
-        finish[i] = start[i] + int(desc.dur[i])
+        finish[i] = start[i] + desc.dur_on(i, d)
         free[d] = finish[i]
         for j in succ[i]:
             left[j] -= 1

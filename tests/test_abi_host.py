@@ -86,6 +86,19 @@ def test_validation_codes():
     assert G.gmg_workspace_bytes(ok) > 0
 
 
+def test_accelerator_type_validation():
+    import dataclasses
+    base = mk([[], [0], [0, 1]], [3, 4, 5], [1, 2, 3], n_dev=2, bw=2, lat=1)
+
+    def typed(dev_type, table):
+        return dataclasses.replace(base, dev_type=np.asarray(dev_type, np.uint8),
+                                   dur_by_type=np.asarray(table, np.int64)).normalized()
+    assert G.gmg_workspace_bytes(typed([0, 1], [[1, 2], [3, 4], [5, 6]])) > 0
+    assert _create_rc(typed([0, 2], [[1, 2], [3, 4], [5, 6]])) == G.GMG_EINVAL   # type >= T
+    assert _create_rc(typed([0, 1], [[1, 2], [3, 0], [5, 6]])) == G.GMG_EINVAL   # duration < 1
+    assert _create_rc(typed([0, 1], [[1, 2], [1 << 61, 4], [5, 6]])) == G.GMG_ERANGE
+
+
 def test_product_never_imports_the_oracle():
     pkg = os.path.join(ROOT, "paper_2608_15762_gb300")
     for dirpath, _, files in os.walk(pkg):

@@ -39,6 +39,8 @@ def _run(desc, base, moves, **kw):
     (7, 1500, 16, dict(edge_p=0.8, max_pred=4, dur_hi=3000)),
     (8, 300, 8, dict(dur_hi=1 << 32)),             # times beyond 2^31: 64-bit instances
     (9, 300, 40, dict(dur_hi=1 << 31, explicit_cons=True)),
+    (10, 400, 8, dict(n_types=2)),                 # per-type durations
+    (11, 300, 33, dict(n_types=3, explicit_cons=True)),
 ])
 def test_random_incremental_bit_exact(seed, n, D, kw):
     d = W.random_desc(5000 + seed, n, D, **kw)

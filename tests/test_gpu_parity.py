@@ -46,6 +46,9 @@ def _random_case(seed, n, D, **kw):
     (15, 300, 8, dict(dur_hi=1 << 32)),               # times beyond 2^31: 64-bit instances
     (16, 200, 40, dict(dur_hi=1 << 31, explicit_cons=True)),
     (17, 150, 4, dict(dur_hi=1 << 40, link_hetero=False)),
+    (18, 300, 8, dict(n_types=2)),                    # per-type durations (Sec. 3.3.1)
+    (19, 200, 40, dict(n_types=3, explicit_cons=True)),
+    (20, 150, 4, dict(n_types=2, dur_hi=1 << 32)),
 ])
 def test_random_dags_bit_exact(seed, n, D, kw):
     d, rows = _random_case(seed, n, D, **kw)
@@ -169,6 +172,24 @@ def test_workload_prefill_all_candidates():
     assert best.cpu().tolist() == list(O.select_best(s, 0))
     assert best1.cpu().tolist() == list(O.select_best(s, 1))
     assert (s["sla_miss"] > 0).any()
+
+
+def test_workload_two_accelerator_types_all_candidates():
+    """Every placement of the prefill graph on two accelerator types."""
+    wl = W.config6()
+    rows = wl.all_full_rows()
+    g = G.gmg_create(wl.desc)
+    tk = torch.tensor([0, 4095], dtype=torch.int32, device="cuda")
+    out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk)
+    best = G.select_best(out)
+    torch.cuda.synchronize()
+    got = out.to_numpy()
+    s, pk, rq = oracle_rows(wl.desc, rows)
+    compare(got, s, pk, rq)
+    assert best.cpu().tolist() == list(O.select_best(s, 0))
+    for slot, k in enumerate([0, 4095]):
+        r = O.simulate(wl.desc, rows[k])
+        assert np.array_equal(got["trace_start"][slot], r["start"])
 
 
 def test_workload_memory_tight_all_candidates():

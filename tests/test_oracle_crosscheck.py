@@ -1,6 +1,7 @@
 """The oracle's event loop agrees with two independent formulations: a
 tick-stepped simulator and the priority-sweep restatement (each accelerator
-runs its ops in (ready, id) order, start = max(ready, queue free time))."""
+runs its ops in (ready, id) order, start = max(ready, queue free time)).
+Every fourth seed uses 2-3 accelerator types with per-type durations."""
 import numpy as np
 import pytest
 
@@ -15,7 +16,7 @@ def _rand(seed, n_hi=24, d_hi=4, dur_hi=12):
     n = int(g.integers(1, n_hi))
     D = int(g.integers(1, d_hi + 1))
     d = random_desc(seed, n, D, dur_hi=dur_hi, bytes_hi=64, explicit_cons=bool(seed % 2),
-                    link_hetero=bool(seed % 3))
+                    link_hetero=bool(seed % 3), n_types=(2 + seed % 2) if seed % 4 == 3 else 0)
     # small links so transfers matter at these time scales
     d.bw[:] = np.random.default_rng(seed).integers(4, 40, d.bw.shape[0])
     d.lat[:] = np.random.default_rng(seed + 1).integers(0, 6, d.lat.shape[0])
