@@ -299,6 +299,166 @@ def reference_arm(args):
     return 0
 
 
+# ---------------------------------------------------------------------------
+# Online estimators (include/gmgest.h): refit + durations + links per step
+# ---------------------------------------------------------------------------
+
+EST_METRIC = "estimator feedback samples incorporated/sec (refit of every estimator + durations + links)"
+
+
+def estimator_workload(seed: int = 7):
+    """Executor feedback for the operator estimators (2 accelerator types x 14
+    template operators, 5 features, 16,384 samples each) and the transfer
+    estimators (8 x 8 accelerator pairs, features (bytes, 1), 4,096 samples
+    each), and the ops whose durations are predicted (the decode workload's
+    197,632 ops on 2 types)."""
+    import numpy as np
+    g = np.random.default_rng(seed)
+    w = {}
+    T, Kk, F, cnt = 2, 14, 5, 16384
+    E = T * Kk
+    w["op_off"] = (np.arange(E + 1) * cnt).astype(np.int32)
+    x = g.uniform(0, 10, (E * cnt, F))
+    x[:, -1] = 1.0
+    beta = g.uniform(1, 40, (E, F))
+    w["op_x"] = x
+    w["op_y"] = np.einsum("sf,sf->s", x, np.repeat(beta, cnt, axis=0)) + g.normal(0, 2.0, E * cnt)
+    D, ct = 8, 4096
+    w["tr_off"] = (np.arange(D * D + 1) * ct).astype(np.int32)
+    size = g.uniform(1 << 20, 1 << 28, D * D * ct)
+    q = np.repeat(np.arange(D * D), ct)
+    inv_bw = 1.0 / g.integers(50_000, 400_000, D * D)
+    w["tr_x"] = np.stack([size, np.ones_like(size)], axis=1)
+    w["tr_y"] = size * inv_bw[q] + 10 + g.normal(0, 0.5, size.shape[0])
+    N = 197_632
+    kind = g.integers(0, Kk, N)
+    w["est_of"] = np.stack([t * Kk + kind for t in range(T)], axis=1).astype(np.int32)
+    xo = g.uniform(0, 10, (N, F))
+    xo[:, -1] = 1.0
+    w["op_feat"] = xo
+    w["dflt"] = g.integers(5, 50_000, N).astype(np.int64)
+    w["bw_dflt"] = np.full(D * D, 400_000, np.int64)
+    w["lat_dflt"] = np.full(D * D, 10, np.int64)
+    w.update(T=T, E=E, F=F, D=D, N=N)
+    return w
+
+
+def run_estimators(args):
+    import numpy as np
+    import torch
+    from paper_2608_15762_gb300 import build as lib_build
+    from paper_2608_15762_gb300 import gmgsim as G
+    lib_build.build()
+    device = torch.device("cuda", 0)
+    w = estimator_workload()
+    host = {k: torch.from_numpy(np.ascontiguousarray(v)).pin_memory() for k, v in w.items()
+            if isinstance(v, np.ndarray)}
+    dev = {k: v.to(device) for k, v in host.items()}
+    op, tr = G.Estimators(w["E"], w["F"], device), G.Estimators(w["D"] ** 2, 2, device)
+    op_tmp, tr_tmp = op.tmp_for(w["op_y"].shape[0]), tr.tmp_for(w["tr_y"].shape[0])
+    dur = torch.empty((w["N"], w["T"]), dtype=torch.int64, device=device)
+
+    bw = torch.empty(w["D"] ** 2, dtype=torch.int64, device=device)
+    lat = torch.empty_like(bw)
+    branch = torch.cuda.Stream(device)
+
+    def step():
+        # operator and transfer estimators are independent: two branches
+        main = torch.cuda.current_stream()
+        branch.wait_stream(main)
+        op.update(dev["op_off"], dev["op_x"], dev["op_y"], tmp=op_tmp)
+        op.predict_durations(dev["est_of"], dev["op_feat"], dev["dflt"], out=dur)
+        with torch.cuda.stream(branch):
+            tr.update(dev["tr_off"], dev["tr_x"], dev["tr_y"], tmp=tr_tmp)
+            G._check(G.lib().est_links(tr.state.data_ptr(), w["D"], dev["bw_dflt"].data_ptr(),
+                                       dev["lat_dflt"].data_ptr(), bw.data_ptr(), lat.data_ptr(),
+                                       G._stream_handle(branch)), "est_links")
+        main.wait_stream(branch)
+
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
+    for _ in range(args.warmup):
+        step()
+    torch.cuda.synchronize()
+
+    def timed(run):
+        ev = []
+        for _ in range(args.steps):
+            flush.fill_(1)
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record()
+            run()
+            b.record()
+            ev.append((a, b))
+        torch.cuda.synchronize()
+        return [a.elapsed_time(b) for a, b in ev]
+
+    # the step's 8 small dependent launches, captured once in a CUDA graph
+    graph = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        step()
+    torch.cuda.current_stream().wait_stream(side)
+    with torch.cuda.graph(graph):
+        step()
+    for _ in range(args.warmup):
+        graph.replay()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(0)
+    sampler.start()
+    time.sleep(0.3)
+    ms_launch = timed(step)
+    ms_all = timed(graph.replay)
+    clocks = sampler.stop()
+    ms = statistics.mean(ms_all)
+    samples = w["op_y"].shape[0] + w["tr_y"].shape[0]
+    # end to end: the feedback batch and op features copied in, durations out
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        for k in ("op_x", "op_y", "tr_x", "tr_y", "op_feat"):
+            dev[k].copy_(host[k], non_blocking=True)
+        graph.replay()
+        out = dur.cpu()
+    torch.cuda.synchronize()
+    e2e_ms = 1000 * (time.perf_counter() - t0) / args.steps
+    in_bytes = sum(host[k].numel() * host[k].element_size() for k in ("op_x", "op_y", "tr_x", "tr_y", "op_feat"))
+    alg = (in_bytes + sum(dev[k].numel() * dev[k].element_size() for k in ("op_off", "tr_off", "est_of", "dflt"))
+           + dur.numel() * 8)
+    pk = peaks()
+    line = {"metric": EST_METRIC, "value": samples / (ms / 1000), "unit": "samples/s", "n_gpus": 1,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "ms_per_step_best": min(ms_all),
+            "ms_per_step_median": statistics.median(ms_all), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": "estimators-28op-F5x16384-64link-F2x4096-predict-N197632-T2",
+                       "l2": "flushed between steps (256 MiB write)"},
+            "durations_per_s": w["N"] * w["T"] / (ms / 1000),
+            "roofline": {"bound": "hbm", "achieved": alg / (ms / 1000) / 1e9, "peak": pk["hbm_gbs"],
+                         "unit": "GB/s", "frac": alg / (ms / 1000) / 1e9 / pk["hbm_gbs"], "traffic": None,
+                         "algorithmic_bytes_per_step": alg,
+                         "note": "whole step (8 kernels, CUDA-graph replay) timed"},
+            "ms_per_step_separate_launches": statistics.mean(ms_launch),
+            "e2e": {"value": samples / (e2e_ms / 1000), "unit": "samples/s", "ms_per_step": e2e_ms,
+                    "h2d_bytes_per_step": in_bytes, "d2h_bytes_per_step": out.numel() * 8},
+            "gpu_launches": 8 * args.steps, "clocks": clocks}
+    if not args.no_cpu_baseline:
+        from oracle import estimators as OE
+        t0 = time.perf_counter()
+        o1, o2 = OE.EstimatorsOracle(w["E"], w["F"]), OE.EstimatorsOracle(w["D"] ** 2, 2)
+        o1.update(w["op_off"], w["op_x"], w["op_y"])
+        o2.update(w["tr_off"], w["tr_x"], w["tr_y"])
+        b1, f1 = o1.coefficients()
+        b2, f2 = o2.coefficients()
+        m = 20_000
+        OE.predict_durations(b1, f1, w["est_of"][:m], w["op_feat"][:m], w["dflt"][:m])
+        OE.links(b2, f2, w["D"], w["bw_dflt"], w["lat_dflt"])
+        dt = time.perf_counter() - t0
+        line["cpu_baseline"] = {"value": samples / dt, "unit": "samples/s", "cores": 1, "kind": "oracle",
+                                "sample": "one feedback batch (all %d samples), durations of the first %d of %d "
+                                          "ops" % (samples, m, w["N"])}
+    print(json.dumps(line))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -307,6 +467,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--estimators", action="store_true",
+                    help="time the online estimators (refit, durations, links) instead of the simulation")
     ap.add_argument("--candidates", type=int, default=None,
                     help="profiling aid: simulate only the first N candidates of each half "
                          "(the line then describes that smaller batch)")
@@ -315,6 +477,8 @@ def main():
         args.warmup = 3
     if args.impl == "reference":
         return reference_arm(args)
+    if args.estimators:
+        return run_estimators(args)
 
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))

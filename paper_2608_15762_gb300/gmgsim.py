@@ -25,7 +25,9 @@ SIM_OK, SIM_BADDEV, SIM_MOVE_RANGE, SIM_MOVE_DUP, SIM_BADBASE, SIM_QUEUE, SIM_LO
 EXPORTED = ("gmg_workspace_bytes", "gmg_create", "gmg_destroy", "gmg_get_info", "sim_scratch_bytes",
             "sim_batch", "sim_batch_noalloc", "base_workspace_bytes", "base_create", "base_destroy", "inc_scratch_bytes",
             "sim_incremental", "select_best_tmp_bytes", "select_best", "gmg_strerror",
-            "gmg_ceil_div_host")
+            "gmg_ceil_div_host", "est_state_bytes", "est_reset", "est_update_tmp_bytes", "est_update",
+            "est_coefficients",
+            "est_predict_durations", "est_links")
 
 
 class GmgError(RuntimeError):
@@ -90,6 +92,13 @@ def lib():
             "select_best": ([vp, i32, i32, vp, vp, sz, vp], C.c_int),
             "gmg_strerror": ([C.c_int], C.c_char_p),
             "gmg_ceil_div_host": ([i64, i64], i64),
+            "est_state_bytes": ([i32, i32], sz),
+            "est_reset": ([vp, i32, i32, vp], C.c_int),
+            "est_update_tmp_bytes": ([i32, i32, i64], sz),
+            "est_update": ([vp, i32, i32, vp, vp, vp, i64, vp, sz, vp], C.c_int),
+            "est_coefficients": ([vp, i32, i32, vp, vp, vp], C.c_int),
+            "est_predict_durations": ([vp, i32, i32, i32, i32, vp, vp, vp, vp, vp], C.c_int),
+            "est_links": ([vp, i32, vp, vp, vp, vp, vp], C.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -427,3 +436,73 @@ def moves_to_device(moves, device):
     return (torch.from_numpy(np.ascontiguousarray(moves.off, np.int32)).to(device),
             torch.from_numpy(np.ascontiguousarray(moves.op, np.int32)).to(device),
             torch.from_numpy(np.ascontiguousarray(moves.dev, np.uint8)).to(device))
+
+
+# ---------------------------------------------------------------------------
+# Online linear estimators (include/gmgest.h)
+# ---------------------------------------------------------------------------
+
+def _check(rc: int, what: str) -> None:
+    if rc != GMG_OK:
+        raise GmgError(rc, what)
+
+
+class Estimators:
+    """Device state of n_est linear estimators with n_feat features (running
+    least-squares statistics and fitted coefficients, Sec. 3.3.1)."""
+
+    def __init__(self, n_est: int, n_feat: int, device="cuda", stream=None):
+        nbytes = lib().est_state_bytes(int(n_est), int(n_feat))
+        if nbytes == 0:
+            raise GmgError(GMG_EINVAL, "est_state_bytes")
+        self.n_est, self.n_feat = int(n_est), int(n_feat)
+        self.state = _aligned_empty(nbytes, device)
+        _check(lib().est_reset(self.state.data_ptr(), self.n_est, self.n_feat, _stream_handle(stream)),
+               "est_reset")
+
+    def update(self, off, x, y, tmp=None, stream=None):
+        """Add samples (CSR by estimator: off int32 [n_est+1], x float64
+        [S, n_feat], y float64 [S], device tensors) and refit.  tmp: an
+        optional reusable buffer from tmp_for(S)."""
+        S = int(y.numel())
+        if tmp is None:
+            tmp = self.tmp_for(S)
+        _check(lib().est_update(self.state.data_ptr(), self.n_est, self.n_feat, off.data_ptr(),
+                                x.data_ptr() if S else None, y.data_ptr() if S else None, S, tmp.data_ptr(),
+                                tmp.numel(), _stream_handle(stream)), "est_update")
+
+    def tmp_for(self, n_samples: int):
+        return _aligned_empty(lib().est_update_tmp_bytes(self.n_est, self.n_feat, int(n_samples)),
+                              self.state.device)
+
+    def coefficients(self, stream=None):
+        import torch
+        beta = torch.empty((self.n_est, self.n_feat), dtype=torch.float64, device=self.state.device)
+        fitted = torch.empty(self.n_est, dtype=torch.int32, device=self.state.device)
+        _check(lib().est_coefficients(self.state.data_ptr(), self.n_est, self.n_feat, beta.data_ptr(),
+                                      fitted.data_ptr(), _stream_handle(stream)), "est_coefficients")
+        return beta, fitted
+
+    def predict_durations(self, est_of, x, dflt, out=None, stream=None):
+        """dur_by_type [n_ops, n_types] int64 from est_of int32 [n_ops, n_types],
+        op features x float64 [n_ops, n_feat] and fallback durations dflt
+        int64 [n_ops]."""
+        import torch
+        n_ops, n_types = int(est_of.shape[0]), int(est_of.shape[1])
+        if out is None:
+            out = torch.empty((n_ops, n_types), dtype=torch.int64, device=self.state.device)
+        _check(lib().est_predict_durations(self.state.data_ptr(), self.n_est, self.n_feat, n_ops, n_types,
+                                           est_of.data_ptr(), x.data_ptr(), dflt.data_ptr(), out.data_ptr(),
+                                           _stream_handle(stream)), "est_predict_durations")
+        return out
+
+    def links(self, n_dev, bw_dflt, lat_dflt, stream=None):
+        """(bw, lat) int64 [n_dev*n_dev] from the transfer estimators
+        (n_est = n_dev^2, n_feat = 2)."""
+        import torch
+        bw = torch.empty(n_dev * n_dev, dtype=torch.int64, device=self.state.device)
+        lat = torch.empty_like(bw)
+        _check(lib().est_links(self.state.data_ptr(), int(n_dev), bw_dflt.data_ptr(), lat_dflt.data_ptr(),
+                               bw.data_ptr(), lat.data_ptr(), _stream_handle(stream)), "est_links")
+        return bw, lat
+
