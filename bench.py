@@ -459,6 +459,125 @@ def run_estimators(args):
     return 0
 
 
+# ---------------------------------------------------------------------------
+# Scheduling rounds (include/gmground.h)
+# ---------------------------------------------------------------------------
+
+ROUND_METRIC = "scheduling rounds/sec (Algorithm 1: frontiers, batch, 14 partition candidates simulated, best committed)"
+
+
+def round_setup(seed: int = 12):
+    """The prefill graph (8 requests x 32 layers): one template, role = op
+    position in its request, 14 partitions (8 single accelerators, 4 pairs, 2
+    quads) with each request's layers split evenly over a partition's
+    accelerators, priority = the request's deadline, budget 128 issued ops,
+    batches of at most 64."""
+    import numpy as np
+    from paper_2608_15762_gb300 import workloads as W
+    wl = W.config2()
+    d = wl.desc
+    per = d.n_ops // 8
+    part_off = np.array([0, 1, 2, 3, 4, 5, 6, 7, 8, 10, 12, 14, 16, 20, 24], np.int32)
+    part_dev = np.array(list(range(8)) * 3, np.uint8)
+    sizes = np.diff(part_off)
+    mapping = np.stack([np.arange(per) * sizes[p] // per for p in range(len(sizes))]).astype(np.int32)
+    ld = W.placement_ld(d.n_ops)
+    place = np.zeros(ld, np.uint8)
+    place[:d.n_ops] = np.random.default_rng(seed).integers(0, 8, d.n_ops)
+    return dict(desc=d, per=per, part_off=part_off, part_dev=part_dev, mapping=mapping.reshape(-1), place=place,
+                prio=np.repeat(d.deadline, per).astype(np.int64), tmpl=np.zeros(d.n_ops, np.int32),
+                role=np.tile(np.arange(per), 8).astype(np.int32), budget=128, max_batch=64)
+
+
+def run_rounds(args):
+    import numpy as np
+    import torch
+    from paper_2608_15762_gb300 import build as lib_build
+    from paper_2608_15762_gb300 import gmgsim as G
+    lib_build.build()
+    device = torch.device("cuda", 0)
+    w = round_setup()
+    d = w["desc"]
+
+    def dev(a, dt):
+        return torch.from_numpy(np.ascontiguousarray(a, dtype=dt)).to(device)
+
+    g = G.gmg_create(d, device=device)
+    state = torch.zeros(d.n_ops, dtype=torch.uint8, device=device)
+    place = dev(w["place"], np.uint8)
+    rnd = G.Round(g, state, place, dev(w["prio"], np.int64), dev(w["tmpl"], np.int32), dev(w["role"], np.int32),
+                  dev(w["part_off"], np.int32), dev(w["part_dev"], np.uint8), dev(w["mapping"], np.int32),
+                  w["per"], w["budget"], w["max_batch"])
+
+    def one():
+        rnd.step()
+        state.masked_fill_(state == 1, 2)   # the executor finishes the issued ops
+
+    def reset():
+        state.zero_()
+        place.copy_(dev(w["place"], np.uint8))
+
+    # the rounds from an empty schedule until every op is scheduled (counted
+    # once with the status read back, then replayed without host reads)
+    needed = 0
+    while True:
+        one()
+        needed += 1
+        if int(rnd.info[5].item()) != G.ROUND_BATCH or needed > 100000:
+            break
+    needed -= 1
+    for _ in range(args.warmup):
+        reset()
+        for _ in range(needed):
+            one()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(0)
+    sampler.start()
+    time.sleep(0.3)
+    ev = []
+    for _ in range(max(args.steps, 1)):
+        reset()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        for _ in range(needed):
+            one()
+        b.record()
+        ev.append((a, b))
+    torch.cuda.synchronize()
+    ms_all = [a.elapsed_time(b) / needed for a, b in ev]
+    clocks = sampler.stop()
+    ms = statistics.mean(ms_all)
+    rounds = needed * max(args.steps, 1)
+    scheduled = int((state != 0).sum().item())
+    line = {"metric": ROUND_METRIC, "value": 1000.0 / ms, "unit": "rounds/s", "n_gpus": 1, "steps": rounds,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "int64", "data": "synthetic",
+            "config": {"workload": "rounds-prefill-8x32L-N3088-D8-P14-B128-batch64",
+                       "rounds_to_schedule_every_op": needed, "ops_scheduled": scheduled},
+            "ms_per_step_best": min(ms_all), "ms_per_step_median": statistics.median(ms_all),
+            "candidates_per_s": 14 * 1000.0 / ms,
+            "roofline": {"bound": "alu", "achieved": None, "peak": None, "unit": "Ginst/s", "frac": None,
+                         "traffic": None,
+                         "note": "latency-bound: 14 candidates are 14 warps; a round takes one candidate "
+                                 "simulation's latency plus 8 small launches"},
+            "gpu_launches": 9 * rounds, "clocks": clocks}
+    if not args.no_cpu_baseline:
+        from oracle import round as OR
+        st = np.zeros(d.n_ops, np.uint8)
+        pl = w["place"].copy()
+        t0 = time.perf_counter()
+        k = min(needed, 16)
+        for _ in range(k):
+            _, _, _, _, st, pl = OR.round_step(d, st, pl, w["prio"], w["tmpl"], w["role"], w["part_off"],
+                                               w["part_dev"], w["mapping"], w["per"], w["budget"], w["max_batch"])
+            st[st == 1] = 2
+        dt = (time.perf_counter() - t0) / k
+        line["cpu_baseline"] = {"value": 1.0 / dt, "unit": "rounds/s", "cores": 1, "kind": "oracle",
+                                "sample": "the first %d rounds (Python frontiers/batch, C++ simulations)" % k}
+    print(json.dumps(line))
+    return 0
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -467,6 +586,8 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--rounds", action="store_true",
+                    help="time scheduling rounds (Algorithm 1) instead of the candidate simulation")
     ap.add_argument("--estimators", action="store_true",
                     help="time the online estimators (refit, durations, links) instead of the simulation")
     ap.add_argument("--candidates", type=int, default=None,
@@ -479,6 +600,8 @@ def main():
         return reference_arm(args)
     if args.estimators:
         return run_estimators(args)
+    if args.rounds:
+        return run_rounds(args)
 
     import torch
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -10,7 +10,7 @@
 #include <new>
 #include <vector>
 
-#include "gmg_layout.h"
+#include "gmg_access.h"
 
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
@@ -395,6 +395,8 @@ struct gmg {
   int64_t queue_bound;
   int64_t log_bound;
 };
+
+const DevGmg* gsim::gmg_device_graph(const gmg_t* g) { return g ? &g->dg : nullptr; }
 
 struct gmg_base {
   DevBase db;

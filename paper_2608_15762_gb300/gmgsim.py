@@ -27,7 +27,8 @@ EXPORTED = ("gmg_workspace_bytes", "gmg_create", "gmg_destroy", "gmg_get_info", 
             "sim_incremental", "select_best_tmp_bytes", "select_best", "gmg_strerror",
             "gmg_ceil_div_host", "est_state_bytes", "est_reset", "est_update_tmp_bytes", "est_update",
             "est_coefficients",
-            "est_predict_durations", "est_links")
+            "est_predict_durations", "est_links", "round_scratch_bytes", "round_select", "round_candidates",
+            "round_commit")
 
 
 class GmgError(RuntimeError):
@@ -99,6 +100,10 @@ def lib():
             "est_coefficients": ([vp, i32, i32, vp, vp, vp], C.c_int),
             "est_predict_durations": ([vp, i32, i32, i32, i32, vp, vp, vp, vp, vp], C.c_int),
             "est_links": ([vp, i32, vp, vp, vp, vp, vp], C.c_int),
+            "round_scratch_bytes": ([vp], sz),
+            "round_select": ([vp, vp, vp, i32, i32, C.c_uint32, vp, sz, vp, vp, vp], C.c_int),
+            "round_candidates": ([vp, vp, i32, vp, i32, vp, i32, vp, vp, vp, vp, vp, i32, vp, vp], C.c_int),
+            "round_commit": ([vp, i32, vp, vp, vp, i32, vp, vp, vp], C.c_int),
         }
         for name, (args, res) in sig.items():
             f = getattr(L, name)
@@ -505,4 +510,54 @@ class Estimators:
         _check(lib().est_links(self.state.data_ptr(), int(n_dev), bw_dflt.data_ptr(), lat_dflt.data_ptr(),
                                bw.data_ptr(), lat.data_ptr(), _stream_handle(stream)), "est_links")
         return bw, lat
+
+
+# ---------------------------------------------------------------------------
+# A scheduling round of Algorithm 1 (include/gmground.h)
+# ---------------------------------------------------------------------------
+
+ROUND_BATCH, ROUND_BUDGET, ROUND_EMPTY, ROUND_NO_FEASIBLE = 0, 1, 2, 3
+
+
+class Round:
+    """Device state of the rounds on one GMG: op states, placement row,
+    priorities, templates / roles, partitions and the fixed per-template
+    mappings.  step() runs one round entirely on the device: round_select,
+    round_candidates, sim_batch over the partition rows, select_best,
+    round_commit; the caller reads `info` when it needs to."""
+
+    def __init__(self, g: Gmg, state, place, prio, tmpl, role, part_off, part_dev, mapping, n_roles: int,
+                 budget: int, max_batch: int, score_mode: int = 0):
+        import torch
+        self.g, self.state, self.place, self.prio = g, state, place, prio
+        self.tmpl, self.role, self.part_off, self.part_dev, self.map = tmpl, role, part_off, part_dev, mapping
+        self.n_roles, self.budget, self.max_batch, self.score_mode = int(n_roles), int(budget), int(max_batch), score_mode
+        self.n_part = int(part_off.numel() - 1)
+        dev = place.device
+        self.ld = int(place.numel())
+        self.scratch = _aligned_empty(lib().round_scratch_bytes(g.handle), dev)
+        self.scratch.zero_()
+        self.epoch = 0
+        self.batch = torch.empty(self.max_batch, dtype=torch.int32, device=dev)
+        self.info = torch.zeros(8, dtype=torch.int64, device=dev)
+        self.rows = _aligned_empty(self.n_part * self.ld, dev, 16).view(self.n_part, self.ld)
+        self.out = SimOut.empty(self.n_part, g.desc.n_dev, g.desc.n_req, dev)
+        self.sim_scratch = Scratch(dev)
+        self.best = torch.empty(2, dtype=torch.int64, device=dev)
+
+    def step(self, stream=None):
+        h = _stream_handle(stream)
+        self.epoch += 1
+        _check(lib().round_select(self.g.handle, self.state.data_ptr(), self.prio.data_ptr(), self.budget,
+                                  self.max_batch, self.epoch, self.scratch.data_ptr(), self.scratch.numel(),
+                                  self.batch.data_ptr(), self.info.data_ptr(), h), "round_select")
+        _check(lib().round_candidates(self.g.handle, self.place.data_ptr(), self.ld, self.batch.data_ptr(),
+                                      self.max_batch, self.info.data_ptr(), self.n_part, self.part_off.data_ptr(),
+                                      self.part_dev.data_ptr(), self.tmpl.data_ptr(), self.role.data_ptr(),
+                                      self.map.data_ptr(), self.n_roles, self.rows.data_ptr(), h), "round_candidates")
+        sim_batch(self.g, self.rows, out=self.out, scratch=self.sim_scratch, stream=stream)
+        select_best(self.out, self.n_part, score_mode=self.score_mode, best=self.best, stream=stream)
+        _check(lib().round_commit(self.batch.data_ptr(), self.max_batch, self.info.data_ptr(), self.best.data_ptr(),
+                                  self.rows.data_ptr(), self.ld, self.place.data_ptr(), self.state.data_ptr(), h),
+               "round_commit")
 

@@ -22,7 +22,7 @@ def test_exports_every_declared_symbol():
     hdr = "".join(open(os.path.join(ROOT, "include", f)).read()
                   for f in sorted(os.listdir(os.path.join(ROOT, "include"))) if f.endswith(".h"))
     names = set(re.findall(r"^\s*(?:[\w\*\s]+?)\b(\w+)\s*\(", hdr, re.M)) - {"if", "sizeof"}
-    decl = {n for n in names if n.startswith(("gmg_", "sim_", "base_", "inc_", "select_", "est_"))}
+    decl = {n for n in names if n.startswith(("gmg_", "sim_", "base_", "inc_", "select_", "est_", "round_"))}
     assert decl == set(G.EXPORTED), decl ^ set(G.EXPORTED)
     L = G.lib()
     for n in decl:
