@@ -259,6 +259,16 @@ struct Devices {
     if (kReg) fr_reg = l < (unsigned)D ? (TM)src[l] : (TM)0;
     __syncwarp();
   }
+  // Largest final free time over the accelerators whose free time moved past
+  // their initial availability (0 if none).  Uniform result.
+  __device__ int64_t max_busy(const DevGmg& g) const {
+    uint64_t m = 0;
+    for (int d = lane_id(); d < D; d += 32) {
+      const int64_t f = kReg ? (int64_t)fr_reg : fr[d];
+      if (f > g.avail0[d]) m = (uint64_t)f > m ? (uint64_t)f : m;
+    }
+    return (int64_t)warp_max_u64(m);
+  }
   __device__ void write_peak(int64_t* dst) const {
     for (int d = lane_id(); d < D; d += 32) dst[d] = pk[d];
   }
@@ -331,8 +341,9 @@ struct Sim {
   // running results
   int rootptr;
   uint64_t rkey;    // root_keys[rootptr], kKeyMax past the end
-  int64_t score, iters, nev, readypops;
-  tm_t makespan, last_t;
+  int64_t score, nev, readypops;
+  int32_t iters;        // ops started (loop guard; the event count of a full run)
+  tm_t makespan, last_t;  // running values, kept in base mode only (checkpoints)
   int32_t vflag, vop, vdev, status;
   int64_t vt;
   // base checkpoints
@@ -483,8 +494,8 @@ struct Sim {
     }
     ++opn;
     if (flags & kScored) score += (int64_t)f;
-    makespan = f > makespan ? f : makespan;
-    if (kMode != kInc || r >= T0) ++nev;
+    if (kMode == kBase) makespan = f > makespan ? f : makespan;
+    if (kMode == kInc && r >= T0) ++nev;
     if (kMode == kBase) ++readypops;
     __syncwarp();
 
@@ -942,12 +953,12 @@ struct Sim {
         __syncwarp();
         q.pop();
       }
-      if (++iters > g.max_iter) {
+      if (++iters > (int32_t)g.max_iter) {
         status = GMG_SIM_LOOP;
         break;
       }
       const tm_t t = (tm_t)kc.time(nk);
-      last_t = t;
+      if (kMode == kBase) last_t = t;
       start_op(kc.op(nk), t);
       if (status) break;
     }
@@ -1002,8 +1013,12 @@ struct Sim {
     }
     miss = (int32_t)__reduce_add_sync(kFullMask, (unsigned)miss);
     dv.write_peak(o.peak + k * g.D);
+    // The makespan is the latest finish, i.e. the largest final free time over
+    // the accelerators that ran an op (an op finishes after its accelerator's
+    // initial availability).
+    const int64_t mk = dv.max_busy(g);
     if (lane == 0) {
-      o.makespan[k] = makespan;
+      o.makespan[k] = mk;
       o.score[k] = vflag ? kI64Max : score;
       o.status[k] = GMG_SIM_OK;
       o.viol_flag[k] = vflag;
@@ -1011,7 +1026,7 @@ struct Sim {
       o.viol_dev[k] = vdev;
       o.viol_time[k] = vt;
       o.sla_miss[k] = miss;
-      o.events[k] = nev;
+      o.events[k] = kMode == kFull ? (int64_t)iters : nev;
     }
     const int ts = trace_slot(k);
     if (ts >= 0)
