@@ -141,11 +141,9 @@ struct DevBase {
   uint64_t* ck_qkey;     // [nck*ckq] READY heap
   uint64_t* ck_mkey;     // [nck*ckm] HBM event log entries
   uint8_t* ck_mdev;      // [nck*ckm] their accelerators (when not inside the entries)
-  uint32_t* ck_bits;     // [nck*ck_words] simulated-op bitmap
   int32_t nck;
   int32_t ckq;           // READY entries per checkpoint
   int32_t ckm;           // HBM events per checkpoint
-  int32_t ck_words;      // bitmap words per checkpoint
   int32_t ld;
   int32_t stride_pops;   // READY pops between checkpoints
 };

@@ -527,8 +527,8 @@ void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
 
 struct BasePlan {
   size_t off_row, off_rb, off_fb, off_status, off_res, off_peak, off_creq, off_cktime,
-      off_cksc, off_ckdev, off_ckcreq, off_ckqk, off_ckmk, off_ckmd, off_ckbits, off_slot, total;
-  int nck, ckq, ckm, ckw, ld, stride;
+      off_cksc, off_ckdev, off_ckcreq, off_ckqk, off_ckmk, off_ckmd, off_slot, total;
+  int nck, ckq, ckm, ld, stride;
   Launch L;
 };
 
@@ -542,7 +542,6 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   B.nck = kCheckpoints;
   B.ckq = std::min(L.P.qcap, kCheckpointQueue);
   B.ckm = std::min(L.P.mcap, kCheckpointLog);
-  B.ckw = (G.n + 31) / 32;
   B.ld = (int)align_up(std::max(G.n, 1), 16);
   B.stride = std::max(1, G.n / (B.nck - 1));
   size_t off = 0;
@@ -565,7 +564,6 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   B.off_ckqk = take(8 * (size_t)B.ckq * B.nck);
   B.off_ckmk = take(8 * (size_t)B.ckm * B.nck);
   B.off_ckmd = take((size_t)B.ckm * B.nck);
-  B.off_ckbits = take(4 * (size_t)B.ckw * B.nck);
   B.off_slot = take((size_t)L.P.slot_bytes);
   B.total = off;
   return GMG_OK;
@@ -822,11 +820,9 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   D.ck_qkey = reinterpret_cast<uint64_t*>(w + B.off_ckqk);
   D.ck_mkey = reinterpret_cast<uint64_t*>(w + B.off_ckmk);
   D.ck_mdev = w + B.off_ckmd;
-  D.ck_bits = reinterpret_cast<uint32_t*>(w + B.off_ckbits);
   D.nck = B.nck;
   D.ckq = B.ckq;
   D.ckm = B.ckm;
-  D.ck_words = B.ckw;
   D.ld = B.ld;
   D.stride_pops = B.stride;
   b->g = g;

@@ -131,7 +131,9 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimP
   S.opn = 0;
   S.dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
   for (int r = lane; r < g.R; r += 32) S.creq[r] = B.ck_creq[(int64_t)c * g.R + r];
-  for (int w = lane; w < words; w += 32) S.bits[w] = B.ck_bits[(int64_t)c * B.ck_words + w];
+  // ops started before T_c are those with base ready time < T_c (fin()
+  // reads their base finish); the others start with no finish time
+  S.zero_fin();
   // READY keys at T_c; a moved op's key is recomputed (its inputs' transfer
   // times change; its predecessors all finished before T_c).
   for (int x = lane; x < qsz; x += 32) {
@@ -279,11 +281,11 @@ __device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
       for (uint32_t u = 0; u < nl; ++u) {
         const uint32_t c = __ldg(lst + u);
         if (S.row[c] != du) continue;
-        if (!S.popped(c)) {
+        const int64_t fc = S.fin(c);
+        if (fc == 0) {  // not started yet
           rel = false;
           break;
         }
-        const int64_t fc = S.fin(c);
         tr = fc > tr ? fc : tr;
       }
     }
@@ -297,11 +299,9 @@ __device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
     if (t < nl) {
       const uint32_t c = __ldg(lst + t);
       if (S.row[c] == dp) {
-        if (!S.popped(c)) pending = true;
-        else {
-          const uint64_t fc = (uint64_t)S.fin(c);
-          mx = fc > mx ? fc : mx;
-        }
+        const uint64_t fc = (uint64_t)S.fin(c);
+        if (fc == 0) pending = true;
+        else mx = fc > mx ? fc : mx;
       }
     }
   }

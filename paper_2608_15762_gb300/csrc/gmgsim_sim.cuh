@@ -356,7 +356,9 @@ struct Sim {
     lowmask = kKey ? (1ull << ds) - 1ull : kKeyMax;
   }
 
-  __device__ __forceinline__ bool popped(uint32_t x) const { return (bits[x >> 5] >> (x & 31u)) & 1u; }
+  // Started ops are those with a finish time (every finish time is >= 1;
+  // the finish array is zeroed per candidate).
+  __device__ __forceinline__ bool popped(uint32_t x) const { return fin(x) != 0; }
   // Finish time of a simulated op (incremental: ops before the resume point
   // keep their base finish).
   // The low 32 bits of a base-snapshot time (little-endian int64).
@@ -443,10 +445,17 @@ struct Sim {
     log.n += cnt;
   }
 
+  // Zero this candidate's finish times (16-byte stores; the array is padded).
+  __device__ void zero_fin() {
+    uint4* v = reinterpret_cast<uint4*>(fbuf);
+    const int nv = (int)((sizeof(tm_t) * (size_t)g.n + 15) / 16);
+    for (int x = lane_id(); x < nv; x += 32) v[x] = make_uint4(0u, 0u, 0u, 0u);
+    __syncwarp();
+  }
+
   __device__ void reset_common() {
     const unsigned lane = lane_id();
-    const int words = (g.n + 31) >> 5;
-    for (int w = lane; w < words; w += 32) bits[w] = 0u;
+    zero_fin();
     for (int r = lane; r < g.R; r += 32) creq[r] = 0;
     dv.reset(g);
     q.size = 0;
@@ -486,7 +495,6 @@ struct Sim {
     dv.set_free(d, f);
     if (lane == 0) {
       fbuf[i] = f;
-      atomicOr(&bits[i >> 5], 1u << (i & 31u));
       if (flags & kReqSink)
         atomicMax(reinterpret_cast<unsigned long long*>(creq + (int32_t)cs.z), (unsigned long long)f);
       if (kMode == kBase) P.base.rb[i] = r;
@@ -520,12 +528,12 @@ struct Sim {
           for (uint32_t k = 0; k < jls.w; ++k) {
             const uint32_t p = __ldg(g.pred + jls.z + k) & kIdMask;
             if (p == i) continue;
-            if (!popped(p)) {
+            tm_t a = fin(p);
+            if (a == 0) {  // not started yet
               rdy = false;
               break;
             }
             const int dp = row[p];
-            tm_t a = fin(p);
             if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
             rj = a > rj ? a : rj;
           }
@@ -639,7 +647,8 @@ struct Sim {
             } else if (sb != kSibMany && (sb & kSibLater)) {
               rel = row[sb & ~kSibLater] != d;  // the other consumer finishes later
             } else if (sb != kSibMany) {
-              rel = !(row[sb] == d && !(popped(sb) && fin(sb) < f));
+              const tm_t fs = fin(sb);
+              rel = !(row[sb] == d && !(fs != 0 && fs < f));
             } else {
               const uint4 pls = op_lists(g.ops, p);
               const uint4 pcs = op_cons(g.ops, p);
@@ -649,7 +658,8 @@ struct Sim {
               rel = true;
               for (uint32_t w = 0; w < nl; ++w) {
                 const uint32_t c = __ldg(lst + w);
-                if (c != x && row[c] == d && !(popped(c) && fin(c) < f)) {
+                const tm_t fc = c != x ? fin(c) : 0;
+                if (c != x && row[c] == d && !(fc != 0 && fc < f)) {
                   rel = false;
                   break;
                 }
@@ -1098,8 +1108,6 @@ __device__ void Sim<kReg, kMode, kKey, kT32, kTypes>::maybe_checkpoint(uint64_t 
       B.ck_mkey[(int64_t)ck * B.ckm + x] = *log.kp(x);
       B.ck_mdev[(int64_t)ck * B.ckm + x] = *log.dp(x);
     }
-    const int words = (g.n + 31) >> 5;
-    for (int w = lane; w < words; w += 32) B.ck_bits[(int64_t)ck * B.ck_words + w] = bits[w];
   } else if (lane == 0) {
     B.ck_time[ck] = kI64Max;
   }
