@@ -9,17 +9,18 @@
 
 namespace gsim {
 
-// One 64-byte record per operator: everything the event loop reads when it
-// pops, releases or readies the op, in one L1 sector pair.
+// One 64-byte record per operator, in four 16-byte pieces grouped by use:
+// [dur, bytes] | [release, predecessor list] (readiness checks) | [xq,
+// successor list] (starting the op) | [consumer list, request, flags].
 struct alignas(64) OpRec {
   int64_t dur;       // duration (us), >= 1
   int64_t bytes;     // output size (B)
   int64_t release;   // arrival of the op itself (us)
+  uint32_t pred_off; // predecessors: pred[pred_off .. +npred); bit 31 set if this op
+  uint32_t npred;    //   is a listed consumer of that predecessor's output
   int64_t xq;        // ceil(bytes / bw) when every link has the same bandwidth
   uint32_t succ_off; // successors: succ[succ_off .. +nsucc), ascending
   uint32_t nsucc;
-  uint32_t pred_off; // predecessors: pred[pred_off .. +npred); bit 31 set if this op
-  uint32_t npred;    //   is a listed consumer of that predecessor's output
   uint32_t cons_off; // listed consumers of this op's output: cons[cons_off .. +ncons)
   uint32_t ncons;    //   (equals the successor list when kAllCons is set)
   int32_t req;       // request id or -1

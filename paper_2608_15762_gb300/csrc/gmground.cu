@@ -50,8 +50,12 @@ Layout layout(int32_t n) {
   return L;
 }
 
+// (succ_off, nsucc, pred_off, npred) from the op record's [release, preds]
+// and [xq, succs] pieces.
 __device__ __forceinline__ uint4 op_lists(const DevGmg& g, uint32_t i) {
-  return __ldg(reinterpret_cast<const uint4*>(g.ops + i) + 2);  // succ_off, nsucc, pred_off, npred
+  const uint4 rp = __ldg(reinterpret_cast<const uint4*>(g.ops + i) + 1);
+  const uint4 xs = __ldg(reinterpret_cast<const uint4*>(g.ops + i) + 2);
+  return make_uint4(xs.z, xs.w, rp.z, rp.w);
 }
 
 __device__ __forceinline__ bool key_less(int64_t pa, int64_t ia, int64_t pb, int64_t ib) {

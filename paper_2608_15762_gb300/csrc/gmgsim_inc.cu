@@ -55,10 +55,11 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimP
     const uint8_t dvc = P.move_dev[m0 + t];
     crow[op] = dvc;
     if (dvc != B.row[op]) {
-      const uint4 ls = op_lists(g.ops, (uint32_t)op);
+      const RelPred rp = op_relpred(g.ops, (uint32_t)op);
+      const uint4 ls = make_uint4(0u, 0u, rp.pred_off, rp.npred);
       uint64_t tx;
       if (ls.w == 0) {
-        tx = (uint64_t)op_relxq(g.ops, (uint32_t)op).x;
+        tx = (uint64_t)rp.rel;
       } else {
         tx = kKeyMax;
         for (uint32_t u = 0; u < ls.w; ++u) {
@@ -141,13 +142,14 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimP
     const uint32_t op = S.kc.op(key);
     if (crow[op] != B.row[op]) {
       const int dx = crow[op];
-      const uint4 ls = op_lists(g.ops, op);
-      int64_t rx = op_relxq(g.ops, op).x;
+      const RelPred rp = op_relpred(g.ops, op);
+      const uint4 ls = make_uint4(0u, 0u, rp.pred_off, rp.npred);
+      int64_t rx = rp.rel;
       for (uint32_t u = 0; u < ls.w; ++u) {
         const uint32_t p = __ldg(g.pred + ls.z + u) & kIdMask;
         const int dp = crow[p];
         int64_t a = S.fb[p];
-        if (dp != dx) a += S.xfer(dp, dx, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
+        if (dp != dx) a += S.xfer(dp, dx, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
         rx = a > rx ? a : rx;
       }
       key = S.kc.make(rx, kReady, op);
@@ -246,7 +248,7 @@ __device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
   const unsigned lane = lane_id();
   const int64_t fp = S.fb[p];
   const int dp = S.row[p];
-  const int64_t pb = op_durbytes(g.ops, p).y, pxq = op_relxq(g.ops, p).y;
+  const int64_t pb = op_durbytes(g.ops, p).y, pxq = op_xqsucc(g.ops, p).xq;
   const uint4 pls = op_lists(g.ops, p);
   const uint4 pcs = op_cons(g.ops, p);
   const bool all = (pcs.w & kAllCons) != 0;

@@ -77,11 +77,27 @@ __device__ __forceinline__ uint32_t lanes_below() { return (1u << lane_id()) - 1
 __device__ __forceinline__ longlong2 op_durbytes(const OpRec* ops, uint32_t i) {
   return __ldg(reinterpret_cast<const longlong2*>(ops + i));
 }
-__device__ __forceinline__ longlong2 op_relxq(const OpRec* ops, uint32_t i) {
-  return __ldg(reinterpret_cast<const longlong2*>(ops + i) + 1);
+struct RelPred {
+  int64_t rel;
+  uint32_t pred_off, npred;
+};
+struct XqSucc {
+  int64_t xq;
+  uint32_t succ_off, nsucc;
+};
+__device__ __forceinline__ RelPred op_relpred(const OpRec* ops, uint32_t i) {
+  const uint4 v = __ldg(reinterpret_cast<const uint4*>(ops + i) + 1);
+  return RelPred{(int64_t)(((uint64_t)v.y << 32) | v.x), v.z, v.w};
 }
+__device__ __forceinline__ XqSucc op_xqsucc(const OpRec* ops, uint32_t i) {
+  const uint4 v = __ldg(reinterpret_cast<const uint4*>(ops + i) + 2);
+  return XqSucc{(int64_t)(((uint64_t)v.y << 32) | v.x), v.z, v.w};
+}
+// (succ_off, nsucc, pred_off, npred) from two pieces, for code that needs both lists.
 __device__ __forceinline__ uint4 op_lists(const OpRec* ops, uint32_t i) {
-  return __ldg(reinterpret_cast<const uint4*>(ops + i) + 2);  // succ_off, nsucc, pred_off, npred
+  const XqSucc a = op_xqsucc(ops, i);
+  const RelPred b = op_relpred(ops, i);
+  return make_uint4(a.succ_off, a.nsucc, b.pred_off, b.npred);
 }
 __device__ __forceinline__ uint4 op_cons(const OpRec* ops, uint32_t i) {
   return __ldg(reinterpret_cast<const uint4*>(ops + i) + 3);  // cons_off, ncons, req, flags
@@ -395,11 +411,11 @@ struct Sim {
   // earliest its source copy may be released.  Per lane.
   __device__ tm_t lane_hold(uint32_t p, tm_t fp, int dp) const {
     const int64_t pb = op_durbytes(g.ops, p).y;
-    const int64_t pxq = op_relxq(g.ops, p).y;
-    const uint4 ls = op_lists(g.ops, p);
+    const XqSucc ps = op_xqsucc(g.ops, p);
+    const int64_t pxq = ps.xq;
     tm_t h = fp;
-    for (uint32_t u = 0; u < ls.y; ++u) {
-      const int du = row[__ldg(g.succ + ls.x + u)];
+    for (uint32_t u = 0; u < ps.nsucc; ++u) {
+      const int du = row[__ldg(g.succ + ps.succ_off + u)];
       if (du != dp) {
         const tm_t a = fp + xfer(dp, du, pb, pxq);
         h = a > h ? a : h;
@@ -481,11 +497,10 @@ struct Sim {
   __device__ void start_op(uint32_t i, tm_t r) {
     const unsigned lane = lane_id();
     const longlong2 db = op_durbytes(g.ops, i);
-    const longlong2 rx = op_relxq(g.ops, i);
-    const uint4 ls = op_lists(g.ops, i);
+    const XqSucc xs = op_xqsucc(g.ops, i);
     const uint4 cs = op_cons(g.ops, i);
-    const int64_t bytes = db.y, xq = rx.y;
-    const uint32_t succ_off = ls.x, nsucc = ls.y;
+    const int64_t bytes = db.y, xq = xs.xq;
+    const uint32_t succ_off = xs.succ_off, nsucc = xs.nsucc;
     const uint32_t flags = cs.w;
     const int d = row[i];
     const tm_t dur = (tm_t)dur_of(i, d, db.x);
@@ -519,14 +534,13 @@ struct Sim {
         const int dj = row[j];
         tm_t arr = f;
         if (dj != d) arr = f + xfer(d, dj, bytes, xq);
-        const longlong2 jrx = op_relxq(g.ops, j);
-        const uint4 jls = op_lists(g.ops, j);
-        const tm_t rel = (tm_t)jrx.x;
+        const RelPred jp = op_relpred(g.ops, j);
+        const tm_t rel = (tm_t)jp.rel;
         rj = rel > arr ? rel : arr;
         rdy = true;
-        if (jls.w > 1) {
-          for (uint32_t k = 0; k < jls.w; ++k) {
-            const uint32_t p = __ldg(g.pred + jls.z + k) & kIdMask;
+        if (jp.npred > 1) {
+          for (uint32_t k = 0; k < jp.npred; ++k) {
+            const uint32_t p = __ldg(g.pred + jp.pred_off + k) & kIdMask;
             if (p == i) continue;
             tm_t a = fin(p);
             if (a == 0) {  // not started yet
@@ -534,7 +548,7 @@ struct Sim {
               break;
             }
             const int dp = row[p];
-            if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_relxq(g.ops, p).y);
+            if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
             rj = a > rj ? a : rj;
           }
         }
@@ -572,8 +586,10 @@ struct Sim {
       tm_t f = 0;
       if (v) {
         db = op_durbytes(g.ops, x);
-        rx = op_relxq(g.ops, x);
-        ls = op_lists(g.ops, x);
+        const XqSucc xs = op_xqsucc(g.ops, x);
+        const RelPred rp = op_relpred(g.ops, x);
+        rx = make_longlong2(rp.rel, xs.xq);
+        ls = make_uint4(xs.succ_off, xs.nsucc, rp.pred_off, rp.npred);
         cs = op_cons(g.ops, x);
         d = row[x];
         f = fbuf[x];
@@ -650,7 +666,8 @@ struct Sim {
               const tm_t fs = fin(sb);
               rel = !(row[sb] == d && !(fs != 0 && fs < f));
             } else {
-              const uint4 pls = op_lists(g.ops, p);
+              const XqSucc px = op_xqsucc(g.ops, p);
+              const uint4 pls = make_uint4(px.succ_off, px.nsucc, 0u, 0u);
               const uint4 pcs = op_cons(g.ops, p);
               const bool all = (pcs.w & kAllCons) != 0;
               const uint32_t* lst = all ? g.succ + pls.x : g.cons + pcs.x;
