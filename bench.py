@@ -39,11 +39,35 @@ KERNEL_SOURCES = [os.path.join(ROOT, "paper_2608_15762_gb300", "csrc", f)
                             "gmg_layout.h")]
 
 
+def _code_only(text: str) -> str:
+    """The source without comments or blank lines: a profile stays valid
+    across comment edits, which cannot change the compiled kernel."""
+    import re
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    lines = []
+    for ln in text.splitlines():
+        # drop // comments that are not inside string literals
+        out, in_str = [], False
+        i = 0
+        while i < len(ln):
+            c = ln[i]
+            if c == '"' and (i == 0 or ln[i - 1] != "\\"):
+                in_str = not in_str
+            if not in_str and ln.startswith("//", i):
+                break
+            out.append(c)
+            i += 1
+        s = "".join(out).rstrip()
+        if s:
+            lines.append(s)
+    return "\n".join(lines)
+
+
 def kernel_hash() -> str:
     h = hashlib.sha256()
     for f in KERNEL_SOURCES:
-        with open(f, "rb") as fh:
-            h.update(fh.read())
+        with open(f, encoding="utf-8") as fh:
+            h.update(_code_only(fh.read()).encode())
     return h.hexdigest()[:16]
 
 

@@ -1088,10 +1088,11 @@ struct Sim {
   }
 };
 
-// Base-mode checkpoint: at a time boundary (nothing at the next key's time
-// handled yet), save the complete simulator state -- simulated-op bitmap,
-// accelerator state, READY heap, event log, partial results.  An
-// incremental candidate whose resume time T0 is >= that time restarts there.
+// Base-mode checkpoint: at a time boundary T_c (nothing at the next key's
+// time handled yet), save the complete simulator state -- accelerator state,
+// READY heap, event log, partial results; the ops started by then are those
+// with base ready time < T_c.  An incremental candidate whose resume time T0
+// is >= T_c restarts there.
 template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes>
 __device__ void Sim<kReg, kMode, kKey, kT32, kTypes>::maybe_checkpoint(uint64_t next_key) {
   if (kMode != kBase) return;
