@@ -165,3 +165,23 @@ def test_fitted_durations_drive_the_simulation():
     torch.cuda.synchronize()
     s, pk, rq = oracle_rows(dataclasses.replace(base, dur_by_type=od).normalized(), rows)
     compare(out.to_numpy(), s, pk, rq)
+
+
+def test_empty_batches_one_type_and_one_accelerator():
+    est, orc = G.Estimators(3, 2), OE.EstimatorsOracle(3, 2)
+    off = np.zeros(4, np.int32)
+    est.update(_dev(off, np.int32), torch.zeros((0, 2), dtype=torch.float64, device="cuda"),
+               torch.zeros(0, dtype=torch.float64, device="cuda"))
+    beta, fitted = est.coefficients()
+    assert fitted.cpu().tolist() == [0, 0, 0] and not beta.cpu().numpy().any()
+    g = np.random.default_rng(12)
+    o2, x, y = _batch(g, [40, 0, 9], 2, g.uniform(1, 9, (3, 2)))
+    est.update(_dev(o2, np.int32), _dev(x, np.float64), _dev(y, np.float64))
+    orc.update(o2, x, y)
+    est_of = np.array([[0], [1], [2], [-1]], np.int32)         # one accelerator type
+    xo = np.stack([g.uniform(0, 10, 4), np.ones(4)], axis=1)
+    d, od, _, _ = _predict_both(est, orc, est_of, xo, np.array([5, 6, 7, 8]))
+    assert np.array_equal(d, od) and d[1, 0] == 6 and d[3, 0] == 8
+    tr = G.Estimators(1, 2)                                     # one accelerator: only the diagonal
+    bw, lat = tr.links(1, _dev(np.array([9]), np.int64), _dev(np.array([4]), np.int64))
+    assert bw.cpu().tolist() == [9] and lat.cpu().tolist() == [4]

@@ -49,6 +49,7 @@ def _random_case(seed, n, D, **kw):
     (18, 300, 8, dict(n_types=2)),                    # per-type durations (Sec. 3.3.1)
     (19, 200, 40, dict(n_types=3, explicit_cons=True)),
     (20, 150, 4, dict(n_types=2, dur_hi=1 << 32)),
+    (21, 300, 256, dict(n_types=4, explicit_cons=True)),   # typed, accelerator state in shared memory
 ])
 def test_random_dags_bit_exact(seed, n, D, kw):
     d, rows = _random_case(seed, n, D, **kw)

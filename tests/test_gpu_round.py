@@ -136,3 +136,45 @@ def test_prefill_requests_with_layer_partitions():
         assert np.array_equal(st_d.cpu().numpy(), state) and np.array_equal(pl_d.cpu().numpy(), place)
         state[state == 1] = 2
         st_d.copy_(_dev(state, np.uint8))
+
+
+def _one_round(desc, state, place, budget, max_batch, part_off, part_dev, mapping, n_roles, prio=None):
+    n = desc.n_ops
+    prio = np.arange(n) if prio is None else prio
+    tmpl, role = np.zeros(max(n, 1), np.int32), np.zeros(max(n, 1), np.int32)
+    gm = G.gmg_create(desc)
+    st_d, pl_d = _dev(np.asarray(state, np.uint8) if n else np.zeros(1, np.uint8), np.uint8), _dev(place, np.uint8)
+    rnd = G.Round(gm, st_d, pl_d, _dev(prio if n else np.zeros(1), np.int64), _dev(tmpl, np.int32),
+                  _dev(role, np.int32), _dev(part_off, np.int32), _dev(part_dev, np.uint8), _dev(mapping, np.int32),
+                  n_roles, budget, max_batch)
+    rnd.step()
+    torch.cuda.synchronize()
+    want = R.round_step(desc, state, place, prio, tmpl, role, part_off, part_dev, mapping, n_roles, budget, max_batch)
+    return rnd, st_d, pl_d, want
+
+
+def test_degenerate_rounds():
+    from helpers import mk
+    chain = mk([[], [0], [1], [2]], [3, 4, 5, 6], n_dev=2, bw=1, lat=1)
+    place = np.zeros(16, np.uint8)
+    args = dict(part_off=[0, 1, 2], part_dev=[0, 1], mapping=[0, 0], n_roles=1)
+    # everything done: the unscheduled frontier is empty
+    rnd, st, pl, want = _one_round(chain, [2, 2, 2, 2], place, 8, 8, **args)
+    assert rnd.info.cpu().tolist() == want[0] and want[0][5] == R.EMPTY
+    # budget 0: nothing is scheduled even with a frontier
+    rnd, st, pl, want = _one_round(chain, [0, 0, 0, 0], place, 0, 8, **args)
+    assert rnd.info.cpu().tolist() == want[0] and want[0][5] == R.BUDGET
+    assert st.cpu().tolist() == [0, 0, 0, 0]
+    # batch cap 1: exactly the chosen op
+    rnd, st, pl, want = _one_round(chain, [0, 0, 0, 0], place, 8, 1, **args)
+    assert rnd.info.cpu().tolist() == want[0] and want[1] == [0]
+    assert st.cpu().tolist() == want[4].tolist() and pl.cpu().tolist() == want[5].tolist()
+    # every candidate maps to a slot outside its partition: nothing feasible, nothing written
+    bad = dict(part_off=[0, 1, 2], part_dev=[0, 1], mapping=[3, 3], n_roles=1)
+    rnd, st, pl, want = _one_round(chain, [0, 0, 0, 0], place, 8, 8, **bad)
+    assert want[0][5] == R.NO_FEASIBLE and rnd.info.cpu().tolist() == want[0]
+    assert st.cpu().tolist() == [0, 0, 0, 0] and pl.cpu().tolist() == place.tolist()
+    # an empty graph
+    empty = mk([], [], n_dev=2)
+    rnd, st, pl, want = _one_round(empty, np.zeros(0, np.uint8), place, 8, 8, **args)
+    assert rnd.info.cpu().tolist()[5] == R.EMPTY and rnd.info.cpu().tolist()[1] == -1
