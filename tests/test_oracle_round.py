@@ -98,3 +98,12 @@ def test_rounds_keep_the_schedule_closed_and_pick_the_best_row():
                 assert all(state2[q] for q in pred[i])
         state, place = state2, place2
         state[state == 1] = np.where(g.random(int((state == 1).sum())) < 0.5, 2, 1)   # some finish
+
+
+def test_collection_takes_the_smallest_waiting_id():
+    # 0 -> {1, 3}, 1 -> 2: after 0 and 1, op 2 (smaller id) comes before op 3
+    d = mk([[], [0], [1], [0]], [1] * 4)
+    _, batch = R.select(d, [0] * 4, [0, 1, 2, 3], budget=10, max_batch=3)
+    assert batch == [0, 1, 2]
+    _, batch = R.select(d, [0] * 4, [0, 1, 2, 3], budget=10, max_batch=10)
+    assert batch == [0, 1, 2, 3]
