@@ -63,9 +63,9 @@ def _code_only(text: str) -> str:
     return "\n".join(lines)
 
 
-def kernel_hash() -> str:
+def kernel_hash(extra=()) -> str:
     h = hashlib.sha256()
-    for f in KERNEL_SOURCES:
+    for f in list(KERNEL_SOURCES) + [os.path.join(ROOT, "paper_2608_15762_gb300", "csrc", e) for e in extra]:
         with open(f, encoding="utf-8") as fh:
             h.update(_code_only(fh.read()).encode())
     return h.hexdigest()[:16]
@@ -522,6 +522,33 @@ def round_setup(seed: int = 12):
                 role=np.tile(np.arange(per), 8).astype(np.int32), budget=128, max_batch=64)
 
 
+ROUND_PROFILE = os.path.join(PROFILE_DIR, "rounds_prefill-8x32L-N3088-D8-P14-B128-batch64.txt")
+
+
+def round_roofline(ms):
+    """Issue-slot roofline of a round: warp instructions per round (all its
+    kernels, from the committed ncu summary, if taken on the current sources)
+    over the measured round time."""
+    import torch
+    pk = peaks()
+    props = torch.cuda.get_device_properties(torch.device("cuda", 0))
+    peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9
+    roof = {"bound": "alu", "achieved": None, "peak": peak, "unit": "Ginst/s", "frac": None, "traffic": None,
+            "note": "latency-bound: 14 candidates are 14 warps; a round takes one candidate simulation's "
+                    "latency plus 8 small launches"}
+    vals = {}
+    if os.path.exists(ROUND_PROFILE):
+        with open(ROUND_PROFILE) as f:
+            for line in f:
+                if ":" in line and not line.startswith("#"):
+                    k, v = line.split(":", 1)
+                    vals[k.strip()] = v.strip()
+    if vals.get("kernel_source_sha256") == kernel_hash(("gmground.cu",)) and "inst_per_round" in vals:
+        ach = float(vals["inst_per_round"]) / (ms / 1000) / 1e9
+        roof.update(achieved=ach, frac=ach / peak, inst_src=os.path.relpath(ROUND_PROFILE, ROOT))
+    return roof
+
+
 def run_rounds(args):
     import numpy as np
     import torch
@@ -589,10 +616,7 @@ def run_rounds(args):
                        "rounds_to_schedule_every_op": needed, "ops_scheduled": scheduled},
             "ms_per_step_best": min(ms_all), "ms_per_step_median": statistics.median(ms_all),
             "candidates_per_s": 14 * 1000.0 / ms,
-            "roofline": {"bound": "alu", "achieved": None, "peak": None, "unit": "Ginst/s", "frac": None,
-                         "traffic": None,
-                         "note": "latency-bound: 14 candidates are 14 warps; a round takes one candidate "
-                                 "simulation's latency plus 8 small launches"},
+            "roofline": round_roofline(ms),
             "gpu_launches": 9 * rounds, "clocks": clocks}
     if not args.no_cpu_baseline:
         from oracle import round as OR
