@@ -5,8 +5,10 @@ Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 ``oracle/build.py``) and exposes numpy-level calls:
 
 * ``check(desc)`` -> 0 or a negative error code,
-* ``simulate(desc, place_row)`` -> dict with summary fields, peak, req_done,
-  ready/start/finish per op,
+* ``simulate(desc, place_row, arbitrated=False)`` -> dict with summary
+  fields, peak, req_done, ready/start/finish per op (arbitrated: transfers
+  through the arbiter of Sec. 3.5.2, plus the transfer table),
+* ``transfers(desc, place_row)`` -> the arbitrated transfers of one placement,
 * ``simulate_batch(desc, place, nthreads)`` -> structured summaries, peaks,
   req_done,
 * ``incremental_batch(desc, base, moves, nthreads)`` -> same,
@@ -38,7 +40,8 @@ class _Graph(C.Structure):
         (name, C.c_void_p) for name in (
             "pred_off", "pred_idx", "cons_off", "cons_idx", "dur", "out_bytes", "release",
             "req_id", "scored", "deadline", "cap", "base", "avail0", "bw", "lat")] + [
-        ("n_types", C.c_int32), ("dev_type", C.c_void_p), ("dur_type", C.c_void_p)]
+        ("n_types", C.c_int32), ("dev_type", C.c_void_p), ("dur_type", C.c_void_p),
+        ("transfer_mode", C.c_int32), ("link_id", C.c_void_p)]
 
 
 _LIB = None
@@ -61,6 +64,8 @@ def lib():
         L.orc_incremental_batch.restype = C.c_int
         L.orc_select_best.argtypes = [vp, i32, i32, vp]
         L.orc_select_best.restype = i64
+        L.orc_transfers.argtypes = [vp, vp, vp, i64]
+        L.orc_transfers.restype = i64
         _LIB = L
     return _LIB
 
@@ -72,7 +77,7 @@ def _ptr(a):
 class _GraphHolder:
     """Keeps the numpy arrays alive while the C struct points into them."""
 
-    def __init__(self, desc):
+    def __init__(self, desc, arbitrated=False):
         d = desc.normalized()
         self.desc = d
         self.g = _Graph(d.n_ops, d.n_edges, d.n_dev, d.n_req,
@@ -80,7 +85,7 @@ class _GraphHolder:
                         _ptr(d.dur), _ptr(d.out_bytes), _ptr(d.release), _ptr(d.req_id),
                         _ptr(d.scored), _ptr(d.deadline), _ptr(d.cap), _ptr(d.base),
                         _ptr(d.avail0), _ptr(d.bw), _ptr(d.lat), d.n_types, _ptr(d.dev_type),
-                        _ptr(d.dur_by_type))
+                        _ptr(d.dur_by_type), 1 if arbitrated else 0, _ptr(d.link_id))
 
     @property
     def ref(self):
@@ -91,13 +96,15 @@ def hw_threads() -> int:
     return int(lib().orc_hw_threads())
 
 
-def check(desc) -> int:
-    h = _GraphHolder(desc)
+def check(desc, arbitrated=False) -> int:
+    h = _GraphHolder(desc, arbitrated)
     return int(lib().orc_check(C.addressof(h.g)))
 
 
-def simulate(desc, place_row) -> dict:
-    h = _GraphHolder(desc)
+def simulate(desc, place_row, arbitrated=False) -> dict:
+    """One placement; ``arbitrated``: transfers go through the arbiter of
+    Sec. 3.5.2 (the dict then also holds ``transfers``)."""
+    h = _GraphHolder(desc, arbitrated)
     d = h.desc
     row = np.ascontiguousarray(place_row, dtype=np.uint8)
     assert row.shape[0] >= d.n_ops
@@ -114,12 +121,27 @@ def simulate(desc, place_row) -> dict:
     out = {k: s[0][k].item() for k in SUMMARY_DTYPE.names if k != "reserved"}
     out.update(peak=peak, req_done=req[:d.n_req], ready=r[:d.n_ops], start=st[:d.n_ops],
                finish=fi[:d.n_ops])
+    if arbitrated:
+        out["transfers"] = transfers(desc, row)
     return out
 
 
-def simulate_batch(desc, place, nthreads: int = 0):
+def transfers(desc, place_row) -> np.ndarray:
+    """Arbitrated transfers of one placement in arbitration order: int64 rows
+    (producer, destination, intent time, start, completion)."""
+    h = _GraphHolder(desc, True)
+    row = np.ascontiguousarray(place_row, dtype=np.uint8)
+    m = lib().orc_transfers(C.addressof(h.g), row.ctypes.data, None, 0)
+    if m < 0:
+        raise ValueError("oracle rejected the graph: %d" % m)
+    rows = np.zeros((max(m, 1), 5), np.int64)
+    lib().orc_transfers(C.addressof(h.g), row.ctypes.data, rows.ctypes.data, m)
+    return rows[:m]
+
+
+def simulate_batch(desc, place, nthreads: int = 0, arbitrated=False):
     """place: uint8 [K, ld].  Returns (summary[K], peak[K, D], req_done[K, R])."""
-    h = _GraphHolder(desc)
+    h = _GraphHolder(desc, arbitrated)
     d = h.desc
     place = np.ascontiguousarray(place, dtype=np.uint8)
     K, ld = place.shape

@@ -39,6 +39,20 @@
 //    the rest the one with the smallest average completion time of the
 //    scored operators wins (sum of finish times, same argmin), ties to the
 //    lowest candidate index.
+//  * Arbitrated transfers (Sec. 3.5.2, "Tensor Transfer Arbitration"; the
+//    transfer_mode = 1 variant).  A producer's completion raises one transfer
+//    intent per distinct remote accelerator of its successors.  The master
+//    keeps the pending intents and activates a conflict-free set of them at
+//    every trigger: the arrival of an intent or the completion of a
+//    transfer.  An active transfer s -> e holds s's sending endpoint, e's
+//    receiving endpoint and the communication link of the pair (link ids are
+//    an input; by default every ordered pair has its own link).  The paper
+//    leaves the choice among conflicting intents open; here, after every
+//    completion and intent at time t, the pending intents are visited in
+//    (intent time, producer id, destination id) order and each one that
+//    conflicts with no active transfer starts at t.  It lasts the transfer
+//    estimate; the receive buffer (Recv) is allocated when it starts, and the
+//    consumers' input arrives when it completes.
 //  * Incremental what-if (Sec. 3.4.2): a candidate given as moves against a
 //    base placement is, by definition, the full simulation of the moved
 //    placement; its event count is the number of operators whose base ready
@@ -101,6 +115,8 @@ typedef struct {
   int32_t n_types;           // >= 2: durations per (op, accelerator type)
   const uint8_t* dev_type;   // [n_dev]
   const int64_t* dur_type;   // [n_ops * n_types], op-major
+  int32_t transfer_mode;     // 0 = transfers are pure latency, 1 = arbitrated
+  const int32_t* link_id;    // [n_dev*n_dev] link of each ordered pair; NULL: its own
 } orc_graph;
 
 typedef struct {
@@ -130,6 +146,8 @@ struct Graph {
   int T = 0;                     // accelerator types (0: one type, dur)
   std::vector<uint8_t> dev_type;  // [D]
   std::vector<int64_t> dur_type;  // [n*T]
+  int mode = 0;                   // 1: arbitrated transfers
+  std::vector<int> link;          // [D*D] link id of each ordered pair
 };
 
 // Duration of op i on accelerator d.
@@ -242,6 +260,15 @@ int build(const orc_graph* in, Graph& g) {
       g.lat[size_t(d) * D + e] = in->lat[size_t(d) * D + e];
       if (g.bw[size_t(d) * D + e] < 1 || g.lat[size_t(d) * D + e] < 0) return kEInval;
     }
+  if (in->transfer_mode < 0 || in->transfer_mode > 1) return kEInval;
+  g.mode = in->transfer_mode;
+  g.link.assign(size_t(D) * D, 0);
+  for (int d = 0; d < D; ++d)
+    for (int e = 0; e < D; ++e) {
+      const size_t k = size_t(d) * D + e;
+      g.link[k] = in->link_id ? in->link_id[k] : int(k);
+      if (d != e && (g.link[k] < 0 || g.link[k] >= D * D)) return kEInval;
+    }
   // Overflow guard: every time stays below (start + all durations + one
   // transfer per edge and per op), every score below n times that, every
   // live-memory figure below base + every copy of every tensor.
@@ -271,9 +298,23 @@ int build(const orc_graph* in, Graph& g) {
   return 0;
 }
 
+// One cross-accelerator transfer of op p's output to accelerator e.
+struct Transfer {
+  int p, e;
+  int64_t intent, start, done;
+};
+
 struct Result {
   orc_summary s;
   std::vector<int64_t> peak, req_done, ready, start, finish;
+  std::vector<Transfer> xfers;  // arbitrated mode: every transfer
+};
+
+// A copy of op i's output on another accelerator: allocated when its
+// transfer starts, present there once the transfer has arrived.
+struct Copy {
+  int e;
+  int64_t alloc, arrive;
 };
 
 void fill_invalid(const Graph& g, int32_t status, Result& res) {
@@ -290,60 +331,13 @@ void fill_invalid(const Graph& g, int32_t status, Result& res) {
   res.finish.assign(g.n, 0);
 }
 
-// Sec. 3.3.3: event-driven simulation of one placement.
-void simulate(const Graph& g, const uint8_t* dev, Result& res) {
+// HBM residency, request completion, score and summary of one simulated
+// placement, given every op's ready, start and finish time and the remote
+// copies of every op's output (Sec. 3.3.2, Sec. 3.4.2).
+void settle(const Graph& g, const uint8_t* dev, std::vector<int64_t>& r, std::vector<int64_t>& s,
+            std::vector<int64_t>& f, const std::vector<std::vector<Copy>>& copies, Result& res) {
   const int n = g.n, D = g.D;
-  for (int i = 0; i < n; ++i)
-    if (dev[i] >= D) {
-      fill_invalid(g, kSimBadDev, res);
-      return;
-    }
-  std::vector<int64_t> r(n, 0), s(n, -1), f(n, -1);
-
-  // Event: (time, class, id).  Class 0 = an operator completes (id >= 0) or
-  // an accelerator becomes available (id = -1 - d); class 1 = one input of
-  // operator id arrives (a predecessor's output, or the op's own release).
-  typedef std::tuple<int64_t, int, int> Ev;
-  std::priority_queue<Ev, std::vector<Ev>, std::greater<Ev>> events;
-  std::vector<int> arrived(n, 0);
-  std::vector<std::set<std::pair<int64_t, int>>> ready_q(D);  // (ready time, op)
-  std::vector<int> running(D, -1);
-  for (int i = 0; i < n; ++i) events.push(Ev(g.release[i], 1, i));
-  for (int d = 0; d < D; ++d)
-    if (g.avail0[d] > 0) events.push(Ev(g.avail0[d], 0, -1 - d));
-
-  while (!events.empty()) {
-    const int64_t now = std::get<0>(events.top());
-    // (i) completions at `now`: free the queue, send outputs to successors.
-    while (!events.empty() && std::get<0>(events.top()) == now && std::get<1>(events.top()) == 0) {
-      int id = std::get<2>(events.top());
-      events.pop();
-      if (id < 0) continue;  // accelerator becomes available
-      running[dev[id]] = -1;
-      for (int j : g.succ[id]) events.push(Ev(now + xfer(g, dev[id], dev[j], g.bytes[id]), 1, j));
-    }
-    // (ii) input arrivals at `now`: an op whose inputs are all present is
-    // ready, with ready time = its last arrival.
-    while (!events.empty() && std::get<0>(events.top()) == now && std::get<1>(events.top()) == 1) {
-      int j = std::get<2>(events.top());
-      events.pop();
-      arrived[j] += 1;
-      r[j] = now;
-      if (arrived[j] == int(g.pred[j].size()) + 1) ready_q[dev[j]].insert({r[j], j});
-    }
-    // (iii) every idle queue starts its ready op with the earliest ready time.
-    for (int d = 0; d < D; ++d) {
-      if (running[d] >= 0 || g.avail0[d] > now || ready_q[d].empty()) continue;
-      int i = ready_q[d].begin()->second;
-      ready_q[d].erase(ready_q[d].begin());
-      running[d] = i;
-      s[i] = now;
-      f[i] = now + dur_on(g, i, d);
-      events.push(Ev(f[i], 0, i));
-    }
-  }
-
-  // HBM evolution: per accelerator, every copy is an interval [alloc, free).
+  // per accelerator, every copy is an interval [alloc, free)
   struct MemEv {
     int64_t t;
     int cls;  // 0 = free, 1 = alloc (frees first at equal times)
@@ -354,9 +348,6 @@ void simulate(const Graph& g, const uint8_t* dev, Result& res) {
   for (int i = 0; i < n; ++i) {
     const int d = dev[i];
     const int64_t b = g.bytes[i];
-    std::map<int, int64_t> arrival;  // remote accelerator -> arrival time
-    for (int j : g.succ[i])
-      if (dev[j] != d) arrival[dev[j]] = f[i] + xfer(g, d, dev[j], b);
     std::map<int, int64_t> last_use;  // accelerator -> latest finish of a listed consumer
     for (int c : g.cons[i]) {
       auto it = last_use.find(dev[c]);
@@ -364,15 +355,15 @@ void simulate(const Graph& g, const uint8_t* dev, Result& res) {
       else it->second = std::max(it->second, f[c]);
     }
     int64_t src_free = f[i];
-    for (auto& kv : arrival) src_free = std::max(src_free, kv.second);
+    for (const Copy& c : copies[i]) src_free = std::max(src_free, c.arrive);
     if (last_use.count(d)) src_free = std::max(src_free, last_use[d]);
     mem[d].push_back({s[i], 1, i, b});
     mem[d].push_back({src_free, 0, i, -b});
-    for (auto& kv : arrival) {
-      int64_t t_free = kv.second;
-      if (last_use.count(kv.first)) t_free = std::max(t_free, last_use[kv.first]);
-      mem[kv.first].push_back({f[i], 1, i, b});
-      mem[kv.first].push_back({t_free, 0, i, -b});
+    for (const Copy& c : copies[i]) {
+      int64_t t_free = c.arrive;
+      if (last_use.count(c.e)) t_free = std::max(t_free, last_use[c.e]);
+      mem[c.e].push_back({c.alloc, 1, i, b});
+      mem[c.e].push_back({t_free, 0, i, -b});
     }
   }
   res.peak.assign(D, 0);
@@ -426,6 +417,195 @@ void simulate(const Graph& g, const uint8_t* dev, Result& res) {
   res.finish = std::move(f);
 }
 
+
+// Sec. 3.3.3 with the arbitrated transfers of Sec. 3.5.2: the same
+// event-driven loop, where a remote input arrives when its transfer, started
+// by the arbiter, completes.  Equal-time order: operator and transfer
+// completions, new intents, arbitration (repeated while a transfer started
+// at this time also completes at it), then input arrivals, then dispatch on
+// every idle accelerator.
+void simulate_arb(const Graph& g, const uint8_t* dev, Result& res) {
+  const int n = g.n, D = g.D;
+  std::vector<int64_t> r(n, 0), s(n, -1), f(n, -1);
+  std::vector<Transfer> X;
+
+  // Event: (time, class, id).  Class 0 = an operator completes (id >= 0) or
+  // an accelerator becomes available (id = -1 - d); class 1 = transfer id
+  // completes; class 2 = one input of operator id arrives (a local
+  // predecessor's output, a transferred one, or the op's own release).
+  typedef std::tuple<int64_t, int, int> Ev;
+  std::priority_queue<Ev, std::vector<Ev>, std::greater<Ev>> events;
+  std::vector<int> arrived(n, 0);
+  std::vector<std::set<std::pair<int64_t, int>>> ready_q(D);
+  std::vector<int> running(D, -1);
+  // the communication graph: pending intents in arbitration order, and the
+  // endpoints and links held by the active transfers
+  std::set<std::tuple<int64_t, int, int, int>> pending;  // (intent time, p, e, transfer id)
+  std::vector<bool> sending(D, false), receiving(D, false);
+  std::set<int> links_busy;
+  for (int i = 0; i < n; ++i) events.push(Ev(g.release[i], 2, i));
+  for (int d = 0; d < D; ++d)
+    if (g.avail0[d] > 0) events.push(Ev(g.avail0[d], 0, -1 - d));
+
+  auto at_now = [&](int64_t now, int cls) {
+    return !events.empty() && std::get<0>(events.top()) == now && std::get<1>(events.top()) == cls;
+  };
+  while (!events.empty()) {
+    const int64_t now = std::get<0>(events.top());
+    while (at_now(now, 0) || at_now(now, 1)) {
+      bool trigger = false;
+      // (i) operator completions: local successors get their input now; one
+      // intent per distinct remote accelerator of a successor.
+      while (at_now(now, 0)) {
+        const int id = std::get<2>(events.top());
+        events.pop();
+        if (id < 0) continue;
+        running[dev[id]] = -1;
+        std::set<int> remote;
+        for (int j : g.succ[id]) {
+          if (dev[j] == dev[id]) events.push(Ev(now, 2, j));
+          else remote.insert(dev[j]);
+        }
+        for (int e : remote) {
+          X.push_back({id, e, now, -1, -1});
+          pending.insert(std::make_tuple(now, id, e, int(X.size()) - 1));
+          trigger = true;
+        }
+      }
+      // (ii) transfer completions: release the endpoints and the link; the
+      // successors on the destination get their input now.
+      while (at_now(now, 1)) {
+        const int x = std::get<2>(events.top());
+        events.pop();
+        Transfer& t = X[x];
+        t.done = now;
+        const int src = dev[t.p];
+        sending[src] = false;
+        receiving[t.e] = false;
+        links_busy.erase(g.link[size_t(src) * D + t.e]);
+        for (int j : g.succ[t.p])
+          if (dev[j] == t.e) events.push(Ev(now, 2, j));
+        trigger = true;
+      }
+      // (iii) arbitration: start every pending intent, in order, whose
+      // endpoints and link are free.
+      if (trigger) {
+        for (auto it = pending.begin(); it != pending.end();) {
+          const int x = std::get<3>(*it);
+          Transfer& t = X[x];
+          const int src = dev[t.p];
+          const int lk = g.link[size_t(src) * D + t.e];
+          if (sending[src] || receiving[t.e] || links_busy.count(lk)) {
+            ++it;
+            continue;
+          }
+          sending[src] = true;
+          receiving[t.e] = true;
+          links_busy.insert(lk);
+          t.start = now;
+          events.push(Ev(now + xfer(g, src, t.e, g.bytes[t.p]), 1, x));
+          it = pending.erase(it);
+        }
+      }
+    }
+    // (iv) input arrivals: an op whose inputs are all present is ready.
+    while (at_now(now, 2)) {
+      const int j = std::get<2>(events.top());
+      events.pop();
+      arrived[j] += 1;
+      r[j] = now;
+      if (arrived[j] == int(g.pred[j].size()) + 1) ready_q[dev[j]].insert({r[j], j});
+    }
+    // (v) every idle queue starts its ready op with the earliest ready time.
+    for (int d = 0; d < D; ++d) {
+      if (running[d] >= 0 || g.avail0[d] > now || ready_q[d].empty()) continue;
+      const int i = ready_q[d].begin()->second;
+      ready_q[d].erase(ready_q[d].begin());
+      running[d] = i;
+      s[i] = now;
+      f[i] = now + dur_on(g, i, d);
+      events.push(Ev(f[i], 0, i));
+    }
+  }
+
+  std::vector<std::vector<Copy>> copies(n);
+  for (const Transfer& t : X) copies[t.p].push_back({t.e, t.start, t.done});
+  std::sort(X.begin(), X.end(), [](const Transfer& a, const Transfer& b) {
+    return std::tie(a.intent, a.p, a.e) < std::tie(b.intent, b.p, b.e);
+  });
+  settle(g, dev, r, s, f, copies, res);
+  res.xfers = std::move(X);
+}
+
+// Sec. 3.3.3: event-driven simulation of one placement.
+void simulate(const Graph& g, const uint8_t* dev, Result& res) {
+  const int n = g.n, D = g.D;
+  for (int i = 0; i < n; ++i)
+    if (dev[i] >= D) {
+      fill_invalid(g, kSimBadDev, res);
+      return;
+    }
+  if (g.mode == 1) {
+    simulate_arb(g, dev, res);
+    return;
+  }
+  std::vector<int64_t> r(n, 0), s(n, -1), f(n, -1);
+
+  // Event: (time, class, id).  Class 0 = an operator completes (id >= 0) or
+  // an accelerator becomes available (id = -1 - d); class 1 = one input of
+  // operator id arrives (a predecessor's output, or the op's own release).
+  typedef std::tuple<int64_t, int, int> Ev;
+  std::priority_queue<Ev, std::vector<Ev>, std::greater<Ev>> events;
+  std::vector<int> arrived(n, 0);
+  std::vector<std::set<std::pair<int64_t, int>>> ready_q(D);  // (ready time, op)
+  std::vector<int> running(D, -1);
+  for (int i = 0; i < n; ++i) events.push(Ev(g.release[i], 1, i));
+  for (int d = 0; d < D; ++d)
+    if (g.avail0[d] > 0) events.push(Ev(g.avail0[d], 0, -1 - d));
+
+  while (!events.empty()) {
+    const int64_t now = std::get<0>(events.top());
+    // (i) completions at `now`: free the queue, send outputs to successors.
+    while (!events.empty() && std::get<0>(events.top()) == now && std::get<1>(events.top()) == 0) {
+      int id = std::get<2>(events.top());
+      events.pop();
+      if (id < 0) continue;  // accelerator becomes available
+      running[dev[id]] = -1;
+      for (int j : g.succ[id]) events.push(Ev(now + xfer(g, dev[id], dev[j], g.bytes[id]), 1, j));
+    }
+    // (ii) input arrivals at `now`: an op whose inputs are all present is
+    // ready, with ready time = its last arrival.
+    while (!events.empty() && std::get<0>(events.top()) == now && std::get<1>(events.top()) == 1) {
+      int j = std::get<2>(events.top());
+      events.pop();
+      arrived[j] += 1;
+      r[j] = now;
+      if (arrived[j] == int(g.pred[j].size()) + 1) ready_q[dev[j]].insert({r[j], j});
+    }
+    // (iii) every idle queue starts its ready op with the earliest ready time.
+    for (int d = 0; d < D; ++d) {
+      if (running[d] >= 0 || g.avail0[d] > now || ready_q[d].empty()) continue;
+      int i = ready_q[d].begin()->second;
+      ready_q[d].erase(ready_q[d].begin());
+      running[d] = i;
+      s[i] = now;
+      f[i] = now + dur_on(g, i, d);
+      events.push(Ev(f[i], 0, i));
+    }
+  }
+
+  // Transfers are pure latency: every remote copy is allocated when the
+  // producer completes and arrives one transfer estimate later.
+  std::vector<std::vector<Copy>> copies(n);
+  for (int i = 0; i < n; ++i) {
+    std::map<int, int64_t> arrival;  // remote accelerator -> arrival time
+    for (int j : g.succ[i])
+      if (dev[j] != dev[i]) arrival[dev[j]] = f[i] + xfer(g, dev[i], dev[j], g.bytes[i]);
+    for (auto& kv : arrival) copies[i].push_back({kv.first, f[i], kv.second});
+  }
+  settle(g, dev, r, s, f, copies, res);
+}
+
 void write_out(const Graph& g, const Result& res, int64_t k, orc_summary* out, int64_t* peak,
                int64_t* req_done) {
   out[k] = res.s;
@@ -477,6 +657,25 @@ int orc_simulate(const orc_graph* in, const uint8_t* place, orc_summary* out, in
   if (start) std::memcpy(start, res.start.data(), sizeof(int64_t) * g.n);
   if (finish) std::memcpy(finish, res.finish.data(), sizeof(int64_t) * g.n);
   return 0;
+}
+
+// Arbitrated mode: the transfers of one candidate in arbitration order, as
+// rows (producer, destination, intent time, start, completion); returns
+// their number (rows beyond `cap` are not written) or a negative error.
+int64_t orc_transfers(const orc_graph* in, const uint8_t* place, int64_t* rows, int64_t cap) {
+  Graph g;
+  int rc = build(in, g);
+  if (rc) return rc;
+  if (g.mode != 1) return kEInval;
+  Result res;
+  simulate(g, place, res);
+  const int64_t m = int64_t(res.xfers.size());
+  for (int64_t x = 0; x < std::min(m, cap); ++x) {
+    const Transfer& t = res.xfers[x];
+    const int64_t v[5] = {t.p, t.e, t.intent, t.start, t.done};
+    std::memcpy(rows + 5 * x, v, sizeof(v));
+  }
+  return m;
 }
 
 // K candidates, row k of `place` at place + k*ld (Algorithm 1: each

@@ -91,6 +91,10 @@ class GmgDesc:
     # duration on every type ([N, T]); None = one type, `dur` everywhere
     dev_type: Optional[np.ndarray] = None
     dur_by_type: Optional[np.ndarray] = None
+    # arbitrated transfers: the communication link of every ordered accelerator
+    # pair ([D*D], row = source, ids in [0, D*D)); transfers over pairs with
+    # one id compete for that link.  None = every ordered pair its own link.
+    link_id: Optional[np.ndarray] = None
 
     @property
     def n_types(self) -> int:
@@ -128,7 +132,7 @@ class GmgDesc:
             avail0=c(self.avail0, np.int64), bw=c(self.bw, np.int64),
             lat=c(self.lat, np.int64), cons_off=c(self.cons_off, np.int32),
             cons_idx=c(self.cons_idx, np.int32), dev_type=c(self.dev_type, np.uint8),
-            dur_by_type=c(self.dur_by_type, np.int64))
+            dur_by_type=c(self.dur_by_type, np.int64), link_id=c(self.link_id, np.int32))
 
 
 @dataclass

@@ -14,6 +14,11 @@ notes) without looking at the oracle's event loop:
 * ``copies`` / ``memory_brute``: HBM copy intervals [alloc, free) derived
   from the residency rules, and live memory evaluated directly at every
   instant where it can change.
+* ``tick_sim_arb``: the tick simulation with arbitrated transfers (Sec.
+  3.5.2): at each microsecond, completions free their endpoints and links,
+  finished producers raise one intent per remote accelerator, and pending
+  intents start, in (intent time, producer, destination) order, whenever
+  their sending endpoint, receiving endpoint and link are free.
 """
 from __future__ import annotations
 
@@ -124,27 +129,110 @@ def sweep_sim(desc, place):
     return ready, start, finish
 
 
-def copies(desc, place, start, finish) -> List[Dict]:
-    """Every HBM copy as {dev, op, bytes, alloc, free}."""
+def link_of(desc, d, e):
+    D = desc.n_dev
+    return d * D + e if desc.link_id is None else int(desc.link_id[d * D + e])
+
+
+def tick_sim_arb(desc, place, t_max=100000):
+    """Returns (ready, start, finish, transfers); transfers: dicts with p, e,
+    intent, start, done."""
+    n, D = desc.n_ops, desc.n_dev
+    pred, succ, _ = lists(desc)
+    dev = [int(x) for x in place[:n]]
+    ready = [None] * n
+    start = [None] * n
+    finish = [None] * n
+    running = [None] * D
+    xs = {}            # (p, e) -> transfer
+    done_ops = 0
+    t = 0
+    while done_ops < n:
+        assert t <= t_max, "tick simulation did not finish"
+        for d in range(D):
+            i = running[d]
+            if i is not None and finish[i] == t:
+                running[d] = None
+                done_ops += 1
+                for e in sorted({dev[j] for j in succ[i] if dev[j] != d}):
+                    xs[(i, e)] = dict(p=i, e=e, intent=t, start=None, done=None)
+        # arbitration, repeated while a transfer completes at this tick
+        while True:
+            active = [x for x in xs.values() if x["start"] is not None and x["done"] > t]
+            pend = sorted((x for x in xs.values() if x["start"] is None),
+                          key=lambda x: (x["intent"], x["p"], x["e"]))
+            started = False
+            for x in pend:
+                src = dev[x["p"]]
+                clash = any(dev[y["p"]] == src or y["e"] == x["e"] or
+                            link_of(desc, dev[y["p"]], y["e"]) == link_of(desc, src, x["e"])
+                            for y in active)
+                if not clash:
+                    x["start"] = t
+                    x["done"] = t + xfer(desc, src, x["e"], desc.out_bytes[x["p"]])
+                    active.append(x)
+                    started = True
+            if not (started and any(x["done"] == t for x in active)):
+                break
+        for i in range(n):
+            if ready[i] is not None:
+                continue
+            ok = t >= int(desc.release[i])
+            for p in pred[i]:
+                if finish[p] is None or finish[p] > t:
+                    ok = False
+                elif dev[p] != dev[i]:
+                    x = xs.get((p, dev[i]))
+                    ok = ok and x is not None and x["done"] is not None and x["done"] <= t
+                if not ok:
+                    break
+            if ok:
+                ready[i] = t
+        for d in range(D):
+            if running[d] is not None or t < int(desc.avail0[d]):
+                continue
+            cands = [(ready[i], i) for i in range(n)
+                     if dev[i] == d and ready[i] is not None and start[i] is None]
+            if cands:
+                _, i = min(cands)
+                start[i] = t
+                finish[i] = t + desc.dur_on(i, d)
+                running[d] = i
+        t += 1
+    xl = sorted(xs.values(), key=lambda x: (x["intent"], x["p"], x["e"]))
+    return ready, start, finish, xl
+
+
+def copies(desc, place, start, finish, transfers=None) -> List[Dict]:
+    """Every HBM copy as {dev, op, bytes, alloc, free}.  Without
+    ``transfers`` a remote copy is allocated at the producer's finish and
+    arrives one transfer estimate later; with them (arbitrated transfers) it
+    is allocated when its transfer starts and arrives when it is done."""
     n = desc.n_ops
     pred, succ, cons = lists(desc)
     dev = [int(x) for x in place[:n]]
+    tx = {} if transfers is None else {(x["p"], x["e"]): x for x in transfers}
     out = []
     for i in range(n):
         b = int(desc.out_bytes[i])
         d = dev[i]
         remote = sorted({dev[j] for j in succ[i] if dev[j] != d})
-        arrive = {e: finish[i] + xfer(desc, d, e, b) for e in remote}
+        if transfers is None:
+            alloc = {e: finish[i] for e in remote}
+            arrive = {e: finish[i] + xfer(desc, d, e, b) for e in remote}
+        else:
+            alloc = {e: tx[(i, e)]["start"] for e in remote}
+            arrive = {e: tx[(i, e)]["done"] for e in remote}
         src_free = max([finish[i]] + list(arrive.values()) +
                        [finish[c] for c in cons[i] if dev[c] == d])
         out.append(dict(dev=d, op=i, bytes=b, alloc=start[i], free=src_free))
         for e in remote:
             t_free = max([arrive[e]] + [finish[c] for c in cons[i] if dev[c] == e])
-            out.append(dict(dev=e, op=i, bytes=b, alloc=finish[i], free=t_free))
+            out.append(dict(dev=e, op=i, bytes=b, alloc=alloc[e], free=t_free))
     return out
 
 
-def memory_brute(desc, place, start, finish):
+def memory_brute(desc, place, start, finish, transfers=None):
     """Peak per device and first violation (time, op, dev) by evaluating live
     memory directly from the copy intervals at every time where it can change
     (every alloc and free instant; it is constant in between).  At an instant
@@ -152,7 +240,7 @@ def memory_brute(desc, place, start, finish):
     allocated at t are added in op order; the first one that leaves the total
     above capacity is that device's violation at t."""
     D = desc.n_dev
-    cps = copies(desc, place, start, finish)
+    cps = copies(desc, place, start, finish, transfers)
     peak = [int(desc.base[d]) for d in range(D)]
     viol = None
     for d in range(D):
@@ -173,10 +261,10 @@ def memory_brute(desc, place, start, finish):
     return peak, viol
 
 
-def summarize(desc, place, start, finish, ready=None):
+def summarize(desc, place, start, finish, ready=None, transfers=None):
     """Summary dict computed from a schedule by the stated definitions."""
     n = desc.n_ops
-    peak, viol = memory_brute(desc, place, start, finish)
+    peak, viol = memory_brute(desc, place, start, finish, transfers)
     R = desc.n_req
     done = [0] * R
     for i in range(n):
