@@ -105,10 +105,20 @@ typedef struct {
   int32_t n_types;             /* T in [0, 256] */
   const uint8_t* dev_type;     /* [D] each < T */
   const int64_t* dur_by_type;  /* [N*T] row-major by op: dur of op i on type t at [i*T + t], >= 1 */
+  /* Communication links, read only by arbitrated transfers (sim_opts_t.
+   * transfer_mode): transfers over ordered pairs with the same id compete for
+   * that link (Sec. 3.5.2).  Optional (NULL: every ordered pair has a link of
+   * its own, so only the endpoints are shared).  Off-diagonal ids in
+   * [0, D*D); the diagonal is ignored. */
+  const int32_t* link_id;      /* [D*D] row = source */
 } gmg_desc_t;
 
 typedef struct gmg gmg_t;           /* opaque; host metadata + borrowed device workspace */
 typedef struct gmg_base gmg_base_t; /* opaque; base schedule snapshot for incremental runs */
+
+/* sim_opts_t.transfer_mode */
+#define GMG_TRANSFER_LATENCY 0    /* a transfer starts when its producer finishes (Sec. 3.3.2) */
+#define GMG_TRANSFER_ARBITRATED 1 /* transfers wait for the arbiter (Sec. 3.5.2); sim_batch only */
 
 typedef struct {
   int32_t score_mode;       /* select_best: 0 = score, 1 = (sla_miss, score) */
@@ -116,7 +126,8 @@ typedef struct {
   const int32_t* d_trace_k; /* device [n_trace]: candidate indices to trace (distinct) */
   int32_t queue_cap;        /* per-candidate event-queue entries; 0 = library default */
   int32_t warps_per_block;  /* 0 = library default (tuning knob) */
-  int32_t reserved[4];      /* must be 0 */
+  int32_t transfer_mode;    /* GMG_TRANSFER_*; 0 = GMG_TRANSFER_LATENCY */
+  int32_t reserved[3];      /* must be 0 */
 } sim_opts_t;
 
 /* Caller-owned device output arrays for K candidates. */
@@ -173,7 +184,23 @@ size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts);
 /* Simulate K full placements (paper Sec. 3.3.3 for each candidate p of
  * Algorithm 1).  d_place: device uint8 [K][ld], row k = device of every op,
  * ld >= n_ops, ld % 16 == 0, 16-byte aligned.  Writes every field of *d_out
- * for every candidate.  d_scratch >= sim_scratch_bytes, 256-byte aligned. */
+ * for every candidate.  d_scratch >= sim_scratch_bytes, 256-byte aligned.
+ *
+ * opts->transfer_mode = GMG_TRANSFER_ARBITRATED simulates the arbitrated
+ * transfers of Sec. 3.5.2 ("Tensor Transfer Arbitration") instead of pure
+ * latency: a producer's completion raises one transfer intent per distinct
+ * remote accelerator of its successors; after every intent or transfer
+ * completion at time t, the pending intents are visited in (intent time,
+ * producer id, destination id) order and each one whose sending endpoint
+ * (its source accelerator), receiving endpoint (its destination) and link
+ * (gmg_desc_t.link_id) are free of every active transfer starts at t.  It
+ * lasts the transfer estimate; its receive buffer is allocated when it
+ * starts; the successors' input arrives when it completes.  The paper does
+ * not fix the choice among conflicting intents: this FIFO-greedy order is
+ * the library's.  Needs n_dev <= 32 (else GMG_EINVAL) and op ids < 2^27 with
+ * accelerator ids that fit the packed event key (else GMG_ERANGE).
+ * base_create, sim_incremental and their size queries accept only
+ * GMG_TRANSFER_LATENCY (GMG_EINVAL, or 0 bytes, otherwise). */
 int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld,
               const sim_opts_t* opts, const sim_out_t* d_out, void* d_scratch,
               size_t scratch_bytes, gmg_stream_t stream);

@@ -1,0 +1,37 @@
+// Launch parameters of the arbitrated-transfer simulation (sim_batch with
+// transfer_mode = GMG_TRANSFER_ARBITRATED).  Private to the library: shared
+// by the host translation unit (gmgsim_host.cu) and gmgsim_arb.cu.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "gmg_layout.h"
+
+namespace gsim {
+
+struct ArbParams {
+  SimParams P;            // the full simulation's parameters (slot offsets inside P too)
+  const uint16_t* link;   // [D*D] link id of each ordered accelerator pair (< D*D)
+  int32_t xcap;           // transfers per candidate (sum over ops of min(successors, D-1))
+  int32_t tqs;            // transfer-event heap slots in shared memory per warp (>= 33)
+  int32_t tqcap;          // transfer-event heap slots per warp
+  int32_t smem_arb;       // shared bytes of the arbitration state per warp
+  int64_t smem_std;       // shared bytes of the simulation state of all warps of a block
+  // byte offsets inside a warp's scratch slot
+  int64_t off_cnt;        // int32 [N]  inputs present
+  int64_t off_rmax;       // time  [N]  latest input arrival so far
+  int64_t off_refs;       // int32 [N]  holds left on an op's own output copy
+  int64_t off_xent;       // uint32 [xcap]  intent: producer << 5 | destination
+  int64_t off_xnext;      // int32 [xcap]  next intent of the same pair (-1: last)
+  int64_t off_qhead;      // int32 [D*D]  first pending intent of each pair (-1: none)
+  int64_t off_qtail;      // int32 [D*D]
+  int64_t off_tq;         // uint64 [tqcap - tqs]  transfer-event heap beyond shared memory
+};
+
+// Kernel entry of one instance (for occupancy queries) and the launcher.
+const void* arb_kernel_ptr(bool t32, bool types);
+cudaError_t launch_arb(bool t32, bool types, const ArbParams& A, int grid, int block, size_t smem,
+                       cudaStream_t st);
+
+}  // namespace gsim

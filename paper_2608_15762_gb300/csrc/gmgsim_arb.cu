@@ -1,0 +1,491 @@
+// sim_batch with arbitrated transfers (Sec. 3.5.2, "Tensor Transfer
+// Arbitration"): one warp per candidate, as in the pure-latency simulation,
+// with a second event stream for the transfers.
+//
+//   INTENT(f_p, p, e)  producer p finished; its output is wanted on
+//                      accelerator e (one intent per distinct remote
+//                      accelerator of p's successors).  The intent joins the
+//                      FIFO queue of the pair (dev p, e).
+//   DONE(c, p, e)      the transfer arrived: e's receiving endpoint, the
+//                      sender's endpoint and the pair's link are free again;
+//                      p's successors on e have one more input present.
+//
+// After every INTENT / DONE at time t the arbiter starts, in (intent time,
+// producer, destination) order, every pending intent whose sending endpoint,
+// receiving endpoint and link are all free (the communication graph of Sec.
+// 3.5.2; the selection rule among conflicting intents is this FIFO greedy
+// one).  Intents are numbered in the order they are handled, which is that
+// order, and only the head of a pair's queue can start (the rest share its
+// endpoints), so the arbiter repeatedly takes the smallest head number over
+// the pairs whose endpoints and link are free: lane a scans the pairs out of
+// accelerator a, a warp minimum picks the winner.  A started transfer
+// allocates its receive buffer and lasts the transfer estimate.
+//
+// Readiness: an op's inputs are counted as they become present -- a local
+// predecessor's output when that predecessor starts (its finish time is then
+// known), a remote one when its transfer is DONE -- and the op becomes READY
+// at the latest arrival once all are there.  Transfer events at a time are
+// handled before READY keys at that time (a DONE can make an op ready then).
+//
+// HBM events: an op's own copy is released once two holds are gone -- its
+// last local listed consumer has finished (or the op itself, if none) and
+// every outgoing transfer has arrived -- at the later of those times; a
+// receive copy is allocated when its transfer starts and released by its last
+// listed consumer there (or on arrival if none).  Every such event is logged
+// at a time no earlier than the sweep's, so the batched drain of the
+// pure-latency simulation applies unchanged.
+//
+// Requires at most 32 accelerators (endpoint sets are warp bit masks) and an
+// accelerator id that fits beside the packed key.  Every loop is bounded by
+// the graph: transfer events by twice the number of transfers.
+#include "gmg_arb.h"
+#include "gmgsim_sim.cuh"
+
+namespace gsim {
+namespace {
+
+// Transfer-event key: time << (ib + 6) | class << (ib + 5) | op << 5 | e.
+constexpr uint32_t kXDone = 0, kXIntent = 1;
+
+template <bool kT32, bool kTypes>
+struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
+  using Base = Sim<true, kFull, true, kT32, kTypes>;
+  using tm_t = typename Base::tm_t;
+  using Base::g;
+  using Base::P;
+  using Base::row;
+  using Base::status;
+  const ArbParams& A;
+  ReadyHeap tq;      // INTENT / DONE keys
+  int32_t* cnt;      // [N] inputs present
+  tm_t* rmax;        // [N] latest arrival among them
+  int32_t* refs;     // [N] holds left on the op's own copy (its time: Base::holdb)
+  uint32_t* xent;    // [xcap] intent: producer << 5 | destination
+  int32_t* xnext;    // [xcap]
+  int32_t* qhead;    // [D*D]
+  int32_t* qtail;    // [D*D]
+  uint32_t* lbits;   // shared [32]: busy links
+  int32_t nx;        // intents queued so far
+  int32_t xev;       // transfer events handled (loop guard)
+  uint32_t sendm, recvm;  // accelerators whose sending / receiving endpoint is busy
+  uint32_t pm;       // lane a: destinations with a pending intent from a
+  bool arb_due;
+  tm_t t_arb;
+
+  __device__ ArbSim(const ArbParams& a) : Base(a.P), A(a) {}
+
+  __device__ __forceinline__ uint64_t xkey(tm_t t, uint32_t cls, uint32_t op, int e) const {
+    using U = typename std::make_unsigned<tm_t>::type;
+    return ((uint64_t)(U)t << (g.ib + 6)) | ((uint64_t)cls << (g.ib + 5)) | ((uint64_t)op << 5) | (uint64_t)e;
+  }
+  __device__ __forceinline__ tm_t xtime(uint64_t k) const { return (tm_t)(k >> (g.ib + 6)); }
+
+  __device__ void setup_arb(int64_t slot, uint8_t* sm) {
+    uint8_t* sl = P.scratch + slot * P.slot_bytes;
+    tq.sk = reinterpret_cast<uint64_t*>(sm);
+    tq.gk = reinterpret_cast<uint64_t*>(sl + A.off_tq);
+    tq.qs = A.tqs;
+    tq.cap = A.tqcap;
+    tq.size = 0;
+    lbits = reinterpret_cast<uint32_t*>(sm + 8 * (size_t)A.tqs);
+    cnt = reinterpret_cast<int32_t*>(sl + A.off_cnt);
+    rmax = reinterpret_cast<tm_t*>(sl + A.off_rmax);
+    refs = reinterpret_cast<int32_t*>(sl + A.off_refs);
+    xent = reinterpret_cast<uint32_t*>(sl + A.off_xent);
+    xnext = reinterpret_cast<int32_t*>(sl + A.off_xnext);
+    qhead = reinterpret_cast<int32_t*>(sl + A.off_qhead);
+    qtail = reinterpret_cast<int32_t*>(sl + A.off_qtail);
+  }
+
+  __device__ void reset_arb() {
+    const unsigned lane = lane_id();
+    this->reset_common();
+    uint4* c4 = reinterpret_cast<uint4*>(cnt);
+    const int nv = (int)((4 * (size_t)g.n + 15) / 16);
+    for (int x = lane; x < nv; x += 32) c4[x] = make_uint4(0u, 0u, 0u, 0u);
+    for (int x = lane; x < g.D * g.D; x += 32) {
+      qhead[x] = -1;
+      qtail[x] = -1;
+    }
+    lbits[lane] = 0u;
+    tq.size = 0;
+    nx = 0;
+    xev = 0;
+    sendm = recvm = pm = 0u;
+    arb_due = false;
+    t_arb = 0;
+    __syncwarp();
+  }
+
+  // One more input of op j present at time a (per lane); true if it was the
+  // last, with its ready time in rj.
+  __device__ __forceinline__ bool add_input(uint32_t j, tm_t a, tm_t& rj) const {
+    const int32_t c = cnt[j] + 1;
+    cnt[j] = c;
+    const tm_t m = c == 1 ? a : (rmax[j] > a ? rmax[j] : a);
+    rmax[j] = m;
+    const RelPred jp = op_relpred(g.ops, j);
+    if ((uint32_t)c != jp.npred) return false;
+    const tm_t rel = (tm_t)jp.rel;
+    rj = rel > m ? rel : m;
+    return true;
+  }
+
+  __device__ __forceinline__ void push_readies(bool rdy, tm_t rj, uint32_t j) {
+    uint32_t m = __ballot_sync(kFullMask, rdy);
+    while (m) {
+      const int src = __ffs(m) - 1;
+      m &= m - 1;
+      this->push_ready(__shfl_sync(kFullMask, this->kc.make(rj, kReady, j), src));
+    }
+  }
+
+  // READY(r, i): start op i; local successors get this input, remote
+  // accelerators of successors get an intent at its finish.
+  __device__ void start_op(uint32_t i, tm_t r) {
+    const unsigned lane = lane_id();
+    const longlong2 db = op_durbytes(g.ops, i);
+    const XqSucc xs = op_xqsucc(g.ops, i);
+    const uint4 cs = op_cons(g.ops, i);
+    const int d = row[i];
+    const tm_t dur = (tm_t)this->dur_of(i, d, db.x);
+    const tm_t fd = this->dv.get_free(d);
+    const tm_t s = r > fd ? r : fd;
+    const tm_t f = s + dur;
+    this->dv.set_free(d, f);
+    if (lane == 0) {
+      this->fbuf[i] = f;
+      if (cs.w & kReqSink)
+        atomicMax(reinterpret_cast<unsigned long long*>(this->creq + (int32_t)cs.z), (unsigned long long)f);
+      this->oplog[this->opn] = i;
+    }
+    ++this->opn;
+    if (cs.w & kScored) this->score += (int64_t)f;
+    __syncwarp();
+    uint32_t remote = 0u;
+    for (uint32_t c0 = 0; c0 < xs.nsucc; c0 += 32) {
+      const uint32_t t = c0 + lane;
+      uint32_t j = 0;
+      tm_t rj = 0;
+      bool rdy = false;
+      if (t < xs.nsucc) {
+        j = __ldg(g.succ + xs.succ_off + t);
+        const int dj = row[j];
+        if (dj == d) rdy = add_input(j, f, rj);
+        else remote |= 1u << dj;
+      }
+      push_readies(rdy, rj, j);
+    }
+    __syncwarp();
+    remote = __reduce_or_sync(kFullMask, remote);
+    if (lane == 0) {
+      refs[i] = 1 + __popc(remote);
+      this->holdb[i] = f;
+    }
+    __syncwarp();
+    while (remote) {
+      const int e = __ffs(remote) - 1;
+      remote &= remote - 1;
+      if (!tq.push(xkey(f, kXIntent, i, e))) status = GMG_SIM_QUEUE;
+    }
+  }
+
+  // One hold on op p's own copy (on accelerator dp) ends at time v (per
+  // lane; `want`: this lane releases one).  Logs the copy's release when it
+  // was the last hold.
+  __device__ __forceinline__ void drop_hold(bool want, uint32_t p, tm_t v, int dp) {
+    bool last = false;
+    tm_t h = v;
+    if (want) {
+      const int32_t left = refs[p] - 1;
+      refs[p] = left;
+      const tm_t o = this->holdb[p];
+      h = o > v ? o : v;
+      this->holdb[p] = h;
+      last = left == 0;
+    }
+    this->log_event(last, this->kc.make(h, kFree, p), dp);
+  }
+
+  // INTENT or DONE.
+  __device__ void handle_x(uint64_t k) {
+    const unsigned lane = lane_id();
+    const uint32_t cls = (uint32_t)(k >> (g.ib + 5)) & 1u;
+    const uint32_t p = (uint32_t)(k >> 5) & this->kc.mask;
+    const int e = (int)(k & 31u);
+    const tm_t t = xtime(k);
+    const int a = row[p];
+    const int pair = a * g.D + e;
+    if (cls == kXIntent) {
+      if (nx >= A.xcap) {
+        status = GMG_SIM_QUEUE;
+        return;
+      }
+      const int32_t x = nx++;
+      if (lane == 0) {
+        xent[x] = (p << 5) | (uint32_t)e;
+        xnext[x] = -1;
+        const int32_t tl = qtail[pair];
+        if (tl >= 0) xnext[tl] = x;
+        else qhead[pair] = x;
+        qtail[pair] = x;
+      }
+      if ((int)lane == a) pm |= 1u << e;
+      __syncwarp();
+      return;
+    }
+    // DONE: free the endpoints and the link
+    sendm &= ~(1u << a);
+    recvm &= ~(1u << e);
+    const uint32_t lid = __ldg(A.link + pair);
+    if (lane == 0) lbits[lid >> 5] &= ~(1u << (lid & 31u));
+    __syncwarp();
+    // p's successors on e have this input now
+    const XqSucc xs = op_xqsucc(g.ops, p);
+    for (uint32_t c0 = 0; c0 < xs.nsucc; c0 += 32) {
+      const uint32_t u = c0 + lane;
+      uint32_t j = 0;
+      tm_t rj = 0;
+      bool rdy = false;
+      if (u < xs.nsucc) {
+        j = __ldg(g.succ + xs.succ_off + u);
+        if (row[j] == e) rdy = add_input(j, t, rj);
+      }
+      push_readies(rdy, rj, j);
+    }
+    __syncwarp();
+    // the receive copy: released on arrival if no listed consumer is on e
+    const uint4 cs = op_cons(g.ops, p);
+    bool here = (cs.w & kAllCons) != 0;  // the successors there are consumers
+    if (!here) {
+      bool f = false;
+      for (uint32_t u = lane; u < cs.y; u += 32) f |= row[__ldg(g.cons + cs.x + u)] == e;
+      here = __any_sync(kFullMask, f);
+    }
+    this->log_event(lane == 0 && !here, this->kc.make(t, kFree, p), e);
+    // the sender's copy: one hold fewer
+    drop_hold(lane == 0, p, t, a);
+  }
+
+  // Start every pending intent whose endpoints and link are free, in order.
+  __device__ void arbitrate(tm_t t) {
+    const int lane = (int)lane_id();
+    const int D = g.D;
+    while (true) {
+      uint32_t best = 0xffffffffu;
+      int be = 0;
+      if (lane < D && !((sendm >> lane) & 1u)) {
+        uint32_t c = pm & ~recvm;
+        while (c) {
+          const int e = __ffs(c) - 1;
+          c &= c - 1;
+          const uint32_t lid = __ldg(A.link + lane * D + e);
+          if ((lbits[lid >> 5] >> (lid & 31u)) & 1u) continue;
+          const uint32_t h = (uint32_t)qhead[lane * D + e];
+          if (h < best) {
+            best = h;
+            be = e;
+          }
+        }
+      }
+      const uint32_t m = __reduce_min_sync(kFullMask, best);
+      if (m == 0xffffffffu) break;
+      const int src = __ffs(__ballot_sync(kFullMask, best == m)) - 1;
+      const int e = __shfl_sync(kFullMask, be, src);
+      const uint32_t p = xent[m] >> 5;
+      const int32_t nxt = xnext[m];
+      const int pair = src * D + e;
+      const uint32_t lid = __ldg(A.link + pair);
+      __syncwarp();
+      if (lane == 0) {
+        qhead[pair] = nxt;
+        if (nxt < 0) qtail[pair] = -1;
+        lbits[lid >> 5] |= 1u << (lid & 31u);
+      }
+      if (nxt < 0 && lane == src) pm &= ~(1u << e);
+      sendm |= 1u << src;
+      recvm |= 1u << e;
+      __syncwarp();
+      const tm_t done = t + this->xfer(src, e, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
+      if (!tq.push(xkey(done, kXDone, p, e))) {
+        status = GMG_SIM_QUEUE;
+        return;
+      }
+      this->log_event(lane == 0, this->kc.make(t, kAlloc, p), e);
+    }
+  }
+
+  // HBM events of the ops started since the last generation, one op per
+  // lane: the own copy allocated at s; the op's local hold on its own copy
+  // ends at f if no listed consumer is local; every held input whose last
+  // local listed consumer this op is gets released at f (a receive copy) or
+  // loses its local hold (the producer's own copy).
+  __device__ void generate() {
+    const unsigned lane = lane_id();
+    for (int c0 = 0; c0 < this->opn; c0 += 32) {
+      const int idx = c0 + (int)lane;
+      const bool v = idx < this->opn;
+      const uint32_t x = v ? this->oplog[idx] : 0u;
+      longlong2 db = make_longlong2(0, 0);
+      uint4 ls = make_uint4(0, 0, 0, 0), cs = make_uint4(0, 0, 0, 0);
+      int d = 0;
+      tm_t f = 0;
+      if (v) {
+        db = op_durbytes(g.ops, x);
+        ls = op_lists(g.ops, x);
+        cs = op_cons(g.ops, x);
+        d = row[x];
+        f = this->fbuf[x];
+      }
+      this->log_event(v, this->kc.make(f - (tm_t)this->dur_of(x, d, db.x), kAlloc, x), d);
+      bool localc = false;
+      if (v) {
+        const bool all = (cs.w & kAllCons) != 0;
+        const uint32_t* lst = all ? g.succ + ls.x : g.cons + cs.x;
+        const uint32_t nl = all ? ls.y : cs.y;
+        for (uint32_t w = 0; w < nl; ++w)
+          if (row[__ldg(lst + w)] == d) {
+            localc = true;
+            break;
+          }
+      }
+      drop_hold(v && !localc, x, f, d);
+      __syncwarp();
+      const uint32_t npx = ls.w;
+      const uint32_t maxp = __reduce_max_sync(kFullMask, npx);
+      for (uint32_t u = 0; u < maxp; ++u) {
+        bool rel = false;
+        uint32_t p = 0;
+        if (u < npx) {
+          const uint2 ps = __ldg(g.predsib + ls.z + u);
+          p = ps.x & kIdMask;
+          if (ps.x & kHoldBit) {
+            const uint32_t sb = ps.y;
+            if (sb == kSibNone) {
+              rel = true;
+            } else if (sb != kSibMany && (sb & kSibLater)) {
+              rel = row[sb & ~kSibLater] != d;  // the other consumer finishes later
+            } else if (sb != kSibMany) {
+              const tm_t fs = this->fin(sb);
+              rel = !(row[sb] == d && !(fs != 0 && fs < f));
+            } else {
+              const XqSucc px = op_xqsucc(g.ops, p);
+              const uint4 pcs = op_cons(g.ops, p);
+              const bool all = (pcs.w & kAllCons) != 0;
+              const uint32_t* lst = all ? g.succ + px.succ_off : g.cons + pcs.x;
+              const uint32_t nl = all ? px.nsucc : pcs.y;
+              rel = true;
+              for (uint32_t w = 0; w < nl; ++w) {
+                const uint32_t c = __ldg(lst + w);
+                const tm_t fc = c != x ? this->fin(c) : 0;
+                if (c != x && row[c] == d && !(fc != 0 && fc < f)) {
+                  rel = false;
+                  break;
+                }
+              }
+            }
+          }
+        }
+        const bool own = rel && row[p] == d;
+        this->log_event(rel && !own, this->kc.make(f, kFree, p), d);
+        drop_hold(own, p, f, d);
+      }
+    }
+    this->opn = 0;
+    __syncwarp();
+  }
+
+  __device__ void drain(int64_t t_next) {
+    generate();
+    this->opn = 0;  // generate() emptied the op log; the base drain's own call is then a no-op
+    Base::drain(t_next);
+  }
+
+  // The event loop: transfer events, then the arbiter once the last event of
+  // a time is handled, then READY keys.
+  __device__ void run() {
+    if (status) return;
+    const int32_t xlim = 2 * A.xcap + 2;
+    while (true) {
+      const uint64_t tk = tq.top();
+      if (arb_due && (tk == kKeyMax || xtime(tk) > t_arb)) {
+        arbitrate(t_arb);
+        arb_due = false;
+        if (status) break;
+        continue;
+      }
+      const uint64_t top = this->q.top();
+      const uint64_t rm = warp_min_u64(this->rk_reg);
+      const uint64_t rk = this->rkey;
+      uint64_t nk = rk < top ? rk : top;
+      nk = rm < nk ? rm : nk;
+      if (tk != kKeyMax && (nk == kKeyMax || (int64_t)xtime(tk) <= this->kc.time(nk))) {
+        if (++xev > xlim) {
+          status = GMG_SIM_LOOP;
+          break;
+        }
+        __syncwarp();
+        tq.pop();
+        handle_x(tk);
+        arb_due = true;
+        t_arb = xtime(tk);
+        if (status) break;
+        continue;
+      }
+      if (nk == kKeyMax) break;
+      if (this->opn >= P.opcap) drain(this->kc.time(nk));
+      if (nk == rm) {
+        if (this->rk_reg == rm) this->rk_reg = kKeyMax;
+      } else if (nk == rk) {
+        ++this->rootptr;
+        this->load_root();
+      } else {
+        __syncwarp();
+        this->q.pop();
+      }
+      if (++this->iters > (int32_t)g.max_iter) {
+        status = GMG_SIM_LOOP;
+        break;
+      }
+      start_op(this->kc.op(nk), (tm_t)this->kc.time(nk));
+      if (status) break;
+    }
+    if (!status) drain(kI64Max);
+  }
+};
+
+template <bool kT32, bool kTypes>
+__global__ void __launch_bounds__(128) sim_arb_kernel(const __grid_constant__ ArbParams A) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const unsigned wib = threadIdx.x >> 5;
+  const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
+  const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
+  ArbSim<kT32, kTypes> S(A);
+  setup_slot(S, A.P, wib, slot, smem);
+  S.setup_arb(slot, smem + A.smem_std + (size_t)wib * A.smem_arb);
+  for (int64_t k = slot; k < A.P.K; k += nslots) {
+    S.row = A.P.place + k * A.P.ld;
+    if (S.row_has_bad_device(S.row)) {
+      S.write_invalid(k, GMG_SIM_BADDEV);
+      continue;
+    }
+    S.reset_arb();
+    S.run();
+    S.finish(k);
+  }
+}
+
+}  // namespace
+
+const void* arb_kernel_ptr(bool t32, bool types) {
+  if (t32) return types ? (const void*)sim_arb_kernel<true, true> : (const void*)sim_arb_kernel<true, false>;
+  return types ? (const void*)sim_arb_kernel<false, true> : (const void*)sim_arb_kernel<false, false>;
+}
+
+cudaError_t launch_arb(bool t32, bool types, const ArbParams& A, int grid, int block, size_t smem,
+                       cudaStream_t st) {
+  void* args[] = {const_cast<ArbParams*>(&A)};
+  return cudaLaunchKernel(arb_kernel_ptr(t32, types), dim3(grid), dim3(block), args, smem, st);
+}
+
+}  // namespace gsim

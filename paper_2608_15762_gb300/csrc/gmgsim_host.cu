@@ -11,6 +11,7 @@
 #include <vector>
 
 #include "gmg_access.h"
+#include "gmg_arb.h"
 
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
@@ -34,6 +35,7 @@ constexpr int64_t kI64Max = 0x7fffffffffffffffll;
 constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
 constexpr int kDefaultWarpsPerBlock = 4;
 constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
+constexpr int kSharedXferEntries = 33;   // transfer-event heap: the root and its children
 constexpr int64_t kDefaultQueueCap = 1 << 16;
 constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
@@ -48,7 +50,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
   size_t off_ops, off_succ, off_pred, off_sib, off_cons, off_roots, off_cap, off_base, off_avail,
-      off_dl, off_links, off_durt, off_dtype, total;
+      off_dl, off_links, off_durt, off_dtype, off_linkid, total;
 };
 
 // Everything gmg_create derives from a description.
@@ -63,6 +65,8 @@ struct Built {
   std::vector<LinkRec> links;
   std::vector<int64_t> durt;  // [n*T] when T >= 2
   std::vector<uint8_t> dtype; // [D] when T >= 2
+  std::vector<uint16_t> linkid;  // [D*D] when D <= 32: communication link of each ordered pair
+  int64_t xfer_bound = 0;     // transfers of one placement at most: sum of min(successors, D-1)
   Layout L{};
 };
 
@@ -106,6 +110,7 @@ void plan(Built& b) {
   L.off_links = take(b.uniform ? 0 : sizeof(LinkRec) * (size_t)b.D * b.D);
   L.off_durt = take(8 * b.durt.size());
   L.off_dtype = take(b.dtype.size());
+  L.off_linkid = take(2 * b.linkid.size());
   L.total = o;
 }
 
@@ -343,6 +348,20 @@ int build(const gmg_desc_t* d, Built& b) {
                    : make_link(d->bw_B_per_us[(size_t)s * D + e], d->lat_us[(size_t)s * D + e]);
   }
   for (int i = 0; i < n; ++i) b.ops[i].xq = host_ceil(b.ops[i].bytes, b.bw0);
+  // communication links of the arbitrated transfers (kept for <= 32 accelerators)
+  for (int s = 0; s < D; ++s)
+    for (int e = 0; e < D; ++e) {
+      const size_t k = (size_t)s * D + e;
+      const int64_t id = d->link_id ? d->link_id[k] : (int64_t)k;
+      if (s != e && (id < 0 || id >= (int64_t)D * D)) return GMG_EINVAL;
+    }
+  if (D <= 32) {
+    b.linkid.resize((size_t)D * D);
+    for (size_t k = 0; k < b.linkid.size(); ++k) {
+      const bool diag = k / D == k % D;
+      b.linkid[k] = (uint16_t)(d->link_id && !diag ? d->link_id[k] : (int32_t)k);
+    }
+  }
   // Bounds: every time <= start + all durations + one transfer per edge and
   // per op; it must fit the packed key (61 - ib bits); scores and byte totals
   // must fit int64.
@@ -363,6 +382,7 @@ int build(const gmg_desc_t* d, Built& b) {
     iters += 1;
     qb += r.npred ? 1 : 0;
     lb += 2 + 2 * i128(copies);
+    b.xfer_bound += copies;
     if (t >= tlim || mem >= (i128(1) << 62)) return GMG_ERANGE;
   }
   if (t * i128(std::max(n, 1)) >= (i128(1) << 62)) return GMG_ERANGE;
@@ -394,6 +414,8 @@ struct gmg {
   gmg_info_t info;
   int64_t queue_bound;
   int64_t log_bound;
+  const uint16_t* linkid;  // device [D*D] (NULL above 32 accelerators)
+  int64_t xfer_bound;
 };
 
 const DevGmg* gsim::gmg_device_graph(const gmg_t* g) { return g ? &g->dg : nullptr; }
@@ -501,11 +523,16 @@ int check_out(const sim_out_t* o, const sim_opts_t* opts) {
   if (opts && opts->n_trace < 0) return GMG_EINVAL;
   if (opts && opts->n_trace > 0 && (!opts->d_trace_k || !o->trace_start || !o->trace_finish))
     return GMG_EINVAL;
-  if (opts)
+  if (opts) {
     for (int r : opts->reserved)
       if (r != 0) return GMG_EINVAL;
+    if (opts->transfer_mode != GMG_TRANSFER_LATENCY && opts->transfer_mode != GMG_TRANSFER_ARBITRATED)
+      return GMG_EINVAL;
+  }
   return GMG_OK;
 }
+
+bool arbitrated(const sim_opts_t* o) { return o && o->transfer_mode == GMG_TRANSFER_ARBITRATED; }
 
 void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
   P.out.makespan = o->makespan;
@@ -523,6 +550,61 @@ void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
   P.out.trace_finish = o->trace_finish;
   P.n_trace = opts ? opts->n_trace : 0;
   P.trace_k = opts ? opts->d_trace_k : nullptr;
+}
+
+// Arbitrated transfers: the full simulation's slot plus the transfer state.
+// At most 32 accelerators (endpoint sets are bit masks, link ids < 1024),
+// op ids below 2^27 (an intent packs op << 5 | destination) and accelerator
+// ids that fit beside the packed key (the transfer-event key is 4 bits wider).
+int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams& A) {
+  const DevGmg& G = g->dg;
+  if (G.D > 32 || !g->linkid) return GMG_EINVAL;
+  if (!G.dev_key || G.n >= (1 << 27)) return GMG_ERANGE;
+  const int64_t xcap = std::max<int64_t>(g->xfer_bound, 1);
+  if (xcap > (int64_t(1) << 29)) return GMG_ERANGE;
+  int rc = plan_launch(g, K, o, false, L);
+  if (rc) return rc;
+  std::memset(&A, 0, sizeof(A));
+  SimParams& P = L.P;
+  size_t o2 = (size_t)P.slot_bytes;
+  auto take = [&](size_t bytes) {
+    const size_t at = o2;
+    o2 = align_up(o2 + std::max<size_t>(bytes, 1), 256);
+    return (int64_t)at;
+  };
+  A.xcap = (int32_t)xcap;
+  A.tqs = kSharedXferEntries;
+  A.tqcap = (int32_t)xcap + 1;  // every transfer has at most one key queued at a time
+  const size_t n = (size_t)G.n, DD = (size_t)G.D * G.D;
+  A.off_cnt = take(4 * n);
+  A.off_rmax = take((G.t32 ? 4 : 8) * n);
+  A.off_refs = take(4 * n);
+  A.off_xent = take(4 * (size_t)xcap);
+  A.off_xnext = take(4 * (size_t)xcap);
+  A.off_qhead = take(4 * DD);
+  A.off_qtail = take(4 * DD);
+  A.off_tq = take(8 * (size_t)std::max(A.tqcap - A.tqs, 0));
+  P.slot_bytes = (int64_t)o2;
+  A.smem_arb = (int32_t)align_up(8 * (size_t)A.tqs + 128, 16);
+  A.smem_std = (int64_t)L.smem;
+  L.smem += (size_t)L.wpb * (size_t)A.smem_arb;
+  const int sms = device_sms();
+  if (sms <= 0) return GMG_ECUDA;
+  int bps = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, arb_kernel_ptr(G.t32 != 0, G.ntypes >= 2), 32 * L.wpb,
+                                                    L.smem) != cudaSuccess)
+    return GMG_ECUDA;
+  bps = std::max(bps, 1);
+  const int64_t need = (std::max<int64_t>(K, 1) + L.wpb - 1) / L.wpb;
+  L.grid = (int)std::min<int64_t>(need, (int64_t)sms * bps);
+  L.slots = (int64_t)L.grid * L.wpb;
+  A.link = g->linkid;
+  return GMG_OK;
+}
+
+cudaError_t launch_arb_batch(const gmg* g, Launch& L, ArbParams& A, cudaStream_t st) {
+  A.P = L.P;
+  return launch_arb(g->dg.t32 != 0, g->dg.ntypes >= 2, A, L.grid, 32 * L.wpb, L.smem, st);
 }
 
 struct BasePlan {
@@ -618,6 +700,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
     put(L.off_durt, b.durt.data(), 8 * b.durt.size());
     put(L.off_dtype, b.dtype.data(), b.dtype.size());
   }
+  put(L.off_linkid, b.linkid.data(), 2 * b.linkid.size());
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemcpyAsync(d_ws, host.data(), b.L.total, cudaMemcpyHostToDevice, st) != cudaSuccess)
     return GMG_ECUDA;
@@ -667,6 +750,8 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   I.time_bound = b.time_bound;
   g->queue_bound = b.queue_bound;
   g->log_bound = b.log_bound;
+  g->linkid = b.linkid.empty() ? nullptr : reinterpret_cast<const uint16_t*>(w + L.off_linkid);
+  g->xfer_bound = b.xfer_bound;
   I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
   *out = g;
   return GMG_OK;
@@ -683,7 +768,12 @@ int gmg_get_info(const gmg_t* g, gmg_info_t* info) {
 size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
   if (!g || K < 0) return 0;
   Launch L;
-  if (plan_launch(g, K, opts, false, L)) return 0;
+  if (arbitrated(opts)) {
+    ArbParams A;
+    if (plan_arb(g, K, opts, L, A)) return 0;
+  } else if (plan_launch(g, K, opts, false, L)) {
+    return 0;
+  }
   return (size_t)L.slots * (size_t)L.P.slot_bytes;
 }
 
@@ -695,7 +785,9 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   if (K == 0) return GMG_OK;
   if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
   Launch L;
-  rc = plan_launch(g, K, opts, false, L);
+  ArbParams A;
+  const bool arb = arbitrated(opts);
+  rc = arb ? plan_arb(g, K, opts, L, A) : plan_launch(g, K, opts, false, L);
   if (rc) return rc;
   if (!d_scratch || !aligned(d_scratch, 256) ||
       scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
@@ -706,7 +798,8 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   P.ld = ld;
   P.K = K;
   P.scratch = static_cast<uint8_t*>(d_scratch);
-  cudaError_t e = launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
+  const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = arb ? launch_arb_batch(g, L, A, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 
@@ -757,7 +850,9 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   if (K == 0) return GMG_OK;
   if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
   Launch L;
-  rc = plan_launch(g, K, opts, false, L);
+  ArbParams A;
+  const bool arb = arbitrated(opts);
+  rc = arb ? plan_arb(g, K, opts, L, A) : plan_launch(g, K, opts, false, L);
   if (rc) return rc;
   // As many warp slots as the fixed buffer holds (each warp then takes more
   // candidates in turn); a graph whose single slot does not fit is refused.
@@ -766,7 +861,7 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   if (fit < L.wpb) {
     sim_opts_t one = opts ? *opts : sim_opts_t{};
     one.warps_per_block = 1;
-    rc = plan_launch(g, K, &one, false, L);
+    rc = arb ? plan_arb(g, K, &one, L, A) : plan_launch(g, K, &one, false, L);
     if (rc) return rc;
   }
   L.grid = (int)std::min<int64_t>(L.grid, fit / L.wpb);
@@ -779,12 +874,13 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   P.ld = ld;
   P.K = K;
   P.scratch = scratch;
-  const cudaError_t e = launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
+  const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+  const cudaError_t e = arb ? launch_arb_batch(g, L, A, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 
 size_t base_workspace_bytes(const gmg_t* g, const sim_opts_t* opts) {
-  if (!g) return 0;
+  if (!g || arbitrated(opts)) return 0;
   BasePlan B;
   if (plan_base(g, opts, B)) return 0;
   return B.total;
@@ -795,9 +891,11 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   if (!out) return GMG_EINVAL;
   *out = nullptr;
   if (!g || !d_base_place || !aligned(d_base_place, 16)) return GMG_EINVAL;
-  if (opts)
+  if (opts) {
     for (int r : opts->reserved)
       if (r != 0) return GMG_EINVAL;
+    if (opts->transfer_mode != GMG_TRANSFER_LATENCY) return GMG_EINVAL;  // no resume points for the arbiter
+  }
   BasePlan B;
   int rc = plan_base(g, opts, B);
   if (rc) return rc;
@@ -847,7 +945,7 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
 void base_destroy(gmg_base_t* b) { delete b; }
 
 size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
-  if (!g || K < 0) return 0;
+  if (!g || K < 0 || arbitrated(opts)) return 0;
   Launch L;
   if (plan_launch(g, K, opts, true, L)) return 0;
   return (size_t)L.slots * (size_t)L.P.slot_bytes;
@@ -856,7 +954,7 @@ size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
 int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_off, const int32_t* d_move_op,
                     const uint8_t* d_move_dev, int32_t K, const sim_opts_t* opts, const sim_out_t* d_out,
                     void* d_scratch, size_t scratch_bytes, gmg_stream_t stream) {
-  if (!g || !b || b->g != g || K < 0) return GMG_EINVAL;
+  if (!g || !b || b->g != g || K < 0 || arbitrated(opts)) return GMG_EINVAL;
   int rc = check_out(d_out, opts);
   if (rc) return rc;
   if (K == 0) return GMG_OK;

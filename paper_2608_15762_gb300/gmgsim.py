@@ -20,6 +20,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 LIB_PATH = os.path.join(HERE, "libgmgsim.so")
 
 GMG_OK, GMG_EINVAL, GMG_ENOTTOPO, GMG_ERANGE, GMG_EWS, GMG_ECUDA, GMG_ENOMEM = 0, -1, -2, -3, -4, -5, -6
+GMG_TRANSFER_LATENCY, GMG_TRANSFER_ARBITRATED = 0, 1
 SIM_OK, SIM_BADDEV, SIM_MOVE_RANGE, SIM_MOVE_DUP, SIM_BADBASE, SIM_QUEUE, SIM_LOOP = range(7)
 
 EXPORTED = ("gmg_workspace_bytes", "gmg_create", "gmg_destroy", "gmg_get_info", "sim_scratch_bytes",
@@ -43,13 +44,14 @@ class _Desc(C.Structure):
                     "pred_off", "pred_idx", "cons_off", "cons_idx", "dur_us", "out_bytes",
                     "release_us", "req_id", "scored", "deadline_us", "cap_bytes", "base_bytes",
                     "avail0_us", "bw_B_per_us", "lat_us")] + [
-        ("n_types", C.c_int32), ("dev_type", C.c_void_p), ("dur_by_type", C.c_void_p)]
+        ("n_types", C.c_int32), ("dev_type", C.c_void_p), ("dur_by_type", C.c_void_p),
+        ("link_id", C.c_void_p)]
 
 
 class _Opts(C.Structure):
     _fields_ = [("score_mode", C.c_int32), ("n_trace", C.c_int32), ("d_trace_k", C.c_void_p),
                 ("queue_cap", C.c_int32), ("warps_per_block", C.c_int32),
-                ("reserved", C.c_int32 * 4)]
+                ("transfer_mode", C.c_int32), ("reserved", C.c_int32 * 3)]
 
 
 class _Out(C.Structure):
@@ -135,7 +137,7 @@ class _DescHolder:
                        _np_ptr(d.cons_off), _np_ptr(d.cons_idx), _np_ptr(d.dur), _np_ptr(d.out_bytes),
                        _np_ptr(d.release), _np_ptr(d.req_id), _np_ptr(d.scored), _np_ptr(d.deadline),
                        _np_ptr(d.cap), _np_ptr(d.base), _np_ptr(d.avail0), _np_ptr(d.bw), _np_ptr(d.lat),
-                       d.n_types, _np_ptr(d.dev_type), _np_ptr(d.dur_by_type))
+                       d.n_types, _np_ptr(d.dev_type), _np_ptr(d.dur_by_type), _np_ptr(d.link_id))
 
 
 def gmg_workspace_bytes(desc) -> int:
@@ -143,8 +145,9 @@ def gmg_workspace_bytes(desc) -> int:
     return int(lib().gmg_workspace_bytes(C.addressof(h.c)))
 
 
-def _opts(score_mode=0, trace_k=None, queue_cap=0, warps_per_block=0) -> _Opts:
+def _opts(score_mode=0, trace_k=None, queue_cap=0, warps_per_block=0, arbitrated=False) -> _Opts:
     o = _Opts()
+    o.transfer_mode = GMG_TRANSFER_ARBITRATED if arbitrated else GMG_TRANSFER_LATENCY
     o.score_mode = score_mode
     o.n_trace = 0 if trace_k is None else int(trace_k.numel())
     o.d_trace_k = None if trace_k is None else trace_k.data_ptr()
@@ -288,15 +291,17 @@ class Scratch:
 
 
 def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scratch] = None,
-              req_done=False, trace_k=None, queue_cap=0, warps_per_block=0, stream=None) -> SimOut:
-    """Simulate every row of ``place`` (CUDA uint8 [K, ld], ld % 16 == 0)."""
+              req_done=False, trace_k=None, queue_cap=0, warps_per_block=0, stream=None,
+              arbitrated=False) -> SimOut:
+    """Simulate every row of ``place`` (CUDA uint8 [K, ld], ld % 16 == 0);
+    ``arbitrated``: transfers go through the arbiter of Sec. 3.5.2."""
     import torch
     assert place.dtype == torch.uint8 and place.dim() == 2 and place.is_contiguous()
     K, ld = place.shape
     n_trace = 0 if trace_k is None else int(trace_k.numel())
     if out is None:
         out = SimOut.empty(K, g.n_dev, g.n_req, place.device, req_done, n_trace, g.n_ops)
-    o = _opts(0, trace_k, queue_cap, warps_per_block)
+    o = _opts(0, trace_k, queue_cap, warps_per_block, arbitrated)
     need = lib().sim_scratch_bytes(g.handle, K, C.addressof(o))
     scratch = scratch or Scratch(place.device)
     buf = scratch.get(need)
@@ -309,7 +314,7 @@ def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scr
 
 
 def sim_batch_noalloc(g: Gmg, place, out: Optional[SimOut] = None, req_done=False, trace_k=None,
-                      stream=None) -> SimOut:
+                      stream=None, arbitrated=False) -> SimOut:
     """Like sim_batch, but the library supplies the scratch from its own fixed
     device buffer (for callers that cannot allocate device memory)."""
     import torch
@@ -318,7 +323,7 @@ def sim_batch_noalloc(g: Gmg, place, out: Optional[SimOut] = None, req_done=Fals
     n_trace = 0 if trace_k is None else int(trace_k.numel())
     if out is None:
         out = SimOut.empty(K, g.n_dev, g.n_req, place.device, req_done, n_trace, g.n_ops)
-    o = _opts(0, trace_k)
+    o = _opts(0, trace_k, arbitrated=arbitrated)
     co = out._c()
     rc = lib().sim_batch_noalloc(g.handle, place.data_ptr(), K, ld, C.addressof(o), C.addressof(co),
                                  _stream_handle(stream))

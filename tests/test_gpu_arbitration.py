@@ -1,0 +1,200 @@
+"""GPU parity of the arbitrated-transfer simulation (sim_batch with
+transfer_mode = GMG_TRANSFER_ARBITRATED, Sec. 3.5.2) against the oracle's
+arbitrated mode, bit for bit on every output field and on the traced
+schedules: random graphs with shared links, zero-length transfers, 32- and
+64-bit times, accelerator types, the hand-worked conflict cases, the
+prefill, incremental-shaped and heterogeneous workloads, and the refusals."""
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+
+from gpu_common import compare, torch_place  # noqa: E402
+from helpers import mk  # noqa: E402
+from oracle import oracle as O  # noqa: E402
+from paper_2608_15762_gb300 import gmgsim as G  # noqa: E402
+from paper_2608_15762_gb300 import workloads as W  # noqa: E402
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2608_15762_gb300 import build
+    build.build()
+    assert torch.cuda.is_available()
+
+
+def _links(kind, D, g):
+    if kind == "pair":          # one link per unordered pair (both directions share it)
+        a, b = np.meshgrid(np.arange(D), np.arange(D), indexing="ij")
+        return (np.minimum(a, b) * D + np.maximum(a, b)).astype(np.int32).reshape(-1)
+    if kind == "uplink":        # accelerators 2m and 2m+1 share one uplink
+        return np.repeat(np.arange(D, dtype=np.int32) // 2 * D, D)
+    if kind == "random":
+        return g.integers(0, max(D * D // 3, 1), D * D).astype(np.int32)
+    return None
+
+
+def _case(seed, n, D, links=None, K=37, zero=False, **kw):
+    d = W.random_desc(seed, n, D, **kw)
+    g = np.random.default_rng(seed)
+    d.link_id = _links(links, D, g)
+    if zero:
+        d.out_bytes[::2] = 0
+        d.lat[:] = 0
+    ld = W.placement_ld(n)
+    rows = np.zeros((K, ld), np.uint8)
+    rows[:, :n] = g.integers(0, D, (K, n))
+    return d, rows
+
+
+def _run_and_compare(d, rows, trace=(0,)):
+    g = G.gmg_create(d)
+    K = rows.shape[0]
+    tk = torch.tensor(list(trace), dtype=torch.int32, device="cuda")
+    out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk, arbitrated=True)
+    best = G.select_best(out)
+    torch.cuda.synchronize()
+    got = out.to_numpy()
+    s, pk, rq = O.simulate_batch(d, rows, arbitrated=True)
+    compare(got, s, pk, rq)
+    for slot, k in enumerate(trace):
+        r = O.simulate(d, rows[k], arbitrated=True)
+        assert np.array_equal(got["trace_start"][slot], r["start"]), k
+        assert np.array_equal(got["trace_finish"][slot], r["finish"]), k
+    assert best.cpu().tolist() == list(O.select_best(s, 0))
+    return got, s
+
+
+@pytest.mark.parametrize("seed,n,D,links,kw", [
+    (1, 1, 1, None, {}),
+    (2, 9, 2, None, {}),
+    (3, 40, 3, "pair", dict(explicit_cons=True)),
+    (4, 64, 4, "uplink", dict(link_hetero=False)),
+    (5, 150, 8, None, dict(explicit_cons=True, dur_hi=2000)),
+    (6, 257, 5, "random", dict(max_pred=6)),
+    (7, 300, 32, "pair", dict(explicit_cons=True)),
+    (8, 1000, 16, "uplink", dict(edge_p=0.9, max_pred=4)),
+    (9, 90, 6, None, dict(with_release=False, with_avail0=False, cap=1 << 40)),
+    (10, 300, 8, "random", dict(dur_hi=1 << 32)),      # 64-bit times
+    (12, 300, 8, "pair", dict(n_types=2)),
+    (13, 200, 32, "random", dict(n_types=3, explicit_cons=True)),
+    (14, 150, 4, None, dict(n_types=2, dur_hi=1 << 32)),
+    (15, 400, 7, "uplink", dict(bytes_hi=1 << 20, explicit_cons=True)),
+])
+def test_random_dags_bit_exact(seed, n, D, links, kw):
+    d, rows = _case(seed, n, D, links, **kw)
+    _run_and_compare(d, rows, trace=(0, 5, rows.shape[0] - 1) if rows.shape[0] > 5 else (0,))
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_zero_length_transfers(seed):
+    d, rows = _case(40 + seed, 120, 6, "pair" if seed % 2 else None, zero=True, dur_hi=9)
+    _run_and_compare(d, rows, trace=(0, 1, 2))
+
+
+def test_hand_worked_conflicts():
+    cases = [
+        (mk([[], [0], [0]], [4, 1, 1], out_bytes=[10, 0, 0], n_dev=3, bw=1, lat=0), [0, 1, 2]),
+        (mk([[], [], [0, 1]], [3, 3, 2], out_bytes=[5, 7, 0], n_dev=3, bw=1, lat=0), [0, 1, 2]),
+        (mk([[], [], [], [0], [1], [2]], [1] * 6, out_bytes=[100, 5, 5, 0, 0, 0], n_dev=4, bw=1, lat=0),
+         [0, 2, 2, 1, 1, 3]),
+        (mk([[], [], [0], [1]], [1, 1, 1, 1], out_bytes=[10, 10, 0, 0], n_dev=2, bw=1, lat=0,
+            cons=[[], [3], [], []], cap=[19, 15]), [0, 0, 1, 1]),
+    ]
+    link = mk([[], [], [0], [1]], [2, 2, 1, 1], out_bytes=[6, 6, 0, 0], n_dev=2, bw=1, lat=0)
+    link.link_id = np.array([0, 1, 1, 0], np.int32)
+    cases.append((link, [0, 1, 1, 0]))
+    for d, place in cases:
+        rows = np.zeros((3, 16), np.uint8)
+        rows[:, :len(place)] = place
+        rows[1, :len(place)] = [(x + 1) % d.n_dev for x in place]
+        _run_and_compare(d, rows, trace=(0, 1, 2))
+
+
+@pytest.mark.parametrize("cfg", [2, 6])
+def test_workloads_every_candidate(cfg):
+    """The prefill (8 requests x 32 layers, 8 accelerators) and
+    heterogeneous-prefill workloads, all 4,096 candidates, arbitrated."""
+    wl = W.make_workload(cfg)
+    rows = wl.all_full_rows()
+    g = G.gmg_create(wl.desc)
+    out = G.sim_batch(g, torch_place(rows), arbitrated=True)
+    torch.cuda.synchronize()
+    s, pk, rq = O.simulate_batch(wl.desc, rows, arbitrated=True)
+    compare(out.to_numpy(), s, pk)
+    assert (s["status"] == 0).all()
+
+
+def test_incremental_workload_graph_all_candidates():
+    """The 32 x 32-layer graph on 16 accelerators, its base placement with
+    each candidate's moves applied, arbitrated as full placements."""
+    wl = W.make_workload(3)
+    K = wl.moves.off.shape[0] - 1
+    rows = np.zeros((K, wl.ld), np.uint8)
+    rows[:, :wl.desc.n_ops] = wl.base_place[:wl.desc.n_ops]
+    for k in range(K):
+        a, b = wl.moves.off[k], wl.moves.off[k + 1]
+        rows[k, wl.moves.op[a:b]] = wl.moves.dev[a:b]
+    g = G.gmg_create(wl.desc)
+    out = G.sim_batch(g, torch_place(rows), arbitrated=True)
+    torch.cuda.synchronize()
+    s, pk, _ = O.simulate_batch(wl.desc, rows, arbitrated=True)
+    compare(out.to_numpy(), s, pk)
+
+
+def test_noalloc_equals_scratch_path():
+    d, rows = _case(60, 300, 8, "pair")
+    g = G.gmg_create(d)
+    a = G.sim_batch(g, torch_place(rows), arbitrated=True)
+    b = G.sim_batch_noalloc(g, torch_place(rows), arbitrated=True)
+    torch.cuda.synchronize()
+    ga, gb = a.to_numpy(), b.to_numpy()
+    for k in ga:
+        if ga[k] is not None:
+            assert np.array_equal(ga[k], gb[k]), k
+
+
+def test_degenerate_inputs_and_refusals():
+    # bad device ids, a queue too small, an empty graph
+    d, rows = _case(70, 60, 4, None)
+    rows[3, 17] = 4
+    g = G.gmg_create(d)
+    out = G.sim_batch(g, torch_place(rows), arbitrated=True)
+    torch.cuda.synchronize()
+    s, pk, _ = O.simulate_batch(d, rows, arbitrated=True)
+    compare(out.to_numpy(), s, pk)
+    assert out.to_numpy()["status"][3] == G.SIM_BADDEV
+    # a star: 120 successors ready at once overflow a 3-entry READY queue
+    n = 121
+    star = mk([[]] + [[0]] * 120, [5] * n, [1] * n, n_dev=4, bw=1, lat=1)
+    gs = G.gmg_create(star)
+    srows = np.zeros((8, 128), np.uint8)
+    srows[:, :n] = np.random.default_rng(0).integers(0, 4, (8, n))
+    small = G.sim_batch(gs, torch_place(srows), arbitrated=True, queue_cap=3)
+    full = G.sim_batch(gs, torch_place(srows), arbitrated=True)
+    torch.cuda.synchronize()
+    assert (small.to_numpy()["status"] == G.SIM_QUEUE).all()
+    s, pk, _ = O.simulate_batch(star, srows, arbitrated=True)
+    compare(full.to_numpy(), s, pk)
+    empty = mk([], [], n_dev=3)
+    ge = G.gmg_create(empty)
+    out = G.sim_batch(ge, torch_place(np.zeros((4, 16), np.uint8)), arbitrated=True)
+    torch.cuda.synchronize()
+    e = out.to_numpy()
+    assert (e["status"] == 0).all() and (e["score"] == 0).all() and (e["makespan"] == 0).all()
+    # times so wide that an accelerator id no longer fits beside the key
+    dw, rw = _case(11, 150, 4, None, dur_hi=1 << 40, link_hetero=False)
+    with pytest.raises(G.GmgError) as ei:
+        G.sim_batch(G.gmg_create(dw), torch_place(rw), arbitrated=True)
+    assert ei.value.code == G.GMG_ERANGE
+    # more than 32 accelerators, and the incremental entry points, refuse
+    d40, rows40 = _case(71, 50, 40, None)
+    with pytest.raises(G.GmgError) as ei:
+        G.sim_batch(G.gmg_create(d40), torch_place(rows40), arbitrated=True)
+    assert ei.value.code == G.GMG_EINVAL
+    o = G._opts(arbitrated=True)
+    import ctypes as C
+    assert G.lib().inc_scratch_bytes(g.handle, 4, C.addressof(o)) == 0
+    assert G.lib().base_workspace_bytes(g.handle, C.addressof(o)) == 0
