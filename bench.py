@@ -75,7 +75,7 @@ def profile_path(kernel: str, workload: str) -> str:
     return os.path.join(PROFILE_DIR, "%s_%s.txt" % (kernel, workload))
 
 
-def read_profile(path: str):
+def read_profile(path: str, extra=()):
     """Instruction and DRAM counts per candidate of the dominant kernel from
     the committed ncu summary of that kernel on this workload (captured on
     `candidates_per_launch` candidates), if it was taken on the current kernel
@@ -88,7 +88,7 @@ def read_profile(path: str):
             if ":" in line:
                 k, v = line.split(":", 1)
                 vals[k.strip()] = v.strip()
-    if vals.get("kernel_source_sha256") != kernel_hash():
+    if vals.get("kernel_source_sha256") != kernel_hash(extra):
         return None
     try:
         c = float(vals["candidates_per_launch"])
@@ -167,7 +167,10 @@ class Prepared:
     pass
 
 
-def prepare(config: int, rank: int, device, cap=None):
+ARB_SOURCES = ("gmgsim_arb.cu", "gmg_arb.h")
+
+
+def prepare(config: int, rank: int, device, cap=None, arbitrated=False):
     import numpy as np
     import torch
     from paper_2608_15762_gb300 import gmgsim as G
@@ -175,6 +178,9 @@ def prepare(config: int, rank: int, device, cap=None):
     wl = W.make_workload(config)
     p = Prepared()
     p.wl = wl
+    p.arb = arbitrated
+    if arbitrated and (wl.n_full == 0 or wl.desc.n_dev > 32):
+        raise SystemExit("--arbitrated needs a workload of full placements on at most 32 accelerators")
     p.g = G.gmg_create(wl.desc, device=device)
     p.n_full = wl.n_full
     p.n_inc = 0 if wl.moves is None else wl.moves.n_cand
@@ -215,7 +221,7 @@ def run_step(p, kernel_events=None):
     if p.n_full:
         if kernel_events:
             kernel_events[0].record()
-        G.sim_batch(p.g, p.place, out=_views(p.out, 0, p.n_full), scratch=p.scratch)
+        G.sim_batch(p.g, p.place, out=_views(p.out, 0, p.n_full), scratch=p.scratch, arbitrated=p.arb)
         if kernel_events:
             kernel_events[1].record()
         launches += 1
@@ -256,7 +262,7 @@ def h2d_bytes(p):
     return b
 
 
-def cpu_baseline(wl, min_s=10.0):
+def cpu_baseline(wl, min_s=10.0, arbitrated=False):
     """The CPU oracle as it stands on this host's cores, on a bounded sample of
     the same workload: up to ~3e8 op-events of candidates, repeated as whole
     batches until at least min_s seconds of wall time."""
@@ -268,8 +274,8 @@ def cpu_baseline(wl, min_s=10.0):
         rows = wl.full_rows(range(k))
 
         def run():
-            O.simulate_batch(wl.desc, rows, nthreads=nt)
-        what = "%d of %d full placements" % (k, wl.n_full)
+            O.simulate_batch(wl.desc, rows, nthreads=nt, arbitrated=arbitrated)
+        what = "%d of %d full placements%s" % (k, wl.n_full, ", arbitrated transfers" if arbitrated else "")
     else:
         from paper_2608_15762_gb300.workloads import Moves
         k = min(wl.moves.n_cand, budget)
@@ -305,7 +311,7 @@ def reference_arm(args):
         rows = wl.full_rows(range(k))
 
         def step():
-            O.simulate_batch(wl.desc, rows, nthreads=nt)
+            O.simulate_batch(wl.desc, rows, nthreads=nt, arbitrated=args.arbitrated)
     else:
         mv = W.Moves(wl.moves.off[:k + 1].copy(), wl.moves.op[:wl.moves.off[k]],
                      wl.moves.dev[:wl.moves.off[k]])
@@ -324,7 +330,8 @@ def reference_arm(args):
     line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.name, "candidates_per_step": k, "n_ops": wl.desc.n_ops},
+            "config": {"workload": wl.name, "candidates_per_step": k, "n_ops": wl.desc.n_ops,
+                       "transfers": "arbitrated" if args.arbitrated else "latency"},
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": nt, "kind": "oracle",
                              "sample": "%d candidates per step" % k},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -647,6 +654,8 @@ def main():
                     help="time scheduling rounds (Algorithm 1) instead of the candidate simulation")
     ap.add_argument("--estimators", action="store_true",
                     help="time the online estimators (refit, durations, links) instead of the simulation")
+    ap.add_argument("--arbitrated", action="store_true",
+                    help="arbitrated transfers (Sec. 3.5.2) instead of pure-latency ones")
     ap.add_argument("--candidates", type=int, default=None,
                     help="profiling aid: simulate only the first N candidates of each half "
                          "(the line then describes that smaller batch)")
@@ -672,7 +681,7 @@ def main():
 
     from paper_2608_15762_gb300 import build as lib_build
     lib_build.build()
-    p = prepare(args.config, rank, device, cap=args.candidates)
+    p = prepare(args.config, rank, device, cap=args.candidates, arbitrated=args.arbitrated)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
 
     def barrier():
@@ -735,7 +744,7 @@ def main():
     pk = peaks()
     # the timed kernel: the full-placement simulation if the batch has one,
     # else the incremental one
-    kern = "sim_full_kernel" if p.n_full else "sim_inc_kernel"
+    kern = ("sim_arb_kernel" if p.arb else "sim_full_kernel") if p.n_full else "sim_inc_kernel"
     kcand = p.n_full if p.n_full else p.n_inc
     out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
     if p.n_full:
@@ -746,7 +755,7 @@ def main():
     props = torch.cuda.get_device_properties(device)
     issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
     ppath = profile_path(kern, wl.name)
-    prof = read_profile(ppath)
+    prof = read_profile(ppath, ARB_SOURCES if p.arb else ())
     roof = {"bound": "alu", "unit": "Ginst/s", "peak": issue_peak,
             "peak_src": "%d SMs x 4 issue slots x %.0f MHz (%s sm_max_mhz)" % (
                 props.multi_processor_count, pk["sm_max_mhz"], pk["src"]),
@@ -763,6 +772,7 @@ def main():
         "vs_baseline": None, "dtype": "int64", "data": "synthetic",
         "ms_per_step_best": min(step_ms), "ms_per_step_median": statistics.median(step_ms),
         "config": {"workload": wl.name, "candidates": K, "n_ops": N, "n_dev": D,
+                   "transfers": "arbitrated" if p.arb else "latency",
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
                    "parallelism": "dp%d over candidates" % world},
         # full placements simulate every op; an incremental candidate re-simulates
@@ -779,7 +789,7 @@ def main():
         "best": best,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl)
+        line["cpu_baseline"] = cpu_baseline(wl, arbitrated=p.arb)
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

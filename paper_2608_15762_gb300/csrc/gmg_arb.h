@@ -13,20 +13,21 @@ namespace gsim {
 struct ArbParams {
   SimParams P;            // the full simulation's parameters (slot offsets inside P too)
   const uint16_t* link;   // [D*D] link id of each ordered accelerator pair (< D*D)
+  int32_t shared_links;   // 1 if two ordered pairs share a link id (else the sender check covers links)
   int32_t xcap;           // transfers per candidate (sum over ops of min(successors, D-1))
-  int32_t tqs;            // transfer-event heap slots in shared memory per warp (>= 33)
-  int32_t tqcap;          // transfer-event heap slots per warp
+  int32_t heads_shared;   // 1: the pair queue heads live in shared memory (D <= 16)
   int32_t smem_arb;       // shared bytes of the arbitration state per warp
   int64_t smem_std;       // shared bytes of the simulation state of all warps of a block
   // byte offsets inside a warp's scratch slot
   int64_t off_cnt;        // int32 [N]  inputs present
   int64_t off_rmax;       // time  [N]  latest input arrival so far
   int64_t off_refs;       // int32 [N]  holds left on an op's own output copy
-  int64_t off_xent;       // uint32 [xcap]  intent: producer << 5 | destination
+  int64_t off_rmask;      // uint32 [N] remote accelerators of an op's successors
+  int64_t off_nextop;     // int32 [N]  next started op of the same accelerator with remote successors
+  int64_t off_xent;       // uint32 [xcap]  arrived intent: producer << 5 | destination
   int64_t off_xnext;      // int32 [xcap]  next intent of the same pair (-1: last)
-  int64_t off_qhead;      // int32 [D*D]  first pending intent of each pair (-1: none)
+  int64_t off_qhead;      // int32 [D*D]  first pending intent of each pair (-1: none), when not shared
   int64_t off_qtail;      // int32 [D*D]
-  int64_t off_tq;         // uint64 [tqcap - tqs]  transfer-event heap beyond shared memory
 };
 
 // Kernel entry of one instance (for occupancy queries) and the launcher.

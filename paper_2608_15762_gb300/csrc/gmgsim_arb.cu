@@ -1,25 +1,33 @@
 // sim_batch with arbitrated transfers (Sec. 3.5.2, "Tensor Transfer
 // Arbitration"): one warp per candidate, as in the pure-latency simulation,
-// with a second event stream for the transfers.
+// with two more kinds of event.
 //
-//   INTENT(f_p, p, e)  producer p finished; its output is wanted on
-//                      accelerator e (one intent per distinct remote
-//                      accelerator of p's successors).  The intent joins the
-//                      FIFO queue of the pair (dev p, e).
-//   DONE(c, p, e)      the transfer arrived: e's receiving endpoint, the
-//                      sender's endpoint and the pair's link are free again;
+//   INTENT(f_p, p)     producer p finished; its output is wanted on every
+//                      distinct remote accelerator e of p's successors: one
+//                      intent per e joins the FIFO queue of the pair (dev p, e).
+//   DONE(c, p, e)      the transfer arrived: the sender's endpoint, e's
+//                      receiving endpoint and the pair's link are free again;
 //                      p's successors on e have one more input present.
+//
+// Lane a keeps accelerator a's side of both in registers.  An accelerator
+// sends one transfer at a time, so lane a holds the completion time of the
+// transfer it is sending, if any; and its ops finish in the order they start,
+// so the ops with remote successors that it has started but whose intents
+// have not arrived form a FIFO in finish order: lane a holds its head.  The
+// next DONE and the next INTENT are warp minima over the lanes (intents by
+// (time, producer)).
 //
 // After every INTENT / DONE at time t the arbiter starts, in (intent time,
 // producer, destination) order, every pending intent whose sending endpoint,
 // receiving endpoint and link are all free (the communication graph of Sec.
 // 3.5.2; the selection rule among conflicting intents is this FIFO greedy
-// one).  Intents are numbered in the order they are handled, which is that
-// order, and only the head of a pair's queue can start (the rest share its
-// endpoints), so the arbiter repeatedly takes the smallest head number over
-// the pairs whose endpoints and link are free: lane a scans the pairs out of
-// accelerator a, a warp minimum picks the winner.  A started transfer
-// allocates its receive buffer and lasts the transfer estimate.
+// one).  Intents are numbered as they arrive, which is that order, and only
+// the head of a pair's queue can start (the rest share its endpoints), so the
+// arbiter repeatedly takes the smallest head number over the pairs whose
+// endpoints and link are free: lane a scans the pairs out of accelerator a, a
+// warp minimum picks the winner.  A started transfer allocates its receive
+// buffer and lasts the transfer estimate.  When no two ordered pairs share a
+// link id, a busy link implies a busy sender and the link state is not kept.
 //
 // Readiness: an op's inputs are counted as they become present -- a local
 // predecessor's output when that predecessor starts (its finish time is then
@@ -37,81 +45,89 @@
 //
 // Requires at most 32 accelerators (endpoint sets are warp bit masks) and an
 // accelerator id that fits beside the packed key.  Every loop is bounded by
-// the graph: transfer events by twice the number of transfers.
+// the graph: DONEs by the number of transfers, INTENTs by the number of ops.
 #include "gmg_arb.h"
 #include "gmgsim_sim.cuh"
 
 namespace gsim {
 namespace {
 
-// Transfer-event key: time << (ib + 6) | class << (ib + 5) | op << 5 | e.
-constexpr uint32_t kXDone = 0, kXIntent = 1;
-
 template <bool kT32, bool kTypes>
 struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
   using Base = Sim<true, kFull, true, kT32, kTypes>;
   using tm_t = typename Base::tm_t;
+  using U = typename std::make_unsigned<tm_t>::type;
   using Base::g;
   using Base::P;
   using Base::row;
   using Base::status;
+  static constexpr tm_t kNever = (tm_t)(~(U)0 >> 1);
   const ArbParams& A;
-  ReadyHeap tq;      // INTENT / DONE keys
-  int32_t* cnt;      // [N] inputs present
-  tm_t* rmax;        // [N] latest arrival among them
-  int32_t* refs;     // [N] holds left on the op's own copy (its time: Base::holdb)
-  uint32_t* xent;    // [xcap] intent: producer << 5 | destination
-  int32_t* xnext;    // [xcap]
-  int32_t* qhead;    // [D*D]
-  int32_t* qtail;    // [D*D]
-  uint32_t* lbits;   // shared [32]: busy links
-  int32_t nx;        // intents queued so far
+  // The warp's scratch slot and shared area; the arrays in them are found
+  // from the launch parameters' offsets when used (registers are scarce).
+  uint8_t* sl;
+  uint8_t* sm;       // [0, 128): busy links (32 words); then the queue heads if shared
+  int32_t nx;        // intents arrived so far
   int32_t xev;       // transfer events handled (loop guard)
   uint32_t sendm, recvm;  // accelerators whose sending / receiving endpoint is busy
-  uint32_t pm;       // lane a: destinations with a pending intent from a
+  // lane a: accelerator a's transfer state
+  uint32_t pm;       // destinations with a pending intent from a
+  tm_t xd;           // completion of the transfer a is sending (kNever: none)
+  uint32_t xdp;      // its producer
+  int xde;           // its destination
+  int32_t fh, ft;    // FIFO of started ops with remote successors (-1: empty)
+  tm_t fa;           // finish time of the FIFO head (kNever: empty)
   bool arb_due;
   tm_t t_arb;
 
   __device__ ArbSim(const ArbParams& a) : Base(a.P), A(a) {}
 
-  __device__ __forceinline__ uint64_t xkey(tm_t t, uint32_t cls, uint32_t op, int e) const {
-    using U = typename std::make_unsigned<tm_t>::type;
-    return ((uint64_t)(U)t << (g.ib + 6)) | ((uint64_t)cls << (g.ib + 5)) | ((uint64_t)op << 5) | (uint64_t)e;
+  template <typename T>
+  __device__ __forceinline__ T* at(int64_t off) const { return reinterpret_cast<T*>(sl + off); }
+  __device__ __forceinline__ int32_t* cnt() const { return at<int32_t>(A.off_cnt); }      // [N] inputs present
+  __device__ __forceinline__ tm_t* rmax() const { return at<tm_t>(A.off_rmax); }          // [N] latest arrival
+  __device__ __forceinline__ int32_t* refs() const { return at<int32_t>(A.off_refs); }    // [N] holds left
+  __device__ __forceinline__ uint32_t* rmask() const { return at<uint32_t>(A.off_rmask); }  // [N] remote accs
+  __device__ __forceinline__ int32_t* nextop() const { return at<int32_t>(A.off_nextop); }  // [N] FIFO link
+  __device__ __forceinline__ uint32_t* xent() const { return at<uint32_t>(A.off_xent); }  // [xcap] p << 5 | e
+  __device__ __forceinline__ int32_t* xnext() const { return at<int32_t>(A.off_xnext); }  // [xcap]
+  __device__ __forceinline__ int32_t* qtail() const { return at<int32_t>(A.off_qtail); }  // [D*D]
+  __device__ __forceinline__ int32_t* qhead() const {                                      // [D*D]
+    return A.heads_shared ? reinterpret_cast<int32_t*>(sm + 128) : at<int32_t>(A.off_qhead);
   }
-  __device__ __forceinline__ tm_t xtime(uint64_t k) const { return (tm_t)(k >> (g.ib + 6)); }
+  __device__ __forceinline__ uint32_t* lbits() const { return reinterpret_cast<uint32_t*>(sm); }
 
-  __device__ void setup_arb(int64_t slot, uint8_t* sm) {
-    uint8_t* sl = P.scratch + slot * P.slot_bytes;
-    tq.sk = reinterpret_cast<uint64_t*>(sm);
-    tq.gk = reinterpret_cast<uint64_t*>(sl + A.off_tq);
-    tq.qs = A.tqs;
-    tq.cap = A.tqcap;
-    tq.size = 0;
-    lbits = reinterpret_cast<uint32_t*>(sm + 8 * (size_t)A.tqs);
-    cnt = reinterpret_cast<int32_t*>(sl + A.off_cnt);
-    rmax = reinterpret_cast<tm_t*>(sl + A.off_rmax);
-    refs = reinterpret_cast<int32_t*>(sl + A.off_refs);
-    xent = reinterpret_cast<uint32_t*>(sl + A.off_xent);
-    xnext = reinterpret_cast<int32_t*>(sl + A.off_xnext);
-    qhead = reinterpret_cast<int32_t*>(sl + A.off_qhead);
-    qtail = reinterpret_cast<int32_t*>(sl + A.off_qtail);
+  __device__ __forceinline__ tm_t warp_min_t(tm_t v) const {
+    if (kT32) return (tm_t)__reduce_min_sync(kFullMask, (int)v);
+    return (tm_t)warp_min_u64((uint64_t)v);  // times are >= 0
+  }
+
+  __device__ void setup_arb(int64_t slot, uint8_t* smem_warp) {
+    sl = P.scratch + slot * P.slot_bytes;
+    sm = smem_warp;
   }
 
   __device__ void reset_arb() {
     const unsigned lane = lane_id();
     this->reset_common();
-    uint4* c4 = reinterpret_cast<uint4*>(cnt);
+    uint4* c4 = reinterpret_cast<uint4*>(cnt());
+    int32_t* qh = qhead();
+    int32_t* qt = qtail();
     const int nv = (int)((4 * (size_t)g.n + 15) / 16);
     for (int x = lane; x < nv; x += 32) c4[x] = make_uint4(0u, 0u, 0u, 0u);
     for (int x = lane; x < g.D * g.D; x += 32) {
-      qhead[x] = -1;
-      qtail[x] = -1;
+      qh[x] = -1;
+      qt[x] = -1;
     }
-    lbits[lane] = 0u;
-    tq.size = 0;
+    lbits()[lane] = 0u;
     nx = 0;
     xev = 0;
     sendm = recvm = pm = 0u;
+    xd = kNever;
+    xdp = 0u;
+    xde = 0;
+    fh = ft = -1;
+    fa = kNever;
     arb_due = false;
     t_arb = 0;
     __syncwarp();
@@ -120,10 +136,12 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
   // One more input of op j present at time a (per lane); true if it was the
   // last, with its ready time in rj.
   __device__ __forceinline__ bool add_input(uint32_t j, tm_t a, tm_t& rj) const {
-    const int32_t c = cnt[j] + 1;
-    cnt[j] = c;
-    const tm_t m = c == 1 ? a : (rmax[j] > a ? rmax[j] : a);
-    rmax[j] = m;
+    int32_t* cp = cnt() + j;
+    tm_t* mp = rmax() + j;
+    const int32_t c = *cp + 1;
+    *cp = c;
+    const tm_t m = c == 1 ? a : (*mp > a ? *mp : a);
+    *mp = m;
     const RelPred jp = op_relpred(g.ops, j);
     if ((uint32_t)c != jp.npred) return false;
     const tm_t rel = (tm_t)jp.rel;
@@ -140,8 +158,8 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     }
   }
 
-  // READY(r, i): start op i; local successors get this input, remote
-  // accelerators of successors get an intent at its finish.
+  // READY(r, i): start op i; local successors get this input; if some
+  // successor is remote, i joins its accelerator's FIFO of coming intents.
   __device__ void start_op(uint32_t i, tm_t r) {
     const unsigned lane = lane_id();
     const longlong2 db = op_durbytes(g.ops, i);
@@ -176,18 +194,22 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       }
       push_readies(rdy, rj, j);
     }
-    __syncwarp();
     remote = __reduce_or_sync(kFullMask, remote);
     if (lane == 0) {
-      refs[i] = 1 + __popc(remote);
+      refs()[i] = 1 + __popc(remote);
       this->holdb[i] = f;
+      if (remote) rmask()[i] = remote;
+    }
+    if (remote && (int)lane == d) {
+      if (fh < 0) {
+        fh = (int32_t)i;
+        fa = f;
+      } else {
+        nextop()[ft] = (int32_t)i;
+      }
+      ft = (int32_t)i;
     }
     __syncwarp();
-    while (remote) {
-      const int e = __ffs(remote) - 1;
-      remote &= remote - 1;
-      if (!tq.push(xkey(f, kXIntent, i, e))) status = GMG_SIM_QUEUE;
-    }
   }
 
   // One hold on op p's own copy (on accelerator dp) ends at time v (per
@@ -197,8 +219,9 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     bool last = false;
     tm_t h = v;
     if (want) {
-      const int32_t left = refs[p] - 1;
-      refs[p] = left;
+      int32_t* rp = refs() + p;
+      const int32_t left = *rp - 1;
+      *rp = left;
       const tm_t o = this->holdb[p];
       h = o > v ? o : v;
       this->holdb[p] = h;
@@ -207,39 +230,63 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     this->log_event(last, this->kc.make(h, kFree, p), dp);
   }
 
-  // INTENT or DONE.
-  __device__ void handle_x(uint64_t k) {
+  // The intents of the earliest FIFO head arrive: one per remote
+  // accelerator, numbered in destination order.
+  __device__ void intents_arrive(uint32_t p) {
     const unsigned lane = lane_id();
-    const uint32_t cls = (uint32_t)(k >> (g.ib + 5)) & 1u;
-    const uint32_t p = (uint32_t)(k >> 5) & this->kc.mask;
-    const int e = (int)(k & 31u);
-    const tm_t t = xtime(k);
     const int a = row[p];
-    const int pair = a * g.D + e;
-    if (cls == kXIntent) {
-      if (nx >= A.xcap) {
-        status = GMG_SIM_QUEUE;
-        return;
-      }
-      const int32_t x = nx++;
-      if (lane == 0) {
-        xent[x] = (p << 5) | (uint32_t)e;
-        xnext[x] = -1;
-        const int32_t tl = qtail[pair];
-        if (tl >= 0) xnext[tl] = x;
-        else qhead[pair] = x;
-        qtail[pair] = x;
-      }
-      if ((int)lane == a) pm |= 1u << e;
-      __syncwarp();
+    const uint32_t R = rmask()[p];
+    if (nx + __popc(R) > A.xcap) {
+      status = GMG_SIM_QUEUE;
       return;
     }
-    // DONE: free the endpoints and the link
-    sendm &= ~(1u << a);
-    recvm &= ~(1u << e);
-    const uint32_t lid = __ldg(A.link + pair);
-    if (lane == 0) lbits[lid >> 5] &= ~(1u << (lid & 31u));
+    if (lane == 0) {
+      uint32_t* xe = xent();
+      int32_t* xn = xnext();
+      int32_t* qh = qhead();
+      int32_t* qt = qtail();
+      uint32_t r = R;
+      while (r) {
+        const int e = __ffs(r) - 1;
+        r &= r - 1;
+        const int32_t x = nx++;
+        const int pair = a * g.D + e;
+        xe[x] = (p << 5) | (uint32_t)e;
+        xn[x] = -1;
+        const int32_t tl = qt[pair];
+        if (tl >= 0) xn[tl] = x;
+        else qh[pair] = x;
+        qt[pair] = x;
+      }
+    } else {
+      nx += __popc(R);
+    }
+    if ((int)lane == a) {
+      pm |= R;
+      if (fh == ft) {
+        fh = ft = -1;
+        fa = kNever;
+      } else {
+        fh = nextop()[fh];
+        fa = this->fbuf[fh];
+      }
+    }
     __syncwarp();
+  }
+
+  // The transfer sent by lane src completes at time t.
+  __device__ void transfer_done(int src, tm_t t) {
+    const unsigned lane = lane_id();
+    const uint32_t p = __shfl_sync(kFullMask, xdp, src);
+    const int e = __shfl_sync(kFullMask, xde, src);
+    if ((int)lane == src) xd = kNever;
+    sendm &= ~(1u << src);
+    recvm &= ~(1u << e);
+    if (A.shared_links) {
+      const uint32_t lid = __ldg(A.link + src * g.D + e);
+      if (lane == 0) lbits()[lid >> 5] &= ~(1u << (lid & 31u));
+      __syncwarp();
+    }
     // p's successors on e have this input now
     const XqSucc xs = op_xqsucc(g.ops, p);
     for (uint32_t c0 = 0; c0 < xs.nsucc; c0 += 32) {
@@ -264,13 +311,14 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     }
     this->log_event(lane == 0 && !here, this->kc.make(t, kFree, p), e);
     // the sender's copy: one hold fewer
-    drop_hold(lane == 0, p, t, a);
+    drop_hold(lane == 0, p, t, src);
   }
 
   // Start every pending intent whose endpoints and link are free, in order.
   __device__ void arbitrate(tm_t t) {
     const int lane = (int)lane_id();
     const int D = g.D;
+    const bool links = A.shared_links != 0;
     while (true) {
       uint32_t best = 0xffffffffu;
       int be = 0;
@@ -279,9 +327,11 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
         while (c) {
           const int e = __ffs(c) - 1;
           c &= c - 1;
-          const uint32_t lid = __ldg(A.link + lane * D + e);
-          if ((lbits[lid >> 5] >> (lid & 31u)) & 1u) continue;
-          const uint32_t h = (uint32_t)qhead[lane * D + e];
+          if (links) {
+            const uint32_t lid = __ldg(A.link + lane * D + e);
+            if ((lbits()[lid >> 5] >> (lid & 31u)) & 1u) continue;
+          }
+          const uint32_t h = (uint32_t)qhead()[lane * D + e];
           if (h < best) {
             best = h;
             be = e;
@@ -292,25 +342,28 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       if (m == 0xffffffffu) break;
       const int src = __ffs(__ballot_sync(kFullMask, best == m)) - 1;
       const int e = __shfl_sync(kFullMask, be, src);
-      const uint32_t p = xent[m] >> 5;
-      const int32_t nxt = xnext[m];
+      const uint32_t p = xent()[m] >> 5;
+      const int32_t nxt = xnext()[m];
       const int pair = src * D + e;
-      const uint32_t lid = __ldg(A.link + pair);
       __syncwarp();
       if (lane == 0) {
-        qhead[pair] = nxt;
-        if (nxt < 0) qtail[pair] = -1;
-        lbits[lid >> 5] |= 1u << (lid & 31u);
+        qhead()[pair] = nxt;
+        if (nxt < 0) qtail()[pair] = -1;
+        if (links) {
+          const uint32_t lid = __ldg(A.link + pair);
+          lbits()[lid >> 5] |= 1u << (lid & 31u);
+        }
       }
       if (nxt < 0 && lane == src) pm &= ~(1u << e);
       sendm |= 1u << src;
       recvm |= 1u << e;
-      __syncwarp();
       const tm_t done = t + this->xfer(src, e, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
-      if (!tq.push(xkey(done, kXDone, p, e))) {
-        status = GMG_SIM_QUEUE;
-        return;
+      if (lane == src) {
+        xd = done;
+        xdp = p;
+        xde = e;
       }
+      __syncwarp();
       this->log_event(lane == 0, this->kc.make(t, kAlloc, p), e);
     }
   }
@@ -405,10 +458,13 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
   // a time is handled, then READY keys.
   __device__ void run() {
     if (status) return;
-    const int32_t xlim = 2 * A.xcap + 2;
+    const int32_t xlim = A.xcap + g.n + 2;
     while (true) {
-      const uint64_t tk = tq.top();
-      if (arb_due && (tk == kKeyMax || xtime(tk) > t_arb)) {
+      const tm_t td = warp_min_t(xd);
+      const uint64_t ik = warp_min_u64(fh >= 0 ? (((uint64_t)(U)fa << g.ib) | (uint32_t)fh) : kKeyMax);
+      const tm_t ti = ik == kKeyMax ? kNever : (tm_t)(ik >> g.ib);
+      const tm_t tx = td < ti ? td : ti;
+      if (arb_due && tx > t_arb) {
         arbitrate(t_arb);
         arb_due = false;
         if (status) break;
@@ -419,16 +475,15 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       const uint64_t rk = this->rkey;
       uint64_t nk = rk < top ? rk : top;
       nk = rm < nk ? rm : nk;
-      if (tk != kKeyMax && (nk == kKeyMax || (int64_t)xtime(tk) <= this->kc.time(nk))) {
+      if (tx != kNever && (nk == kKeyMax || (int64_t)tx <= this->kc.time(nk))) {
         if (++xev > xlim) {
           status = GMG_SIM_LOOP;
           break;
         }
-        __syncwarp();
-        tq.pop();
-        handle_x(tk);
+        if (td == tx) transfer_done(__ffs(__ballot_sync(kFullMask, xd == td)) - 1, td);
+        else intents_arrive((uint32_t)(ik & this->kc.mask));
         arb_due = true;
-        t_arb = xtime(tk);
+        t_arb = tx;
         if (status) break;
         continue;
       }
@@ -455,7 +510,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
 };
 
 template <bool kT32, bool kTypes>
-__global__ void __launch_bounds__(128) sim_arb_kernel(const __grid_constant__ ArbParams A) {
+__global__ void __launch_bounds__(128, 7) sim_arb_kernel(const __grid_constant__ ArbParams A) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;

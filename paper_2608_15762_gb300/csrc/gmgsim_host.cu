@@ -67,6 +67,7 @@ struct Built {
   std::vector<uint8_t> dtype; // [D] when T >= 2
   std::vector<uint16_t> linkid;  // [D*D] when D <= 32: communication link of each ordered pair
   int64_t xfer_bound = 0;     // transfers of one placement at most: sum of min(successors, D-1)
+  bool shared_links = false;  // two distinct ordered pairs share a link id
   Layout L{};
 };
 
@@ -357,9 +358,11 @@ int build(const gmg_desc_t* d, Built& b) {
     }
   if (D <= 32) {
     b.linkid.resize((size_t)D * D);
+    std::vector<int> uses((size_t)D * D, 0);
     for (size_t k = 0; k < b.linkid.size(); ++k) {
       const bool diag = k / D == k % D;
       b.linkid[k] = (uint16_t)(d->link_id && !diag ? d->link_id[k] : (int32_t)k);
+      if (!diag && ++uses[b.linkid[k]] > 1) b.shared_links = true;
     }
   }
   // Bounds: every time <= start + all durations + one transfer per edge and
@@ -415,6 +418,7 @@ struct gmg {
   int64_t queue_bound;
   int64_t log_bound;
   const uint16_t* linkid;  // device [D*D] (NULL above 32 accelerators)
+  int32_t shared_links;    // 1 if two distinct ordered pairs share a link id
   int64_t xfer_bound;
 };
 
@@ -555,7 +559,7 @@ void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
 // Arbitrated transfers: the full simulation's slot plus the transfer state.
 // At most 32 accelerators (endpoint sets are bit masks, link ids < 1024),
 // op ids below 2^27 (an intent packs op << 5 | destination) and accelerator
-// ids that fit beside the packed key (the transfer-event key is 4 bits wider).
+// ids that fit beside the packed key.
 int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams& A) {
   const DevGmg& G = g->dg;
   if (G.D > 32 || !g->linkid) return GMG_EINVAL;
@@ -573,19 +577,20 @@ int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams&
     return (int64_t)at;
   };
   A.xcap = (int32_t)xcap;
-  A.tqs = kSharedXferEntries;
-  A.tqcap = (int32_t)xcap + 1;  // every transfer has at most one key queued at a time
+  A.shared_links = g->shared_links;
+  A.heads_shared = G.D <= 16 ? 1 : 0;
   const size_t n = (size_t)G.n, DD = (size_t)G.D * G.D;
   A.off_cnt = take(4 * n);
   A.off_rmax = take((G.t32 ? 4 : 8) * n);
   A.off_refs = take(4 * n);
+  A.off_rmask = take(4 * n);
+  A.off_nextop = take(4 * n);
   A.off_xent = take(4 * (size_t)xcap);
   A.off_xnext = take(4 * (size_t)xcap);
-  A.off_qhead = take(4 * DD);
+  A.off_qhead = take(A.heads_shared ? 0 : 4 * DD);
   A.off_qtail = take(4 * DD);
-  A.off_tq = take(8 * (size_t)std::max(A.tqcap - A.tqs, 0));
   P.slot_bytes = (int64_t)o2;
-  A.smem_arb = (int32_t)align_up(8 * (size_t)A.tqs + 128, 16);
+  A.smem_arb = (int32_t)align_up(128 + (A.heads_shared ? 4 * DD : 0), 16);
   A.smem_std = (int64_t)L.smem;
   L.smem += (size_t)L.wpb * (size_t)A.smem_arb;
   const int sms = device_sms();
@@ -752,6 +757,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   g->log_bound = b.log_bound;
   g->linkid = b.linkid.empty() ? nullptr : reinterpret_cast<const uint16_t*>(w + L.off_linkid);
   g->xfer_bound = b.xfer_bound;
+  g->shared_links = b.shared_links ? 1 : 0;
   I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
   *out = g;
   return GMG_OK;
