@@ -79,6 +79,8 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
   tm_t fa;           // finish time of the FIFO head (kNever: empty)
   bool arb_due;
   tm_t t_arb;
+  tm_t td_c;         // next DONE time (warp minimum of xd), kept current
+  uint64_t ik_c;     // next INTENT key (time << ib | op), kept current
 
   __device__ ArbSim(const ArbParams& a) : Base(a.P), A(a) {}
 
@@ -100,6 +102,11 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
   __device__ __forceinline__ tm_t warp_min_t(tm_t v) const {
     if (kT32) return (tm_t)__reduce_min_sync(kFullMask, (int)v);
     return (tm_t)warp_min_u64((uint64_t)v);  // times are >= 0
+  }
+
+  __device__ __forceinline__ void refresh_done() { td_c = warp_min_t(xd); }
+  __device__ __forceinline__ void refresh_intent() {
+    ik_c = warp_min_u64(fh >= 0 ? (((uint64_t)(U)fa << g.ib) | (uint32_t)fh) : kKeyMax);
   }
 
   __device__ void setup_arb(int64_t slot, uint8_t* smem_warp) {
@@ -130,6 +137,8 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     fa = kNever;
     arb_due = false;
     t_arb = 0;
+    td_c = kNever;
+    ik_c = kKeyMax;
     __syncwarp();
   }
 
@@ -210,6 +219,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       ft = (int32_t)i;
     }
     __syncwarp();
+    if (remote) refresh_intent();
   }
 
   // One hold on op p's own copy (on accelerator dp) ends at time v (per
@@ -272,6 +282,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       }
     }
     __syncwarp();
+    refresh_intent();
   }
 
   // The transfer sent by lane src completes at time t.
@@ -280,6 +291,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     const uint32_t p = __shfl_sync(kFullMask, xdp, src);
     const int e = __shfl_sync(kFullMask, xde, src);
     if ((int)lane == src) xd = kNever;
+    refresh_done();
     sendm &= ~(1u << src);
     recvm &= ~(1u << e);
     if (A.shared_links) {
@@ -319,6 +331,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     const int lane = (int)lane_id();
     const int D = g.D;
     const bool links = A.shared_links != 0;
+    bool started = false;
     while (true) {
       uint32_t best = 0xffffffffu;
       int be = 0;
@@ -340,6 +353,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       }
       const uint32_t m = __reduce_min_sync(kFullMask, best);
       if (m == 0xffffffffu) break;
+      started = true;
       const int src = __ffs(__ballot_sync(kFullMask, best == m)) - 1;
       const int e = __shfl_sync(kFullMask, be, src);
       const uint32_t p = xent()[m] >> 5;
@@ -366,6 +380,7 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
       __syncwarp();
       this->log_event(lane == 0, this->kc.make(t, kAlloc, p), e);
     }
+    if (started) refresh_done();
   }
 
   // HBM events of the ops started since the last generation, one op per
@@ -460,8 +475,8 @@ struct ArbSim : Sim<true, kFull, true, kT32, kTypes> {
     if (status) return;
     const int32_t xlim = A.xcap + g.n + 2;
     while (true) {
-      const tm_t td = warp_min_t(xd);
-      const uint64_t ik = warp_min_u64(fh >= 0 ? (((uint64_t)(U)fa << g.ib) | (uint32_t)fh) : kKeyMax);
+      const tm_t td = td_c;
+      const uint64_t ik = ik_c;
       const tm_t ti = ik == kKeyMax ? kNever : (tm_t)(ik >> g.ib);
       const tm_t tx = td < ti ? td : ti;
       if (arb_due && tx > t_arb) {
