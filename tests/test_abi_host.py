@@ -100,6 +100,24 @@ def test_accelerator_type_validation():
     assert _create_rc(typed([0, 1], [[1, 2], [1 << 61, 4], [5, 6]])) == G.GMG_ERANGE
 
 
+def test_link_id_validation_and_option_layout():
+    import ctypes as C
+    import dataclasses
+    base = mk([[], [0], [0, 1]], [3, 4, 5], [1, 2, 3], n_dev=2, bw=2, lat=1)
+
+    def linked(ids):
+        return dataclasses.replace(base, link_id=np.asarray(ids, np.int32)).normalized()
+    assert G.gmg_workspace_bytes(linked([0, 1, 1, 0])) > 0      # both directions share link 1
+    assert G.gmg_workspace_bytes(linked([-7, 3, 2, 99])) > 0    # the diagonal is not read
+    assert _create_rc(linked([0, 4, 1, 0])) == G.GMG_EINVAL     # id >= D*D
+    assert _create_rc(linked([0, -1, 1, 0])) == G.GMG_EINVAL
+    # sim_opts_t: transfer_mode takes the first reserved word; the struct size is unchanged
+    assert C.sizeof(G._Opts) == 40 and G._Opts.transfer_mode.offset == 24
+    hdr = open(os.path.join(ROOT, "include", "gmgsim.h")).read()
+    assert re.search(r"int32_t transfer_mode;.*\n\s*int32_t reserved\[3\];", hdr)
+    assert "const int32_t* link_id;" in hdr and G._Desc.link_id.offset == C.sizeof(G._Desc) - 8
+
+
 def test_product_never_imports_the_oracle():
     pkg = os.path.join(ROOT, "paper_2608_15762_gb300")
     for dirpath, _, files in os.walk(pkg):
