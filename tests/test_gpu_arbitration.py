@@ -198,3 +198,21 @@ def test_degenerate_inputs_and_refusals():
     import ctypes as C
     assert G.lib().inc_scratch_bytes(g.handle, 4, C.addressof(o)) == 0
     assert G.lib().base_workspace_bytes(g.handle, C.addressof(o)) == 0
+
+
+def test_decode_memtight_full_size_sampled():
+    """The memory-tight decode workload at full size (8 tenants x 64 steps x
+    32 layers, N = 197,632 ops, D = 8, all 8,192 placements in one launch as
+    bench.py runs it), arbitrated; 40 sampled candidates checked against the
+    oracle one by one, every candidate's status checked."""
+    wl = W.make_workload(4)
+    rows = wl.all_full_rows()
+    g = G.gmg_create(wl.desc)
+    out = G.sim_batch(g, torch_place(rows), arbitrated=True)
+    torch.cuda.synchronize()
+    got = out.to_numpy()
+    assert (got["status"] == G.SIM_OK).all()
+    ks = np.unique(np.concatenate([[0, 1, rows.shape[0] - 1],
+                                   np.random.default_rng(4).integers(0, rows.shape[0], 37)]))
+    s, pk, _ = O.simulate_batch(wl.desc, rows[ks], arbitrated=True)
+    compare({k: (None if v is None else v[ks]) for k, v in got.items()}, s, pk)
