@@ -292,9 +292,20 @@ def cpu_baseline(wl, min_s=10.0, arbitrated=False):
         dt = time.perf_counter() - t0
         if dt >= min_s:
             break
-    return {"value": reps * k / dt, "unit": UNIT, "cores": nt, "kind": "oracle",
+    value = reps * k / dt
+    # one core: a smaller sample of the same candidates, about 3 s of work
+    k1 = int(max(1, min(k, 3.0 * value / nt)))
+    t1 = time.perf_counter()
+    if wl.n_full:
+        O.simulate_batch(wl.desc, rows[:k1], nthreads=1, arbitrated=arbitrated)
+    else:
+        O.incremental_batch(wl.desc, wl.base_place, mv.subset(range(k1)), nthreads=1)
+    dt1 = time.perf_counter() - t1
+    return {"value": value, "unit": UNIT, "cores": nt, "kind": "oracle",
             "sample": "%s, %d pass%s" % (what, reps, "" if reps == 1 else "es"), "seconds": round(dt, 3),
-            "op_events_per_s": reps * k * wl.desc.n_ops / dt if wl.n_full else None}
+            "op_events_per_s": reps * k * wl.desc.n_ops / dt if wl.n_full else None,
+            "single_core": {"value": k1 / dt1, "unit": UNIT, "cores": 1,
+                            "sample": "the first %d of those candidates, one pass" % k1}}
 
 
 def reference_arm(args):
