@@ -170,7 +170,13 @@ class Prepared:
 ARB_SOURCES = ("gmgsim_arb.cu", "gmg_arb.h")
 
 
-def prepare(config: int, rank: int, device, cap=None, arbitrated=False):
+def rows_of(wl, ks, structured=False):
+    """Full placement rows of candidates ks: uniform i.i.d. device ids, or the
+    structured variant (contiguous per-request stages on random accelerators)."""
+    return wl.structured_full_rows(ks) if structured else wl.full_rows(ks)
+
+
+def prepare(config: int, rank: int, device, cap=None, arbitrated=False, structured=False):
     import numpy as np
     import torch
     from paper_2608_15762_gb300 import gmgsim as G
@@ -179,8 +185,11 @@ def prepare(config: int, rank: int, device, cap=None, arbitrated=False):
     p = Prepared()
     p.wl = wl
     p.arb = arbitrated
+    p.structured = structured
     if arbitrated and (wl.n_full == 0 or wl.desc.n_dev > 32):
         raise SystemExit("--arbitrated needs a workload of full placements on at most 32 accelerators")
+    if structured and (wl.n_full == 0 or wl.moves is not None):
+        raise SystemExit("--placements structured needs a workload of full placements only")
     p.g = G.gmg_create(wl.desc, device=device)
     p.n_full = wl.n_full
     p.n_inc = 0 if wl.moves is None else wl.moves.n_cand
@@ -194,7 +203,8 @@ def prepare(config: int, rank: int, device, cap=None, arbitrated=False):
     p.K = p.n_full + p.n_inc
     p.host_place = None
     if p.n_full:
-        rows = wl.full_rows(range(p.n_full)) if cap is not None else wl.full_rows(G.shard_range(rank, p.n_full))
+        ks = range(p.n_full) if cap is not None else G.shard_range(rank, p.n_full)
+        rows = rows_of(wl, ks, structured)
         p.host_place = torch.from_numpy(rows).pin_memory()
         p.place = p.host_place.to(device)
     if p.n_inc:
@@ -262,7 +272,7 @@ def h2d_bytes(p):
     return b
 
 
-def cpu_baseline(wl, min_s=10.0, arbitrated=False):
+def cpu_baseline(wl, min_s=10.0, arbitrated=False, structured=False):
     """The CPU oracle as it stands on this host's cores, on a bounded sample of
     the same workload: up to ~3e8 op-events of candidates, repeated as whole
     batches until at least min_s seconds of wall time."""
@@ -271,11 +281,12 @@ def cpu_baseline(wl, min_s=10.0, arbitrated=False):
     budget = max(16, int(3e8 // max(wl.desc.n_ops, 1)))
     if wl.n_full:
         k = min(wl.n_full, budget)
-        rows = wl.full_rows(range(k))
+        rows = rows_of(wl, range(k), structured)
 
         def run():
             O.simulate_batch(wl.desc, rows, nthreads=nt, arbitrated=arbitrated)
-        what = "%d of %d full placements%s" % (k, wl.n_full, ", arbitrated transfers" if arbitrated else "")
+        what = "%d of %d full%s placements%s" % (k, wl.n_full, " structured" if structured else "",
+                                               ", arbitrated transfers" if arbitrated else "")
     else:
         from paper_2608_15762_gb300.workloads import Moves
         k = min(wl.moves.n_cand, budget)
@@ -319,7 +330,7 @@ def reference_arm(args):
     nt = O.hw_threads()
     k = min(wl.n_full or wl.moves.n_cand, max(16, int(3e7 // max(wl.desc.n_ops, 1))))
     if wl.n_full:
-        rows = wl.full_rows(range(k))
+        rows = rows_of(wl, range(k), args.placements == "structured")
 
         def step():
             O.simulate_batch(wl.desc, rows, nthreads=nt, arbitrated=args.arbitrated)
@@ -342,7 +353,8 @@ def reference_arm(args):
             "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic", "impl": "reference",
             "config": {"workload": wl.name, "candidates_per_step": k, "n_ops": wl.desc.n_ops,
-                       "transfers": "arbitrated" if args.arbitrated else "latency"},
+                       "transfers": "arbitrated" if args.arbitrated else "latency",
+                       "placements": args.placements},
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": nt, "kind": "oracle",
                              "sample": "%d candidates per step" % k},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -667,6 +679,9 @@ def main():
                     help="time the online estimators (refit, durations, links) instead of the simulation")
     ap.add_argument("--arbitrated", action="store_true",
                     help="arbitrated transfers (Sec. 3.5.2) instead of pure-latency ones")
+    ap.add_argument("--placements", default="uniform", choices=["uniform", "structured"],
+                    help="full placement rows: uniform i.i.d. device ids, or contiguous per-request "
+                         "stages on random accelerators")
     ap.add_argument("--candidates", type=int, default=None,
                     help="profiling aid: simulate only the first N candidates of each half "
                          "(the line then describes that smaller batch)")
@@ -692,7 +707,8 @@ def main():
 
     from paper_2608_15762_gb300 import build as lib_build
     lib_build.build()
-    p = prepare(args.config, rank, device, cap=args.candidates, arbitrated=args.arbitrated)
+    p = prepare(args.config, rank, device, cap=args.candidates, arbitrated=args.arbitrated,
+                structured=args.placements == "structured")
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
 
     def barrier():
@@ -765,7 +781,7 @@ def main():
     hbm_gbs = alg_bytes / (kms / 1000) / 1e9
     props = torch.cuda.get_device_properties(device)
     issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
-    ppath = profile_path(kern, wl.name)
+    ppath = profile_path(kern, wl.name + ("-structured" if p.structured else ""))
     prof = read_profile(ppath, ARB_SOURCES if p.arb else ())
     roof = {"bound": "alu", "unit": "Ginst/s", "peak": issue_peak,
             "peak_src": "%d SMs x 4 issue slots x %.0f MHz (%s sm_max_mhz)" % (
@@ -784,6 +800,7 @@ def main():
         "ms_per_step_best": min(step_ms), "ms_per_step_median": statistics.median(step_ms),
         "config": {"workload": wl.name, "candidates": K, "n_ops": N, "n_dev": D,
                    "transfers": "arbitrated" if p.arb else "latency",
+                   "placements": "structured" if p.structured else "uniform",
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
                    "parallelism": "dp%d over candidates" % world},
         # full placements simulate every op; an incremental candidate re-simulates
@@ -800,7 +817,7 @@ def main():
         "best": best,
     }
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, arbitrated=p.arb)
+        line["cpu_baseline"] = cpu_baseline(wl, arbitrated=p.arb, structured=p.structured)
     if rank == 0:
         print(json.dumps(line))
     if world > 1:

@@ -181,6 +181,11 @@ class Workload:
     def all_full_rows(self) -> np.ndarray:
         return self.full_rows(range(self.n_full))
 
+    def structured_full_rows(self, ks: Sequence[int]) -> np.ndarray:
+        """Structured placements (contiguous per-request stages on random
+        accelerators) of the given full candidates."""
+        return structured_rows(self.place_seed, ks, self.desc.req_id, self.desc.n_dev)
+
 
 def placement_ld(n_ops: int) -> int:
     """Row pitch of a placement array: n_ops rounded up to 16 bytes."""
@@ -196,6 +201,33 @@ def random_rows(seed: int, ks: Sequence[int], n_ops: int, n_dev: int) -> np.ndar
     for r, k in enumerate(ks):
         g = np.random.default_rng(np.random.SeedSequence([seed, 1000, int(k)]))
         out[r, :n_ops] = g.integers(0, n_dev, size=n_ops, dtype=np.uint8) if n_ops else 0
+    return out
+
+
+def structured_rows(seed: int, ks: Sequence[int], req_id: np.ndarray, n_dev: int,
+                    stages=(1, 2, 4, 8)) -> np.ndarray:
+    """Placements built like the pre-defined partitions of Sec. 3.4.2: each
+    request's ops, in id order, are cut into S contiguous stages of (nearly)
+    equal size, S drawn from `stages`, and each stage goes to a uniformly
+    drawn accelerator; ops outside any request are placed uniformly.  Row k
+    comes from its own seeded stream."""
+    req_id = np.asarray(req_id)
+    n = req_id.shape[0]
+    ld = placement_ld(n)
+    tenants = [np.flatnonzero(req_id == r) for r in range(int(req_id.max()) + 1)] if n else []
+    loose = np.flatnonzero(req_id < 0)
+    ks = list(ks)
+    out = np.zeros((len(ks), ld), dtype=np.uint8)
+    for r, k in enumerate(ks):
+        g = np.random.default_rng(np.random.SeedSequence([seed, 2000, int(k)]))
+        for ops in tenants:
+            if ops.size == 0:
+                continue
+            S = int(g.choice(stages))
+            for part in np.array_split(ops, min(S, ops.size)):
+                out[r, part] = g.integers(0, n_dev)
+        if loose.size:
+            out[r, loose] = g.integers(0, n_dev, size=loose.size, dtype=np.uint8)
     return out
 
 
