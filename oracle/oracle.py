@@ -156,8 +156,8 @@ def simulate_batch(desc, place, nthreads: int = 0, arbitrated=False):
     return s, peak, req[:, :d.n_req]
 
 
-def incremental_batch(desc, base_place, moves, nthreads: int = 0):
-    h = _GraphHolder(desc)
+def incremental_batch(desc, base_place, moves, nthreads: int = 0, arbitrated=False):
+    h = _GraphHolder(desc, arbitrated)
     d = h.desc
     base = np.ascontiguousarray(base_place, dtype=np.uint8)
     off = np.ascontiguousarray(moves.off, dtype=np.int32)

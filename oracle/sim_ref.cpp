@@ -58,7 +58,8 @@
 //    placement; its event count is the number of operators whose base ready
 //    time is at or after the resume time T0 = min over moved ops x of
 //    (min over predecessors p of the base finish of p, or x's release if it
-//    has none).
+//    has none).  With arbitrated transfers the moved placement is simulated
+//    in full and the event count is the number of operators.
 //
 // Everything is int64; no floating point is involved.
 
@@ -741,8 +742,11 @@ int orc_incremental_batch(const orc_graph* in, const uint8_t* base_place, const 
     }
     simulate(g, place.data(), res);
     int64_t ev = 0;
-    if (t0 != kI64Max)
+    if (g.mode == 1) {
+      ev = g.n;  // arbitrated transfers: the moved placement is simulated in full
+    } else if (t0 != kI64Max) {
       for (int i = 0; i < g.n; ++i) ev += base.ready[i] >= t0 ? 1 : 0;
+    }
     res.s.events = ev;
     write_out(g, res, k, out, peak, req_done);
   });

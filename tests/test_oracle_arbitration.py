@@ -12,6 +12,7 @@ import pytest
 import refsim
 from helpers import mk, row
 from oracle import oracle as O
+from paper_2608_15762_gb300 import workloads as W
 from paper_2608_15762_gb300.workloads import random_desc
 
 
@@ -230,3 +231,26 @@ def test_rejects_bad_link_ids():
     assert O.check(d, arbitrated=True) == O.EINVAL
     d.link_id = np.array([9, 1, 2, -3], np.int32)  # the diagonal is not read
     assert O.check(d, arbitrated=True) == 0
+
+
+def test_incremental_is_the_full_arbitrated_simulation_of_the_moved_placement():
+    d = random_desc(5, 80, 4)
+    base = np.random.default_rng(1).integers(0, 4, 80).astype(np.uint8)
+    mv = W.random_moves(3, 24, base, 4, max_moves=5)
+    # two malformed move lists: an out-of-range device and a repeated op
+    mv.dev[mv.off[2]] = 9
+    assert mv.off[6] - mv.off[5] > 1
+    mv.op[mv.off[5] + 1] = mv.op[mv.off[5]]
+    s, pk, rq = O.incremental_batch(d, base, mv, arbitrated=True)
+    sl, _, _ = O.incremental_batch(d, base, mv)
+    assert s["status"].tolist() == sl["status"].tolist() and s["status"][2] == O.SIM_MOVE_RANGE
+    assert s["status"][5] == O.SIM_MOVE_DUP
+    for k in range(24):
+        if s["status"][k]:
+            continue
+        pl = base.copy()
+        a, b = mv.off[k], mv.off[k + 1]
+        pl[mv.op[a:b]] = mv.dev[a:b]
+        r = _arb(d, pl)
+        assert (r["score"], r["makespan"], r["viol_flag"]) == (s["score"][k], s["makespan"][k], s["viol_flag"][k])
+        assert r["peak"].tolist() == pk[k].tolist() and s["events"][k] == d.n_ops
