@@ -199,8 +199,11 @@ size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts);
  * not fix the choice among conflicting intents: this FIFO-greedy order is
  * the library's.  Needs n_dev <= 32 (else GMG_EINVAL) and op ids < 2^27 with
  * accelerator ids that fit the packed event key (else GMG_ERANGE).
- * base_create, sim_incremental and their size queries accept only
- * GMG_TRANSFER_LATENCY (GMG_EINVAL, or 0 bytes, otherwise). */
+ * base_create and base_workspace_bytes accept only GMG_TRANSFER_LATENCY
+ * (GMG_EINVAL, or 0 bytes, otherwise).  sim_incremental with
+ * GMG_TRANSFER_ARBITRATED takes such a base but uses only its placement and
+ * status: every candidate's moved placement is simulated in full (events =
+ * n_ops), since the base's resume points hold no transfer state. */
 int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld,
               const sim_opts_t* opts, const sim_out_t* d_out, void* d_scratch,
               size_t scratch_bytes, gmg_stream_t stream);
@@ -252,7 +255,8 @@ size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts);
  * moves can change is re-simulated, from T0 = min over effective moves x of
  * (min base finish of x's predecessors, or x's release).  Move lists are CSR
  * on the device: ops d_move_op[d_move_off[k]..d_move_off[k+1]) go to
- * d_move_dev[...].  events[k] = ops whose base ready time is >= T0. */
+ * d_move_dev[...].  events[k] = ops whose base ready time is >= T0
+ * (n_ops with GMG_TRANSFER_ARBITRATED: the moved placement is simulated in full). */
 int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_off,
                     const int32_t* d_move_op, const uint8_t* d_move_dev, int32_t K,
                     const sim_opts_t* opts, const sim_out_t* d_out, void* d_scratch,

@@ -28,7 +28,15 @@ struct ArbParams {
   int64_t off_xnext;      // int32 [xcap]  next intent of the same pair (-1: last)
   int64_t off_qhead;      // int32 [D*D]  first pending intent of each pair (-1: none), when not shared
   int64_t off_qtail;      // int32 [D*D]
+  const int32_t* pre_status;  // [K] optional: a nonzero entry is the candidate's status, not simulated
 };
+
+// Incremental candidates under arbitrated transfers: row k = the base row with
+// candidate k's moves applied (rows [K][ld]); status[k] = the move list's
+// GMG_SIM_* code (GMG_SIM_BADBASE for every candidate if *base_status is not OK).
+cudaError_t launch_expand_moves(const uint8_t* base_row, const int32_t* base_status, int32_t ld, int32_t n,
+                                int32_t D, const int32_t* off, const int32_t* op, const uint8_t* dev, int32_t K,
+                                uint8_t* rows, int32_t* status, cudaStream_t st);
 
 // Kernel entry of one instance (for occupancy queries) and the launcher.
 const void* arb_kernel_ptr(bool t32, bool types);

@@ -46,6 +46,8 @@
 // Requires at most 32 accelerators (endpoint sets are warp bit masks) and an
 // accelerator id that fits beside the packed key.  Every loop is bounded by
 // the graph: DONEs by the number of transfers, INTENTs by the number of ops.
+#include <algorithm>
+
 #include "gmg_arb.h"
 #include "gmgsim_sim.cuh"
 
@@ -535,6 +537,13 @@ __global__ void __launch_bounds__(128, 7) sim_arb_kernel(const __grid_constant__
   S.setup_arb(slot, smem + A.smem_std + (size_t)wib * A.smem_arb);
   for (int64_t k = slot; k < A.P.K; k += nslots) {
     S.row = A.P.place + k * A.P.ld;
+    if (A.pre_status) {
+      const int32_t ps = A.pre_status[k];
+      if (ps != GMG_SIM_OK) {
+        S.write_invalid(k, ps);
+        continue;
+      }
+    }
     if (S.row_has_bad_device(S.row)) {
       S.write_invalid(k, GMG_SIM_BADDEV);
       continue;
@@ -545,7 +554,51 @@ __global__ void __launch_bounds__(128, 7) sim_arb_kernel(const __grid_constant__
   }
 }
 
+// One warp per incremental candidate: check the move list (an op or device
+// out of range, then an op moved twice), copy the base row, apply the moves.
+__global__ void __launch_bounds__(128) expand_moves_kernel(const uint8_t* base_row, const int32_t* base_status,
+                                                           int32_t ld, int32_t n, int32_t D, const int32_t* off,
+                                                           const int32_t* op, const uint8_t* dev, int32_t K,
+                                                           uint8_t* rows, int32_t* status) {
+  const unsigned lane = lane_id();
+  const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
+  const bool base_ok = *base_status == GMG_SIM_OK;
+  for (int64_t k = w0; k < K; k += nw) {
+    const int32_t a = off[k], b = off[k + 1];
+    int32_t st = base_ok ? GMG_SIM_OK : GMG_SIM_BADBASE;
+    if (st == GMG_SIM_OK) {
+      bool bad = false;
+      for (int32_t m = a + (int32_t)lane; m < b; m += 32) bad |= op[m] < 0 || op[m] >= n || dev[m] >= D;
+      if (__any_sync(kFullMask, bad)) st = GMG_SIM_MOVE_RANGE;
+    }
+    if (st == GMG_SIM_OK) {
+      bool dup = false;
+      for (int32_t m = a + (int32_t)lane; m < b; m += 32)
+        for (int32_t m2 = m + 1; m2 < b && !dup; ++m2) dup = op[m2] == op[m];
+      if (__any_sync(kFullMask, dup)) st = GMG_SIM_MOVE_DUP;
+    }
+    uint8_t* rw = rows + k * (int64_t)ld;
+    for (int32_t c = (int32_t)lane * 16; c < ld; c += 512)
+      *reinterpret_cast<uint4*>(rw + c) = *reinterpret_cast<const uint4*>(base_row + c);
+    __syncwarp();
+    if (st == GMG_SIM_OK)
+      for (int32_t m = a + (int32_t)lane; m < b; m += 32) rw[op[m]] = dev[m];
+    if (lane == 0) status[k] = st;
+    __syncwarp();
+  }
+}
+
 }  // namespace
+
+cudaError_t launch_expand_moves(const uint8_t* base_row, const int32_t* base_status, int32_t ld, int32_t n,
+                                int32_t D, const int32_t* off, const int32_t* op, const uint8_t* dev, int32_t K,
+                                uint8_t* rows, int32_t* status, cudaStream_t st) {
+  const int blocks = (int)std::min<int64_t>(((int64_t)K + 3) / 4, 152 * 16);
+  expand_moves_kernel<<<std::max(blocks, 1), 128, 0, st>>>(base_row, base_status, ld, n, D, off, op, dev, K,
+                                                           rows, status);
+  return cudaGetLastError();
+}
 
 const void* arb_kernel_ptr(bool t32, bool types) {
   if (t32) return types ? (const void*)sim_arb_kernel<true, true> : (const void*)sim_arb_kernel<true, false>;

@@ -35,7 +35,6 @@ constexpr int64_t kI64Max = 0x7fffffffffffffffll;
 constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
 constexpr int kDefaultWarpsPerBlock = 4;
 constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
-constexpr int kSharedXferEntries = 33;   // transfer-event heap: the root and its children
 constexpr int64_t kDefaultQueueCap = 1 << 16;
 constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
@@ -950,8 +949,22 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
 
 void base_destroy(gmg_base_t* b) { delete b; }
 
+// Arbitrated incremental candidates: [moved rows K x ld | move statuses K | slots].
+static size_t arb_inc_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts, size_t* off_status, size_t* off_slots) {
+  Launch L;
+  ArbParams A;
+  if (plan_arb(g, K, opts, L, A)) return 0;
+  const size_t ld = align_up((size_t)std::max(g->dg.n, 1), 16);
+  const size_t os = align_up((size_t)K * ld, 256);
+  const size_t oz = os + align_up(4 * (size_t)std::max(K, 1), 256);
+  if (off_status) *off_status = os;
+  if (off_slots) *off_slots = oz;
+  return oz + (size_t)L.slots * (size_t)L.P.slot_bytes;
+}
+
 size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
-  if (!g || K < 0 || arbitrated(opts)) return 0;
+  if (!g || K < 0) return 0;
+  if (arbitrated(opts)) return arb_inc_bytes(g, K, opts, nullptr, nullptr);
   Launch L;
   if (plan_launch(g, K, opts, true, L)) return 0;
   return (size_t)L.slots * (size_t)L.P.slot_bytes;
@@ -960,11 +973,42 @@ size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
 int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_off, const int32_t* d_move_op,
                     const uint8_t* d_move_dev, int32_t K, const sim_opts_t* opts, const sim_out_t* d_out,
                     void* d_scratch, size_t scratch_bytes, gmg_stream_t stream) {
-  if (!g || !b || b->g != g || K < 0 || arbitrated(opts)) return GMG_EINVAL;
+  if (!g || !b || b->g != g || K < 0) return GMG_EINVAL;
   int rc = check_out(d_out, opts);
   if (rc) return rc;
   if (K == 0) return GMG_OK;
   if (!d_move_off) return GMG_EINVAL;
+  if (arbitrated(opts)) {
+    // Arbitrated transfers: every candidate's moved placement is simulated in
+    // full (the base snapshot's resume points hold no transfer state).
+    size_t os = 0, oz = 0;
+    const size_t need = arb_inc_bytes(g, K, opts, &os, &oz);
+    if (need == 0) {
+      Launch L0;
+      ArbParams A0;
+      const int prc = plan_arb(g, K, opts, L0, A0);
+      return prc ? prc : GMG_EINVAL;
+    }
+    if (!d_scratch || !aligned(d_scratch, 256) || scratch_bytes < need) return GMG_EWS;
+    Launch L;
+    ArbParams A;
+    rc = plan_arb(g, K, opts, L, A);
+    if (rc) return rc;
+    uint8_t* sc = static_cast<uint8_t*>(d_scratch);
+    const int32_t ld = b->db.ld;
+    const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
+    if (launch_expand_moves(b->db.row, b->db.status, ld, g->dg.n, g->dg.D, d_move_off, d_move_op, d_move_dev, K,
+                            sc, reinterpret_cast<int32_t*>(sc + os), st) != cudaSuccess)
+      return GMG_ECUDA;
+    SimParams& P = L.P;
+    fill_out(P, d_out, opts);
+    P.place = sc;
+    P.ld = ld;
+    P.K = K;
+    P.scratch = sc + oz;
+    A.pre_status = reinterpret_cast<const int32_t*>(sc + os);
+    return launch_arb_batch(g, L, A, st) == cudaSuccess ? GMG_OK : GMG_ECUDA;
+  }
   Launch L;
   rc = plan_launch(g, K, opts, true, L);
   if (rc) return rc;

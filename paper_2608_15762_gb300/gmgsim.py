@@ -371,13 +371,15 @@ def base_create(g: Gmg, base_place, queue_cap=0, stream=None) -> Base:
 
 def sim_incremental(g: Gmg, base: Base, move_off, move_op, move_dev, out: Optional[SimOut] = None,
                     scratch: Optional[Scratch] = None, req_done=False, trace_k=None, queue_cap=0,
-                    warps_per_block=0, stream=None) -> SimOut:
-    """K move lists (CUDA int32 off[K+1], int32 op[M], uint8 dev[M]) against ``base``."""
+                    warps_per_block=0, stream=None, arbitrated=False) -> SimOut:
+    """K move lists (CUDA int32 off[K+1], int32 op[M], uint8 dev[M]) against ``base``;
+    ``arbitrated``: transfers go through the arbiter of Sec. 3.5.2 (each moved
+    placement is then simulated in full)."""
     K = int(move_off.numel()) - 1
     n_trace = 0 if trace_k is None else int(trace_k.numel())
     if out is None:
         out = SimOut.empty(K, g.n_dev, g.n_req, move_off.device, req_done, n_trace, g.n_ops)
-    o = _opts(0, trace_k, queue_cap, warps_per_block)
+    o = _opts(0, trace_k, queue_cap, warps_per_block, arbitrated)
     need = lib().inc_scratch_bytes(g.handle, K, C.addressof(o))
     scratch = scratch or Scratch(move_off.device)
     buf = scratch.get(need)

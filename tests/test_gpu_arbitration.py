@@ -189,14 +189,14 @@ def test_degenerate_inputs_and_refusals():
     with pytest.raises(G.GmgError) as ei:
         G.sim_batch(G.gmg_create(dw), torch_place(rw), arbitrated=True)
     assert ei.value.code == G.GMG_ERANGE
-    # more than 32 accelerators, and the incremental entry points, refuse
+    # more than 32 accelerators refuse; a base snapshot is only made without arbitration
     d40, rows40 = _case(71, 50, 40, None)
     with pytest.raises(G.GmgError) as ei:
         G.sim_batch(G.gmg_create(d40), torch_place(rows40), arbitrated=True)
     assert ei.value.code == G.GMG_EINVAL
     o = G._opts(arbitrated=True)
     import ctypes as C
-    assert G.lib().inc_scratch_bytes(g.handle, 4, C.addressof(o)) == 0
+    assert G.lib().inc_scratch_bytes(g.handle, 4, C.addressof(o)) > 0   # moved placements in full
     assert G.lib().base_workspace_bytes(g.handle, C.addressof(o)) == 0
 
 
@@ -216,3 +216,45 @@ def test_decode_memtight_full_size_sampled():
                                    np.random.default_rng(4).integers(0, rows.shape[0], 37)]))
     s, pk, _ = O.simulate_batch(wl.desc, rows[ks], arbitrated=True)
     compare({k: (None if v is None else v[ks]) for k, v in got.items()}, s, pk)
+
+
+def _inc_compare(d, base_place, mv, **kw):
+    g = G.gmg_create(d)
+    b = G.base_create(g, torch.from_numpy(np.ascontiguousarray(base_place[:d.n_ops])).cuda())
+    off, op, dv = G.moves_to_device(mv, "cuda")
+    out = G.sim_incremental(g, b, off, op, dv, req_done=True, arbitrated=True, **kw)
+    torch.cuda.synchronize()
+    s, pk, rq = O.incremental_batch(d, base_place[:d.n_ops], mv, arbitrated=True)
+    compare(out.to_numpy(), s, pk, rq)
+    return out.to_numpy(), s
+
+
+@pytest.mark.parametrize("seed,n,D,links", [(80, 60, 3, None), (81, 300, 8, "pair"), (82, 500, 16, "uplink"),
+                                            (83, 200, 32, "random")])
+def test_incremental_candidates_bit_exact(seed, n, D, links):
+    """Move lists against a base placement, arbitrated: each candidate is the
+    full arbitrated simulation of its moved placement (events = n), and
+    malformed move lists get the same status codes as without arbitration."""
+    d, rows = _case(seed, n, D, links)
+    base = rows[0, :n].copy()
+    mv = W.random_moves(seed, 64, base, D, max_moves=12)
+    mv.dev[mv.off[3]] = D                           # a device out of range
+    if mv.off[8] - mv.off[7] > 1:
+        mv.op[mv.off[7] + 1] = mv.op[mv.off[7]]     # an op moved twice
+    got, s = _inc_compare(d, base, mv)
+    assert got["status"][3] == G.SIM_MOVE_RANGE
+    assert (got["events"][got["status"] == 0] == n).all()
+
+
+def test_incremental_workload_moves_and_a_bad_base():
+    """The incremental workload's 16,384 move lists (32 x 32-layer graph, 16
+    accelerators) through sim_incremental, arbitrated, every candidate; then
+    a base placement with a device out of range (every candidate BADBASE)."""
+    wl = W.make_workload(3)
+    _inc_compare(wl.desc, wl.base_place, wl.moves)
+    d, rows = _case(84, 40, 3, None)
+    bad = rows[0, :40].copy()
+    bad[5] = 7
+    mv = W.random_moves(84, 8, rows[0, :40].copy(), 3, max_moves=4)
+    got, s = _inc_compare(d, bad, mv)
+    assert (got["status"] == G.SIM_BADBASE).all()
