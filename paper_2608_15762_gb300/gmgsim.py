@@ -10,6 +10,7 @@ Names follow the C ABI: ``gmg_create``, ``sim_batch``, ``base_create``,
 from __future__ import annotations
 
 import ctypes as C
+import functools
 import os
 from dataclasses import dataclass
 from typing import Optional
@@ -30,6 +31,27 @@ EXPORTED = ("gmg_workspace_bytes", "gmg_create", "gmg_destroy", "gmg_get_info", 
             "est_coefficients",
             "est_predict_durations", "est_links", "round_scratch_bytes", "round_select", "round_candidates",
             "round_commit")
+
+
+# NVTX ranges around the public calls (for nsys / ncu range filters), when
+# the environment sets GMGSIM_NVTX=1; nothing is pushed otherwise.
+NVTX = os.environ.get("GMGSIM_NVTX", "") not in ("", "0")
+
+
+def _traced(name: str):
+    def wrap(fn):
+        @functools.wraps(fn)
+        def call(*a, **kw):
+            if not NVTX:
+                return fn(*a, **kw)
+            import torch
+            torch.cuda.nvtx.range_push("gmgsim." + name)
+            try:
+                return fn(*a, **kw)
+            finally:
+                torch.cuda.nvtx.range_pop()
+        return call
+    return wrap
 
 
 class GmgError(RuntimeError):
@@ -216,6 +238,7 @@ class Gmg:
             pass
 
 
+@_traced("gmg_create")
 def gmg_create(desc, device="cuda", stream=None) -> Gmg:
     return Gmg(desc, device, stream)
 
@@ -290,6 +313,7 @@ class Scratch:
         return self.buf
 
 
+@_traced("sim_batch")
 def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scratch] = None,
               req_done=False, trace_k=None, queue_cap=0, warps_per_block=0, stream=None,
               arbitrated=False) -> SimOut:
@@ -313,6 +337,7 @@ def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scr
     return out
 
 
+@_traced("sim_batch_noalloc")
 def sim_batch_noalloc(g: Gmg, place, out: Optional[SimOut] = None, req_done=False, trace_k=None,
                       stream=None, arbitrated=False) -> SimOut:
     """Like sim_batch, but the library supplies the scratch from its own fixed
@@ -365,10 +390,12 @@ class Base:
             pass
 
 
+@_traced("base_create")
 def base_create(g: Gmg, base_place, queue_cap=0, stream=None) -> Base:
     return Base(g, base_place, queue_cap, stream)
 
 
+@_traced("sim_incremental")
 def sim_incremental(g: Gmg, base: Base, move_off, move_op, move_dev, out: Optional[SimOut] = None,
                     scratch: Optional[Scratch] = None, req_done=False, trace_k=None, queue_cap=0,
                     warps_per_block=0, stream=None, arbitrated=False) -> SimOut:
@@ -393,6 +420,7 @@ def sim_incremental(g: Gmg, base: Base, move_off, move_op, move_dev, out: Option
     return out
 
 
+@_traced("select_best")
 def select_best(out: SimOut, K: Optional[int] = None, score_mode: int = 0, best=None, tmp=None,
                 stream=None):
     """Device int64[2] = (best candidate or -1, its score)."""
@@ -472,6 +500,7 @@ class Estimators:
         _check(lib().est_reset(self.state.data_ptr(), self.n_est, self.n_feat, _stream_handle(stream)),
                "est_reset")
 
+    @_traced("est_update")
     def update(self, off, x, y, tmp=None, stream=None):
         """Add samples (CSR by estimator: off int32 [n_est+1], x float64
         [S, n_feat], y float64 [S], device tensors) and refit.  tmp: an
@@ -495,6 +524,7 @@ class Estimators:
                                       fitted.data_ptr(), _stream_handle(stream)), "est_coefficients")
         return beta, fitted
 
+    @_traced("est_predict_durations")
     def predict_durations(self, est_of, x, dflt, out=None, stream=None):
         """dur_by_type [n_ops, n_types] int64 from est_of int32 [n_ops, n_types],
         op features x float64 [n_ops, n_feat] and fallback durations dflt
@@ -508,6 +538,7 @@ class Estimators:
                                            _stream_handle(stream)), "est_predict_durations")
         return out
 
+    @_traced("est_links")
     def links(self, n_dev, bw_dflt, lat_dflt, stream=None):
         """(bw, lat) int64 [n_dev*n_dev] from the transfer estimators
         (n_est = n_dev^2, n_feat = 2)."""
@@ -552,6 +583,7 @@ class Round:
         self.sim_scratch = Scratch(dev)
         self.best = torch.empty(2, dtype=torch.int64, device=dev)
 
+    @_traced("round_step")
     def step(self, stream=None):
         h = _stream_handle(stream)
         self.epoch += 1

@@ -125,3 +125,24 @@ def test_product_never_imports_the_oracle():
             if f.endswith((".py", ".cu", ".h", ".cpp")):
                 src = open(os.path.join(dirpath, f)).read()
                 assert not re.search(r"^\s*(from|import)\s+oracle|liboracle|sim_ref", src, re.M), f
+
+
+def test_nvtx_ranges_are_opt_in_and_balanced(monkeypatch):
+    torch = pytest.importorskip("torch")
+    calls = []
+    monkeypatch.setattr(torch.cuda.nvtx, "range_push", lambda n: calls.append(("push", n)))
+    monkeypatch.setattr(torch.cuda.nvtx, "range_pop", lambda: calls.append(("pop",)))
+
+    @G._traced("probe")
+    def probe(fail):
+        if fail:
+            raise ValueError("x")
+        return 7
+    monkeypatch.setattr(G, "NVTX", False)
+    assert probe(False) == 7 and calls == []
+    monkeypatch.setattr(G, "NVTX", True)
+    assert probe(False) == 7
+    with pytest.raises(ValueError):
+        probe(True)
+    assert calls == [("push", "gmgsim.probe"), ("pop",), ("push", "gmgsim.probe"), ("pop",)]
+    assert G.sim_batch.__name__ == "sim_batch" and G.sim_incremental.__wrapped__ is not None
