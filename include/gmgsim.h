@@ -197,8 +197,9 @@ size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts);
  * lasts the transfer estimate; its receive buffer is allocated when it
  * starts; the successors' input arrives when it completes.  The paper does
  * not fix the choice among conflicting intents: this FIFO-greedy order is
- * the library's.  Needs n_dev <= 32 (else GMG_EINVAL) and op ids < 2^27 with
- * accelerator ids that fit the packed event key (else GMG_ERANGE).
+ * the library's.  Needs accelerator ids that fit the packed event key and
+ * op ids < 2^27 (n_dev <= 32) or < 2^24 (33 to 256 accelerators), else
+ * GMG_ERANGE.
  * base_create and base_workspace_bytes accept only GMG_TRANSFER_LATENCY
  * (GMG_EINVAL, or 0 bytes, otherwise).  sim_incremental with
  * GMG_TRANSFER_ARBITRATED takes such a base but uses only its placement and

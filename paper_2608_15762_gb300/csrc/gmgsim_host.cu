@@ -12,6 +12,7 @@
 
 #include "gmg_access.h"
 #include "gmg_arb.h"
+#include "gmg_arbw.h"
 
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
@@ -64,7 +65,7 @@ struct Built {
   std::vector<LinkRec> links;
   std::vector<int64_t> durt;  // [n*T] when T >= 2
   std::vector<uint8_t> dtype; // [D] when T >= 2
-  std::vector<uint16_t> linkid;  // [D*D] when D <= 32: communication link of each ordered pair
+  std::vector<uint16_t> linkid;  // [D*D] communication link of each ordered pair
   int64_t xfer_bound = 0;     // transfers of one placement at most: sum of min(successors, D-1)
   bool shared_links = false;  // two distinct ordered pairs share a link id
   Layout L{};
@@ -348,14 +349,14 @@ int build(const gmg_desc_t* d, Built& b) {
                    : make_link(d->bw_B_per_us[(size_t)s * D + e], d->lat_us[(size_t)s * D + e]);
   }
   for (int i = 0; i < n; ++i) b.ops[i].xq = host_ceil(b.ops[i].bytes, b.bw0);
-  // communication links of the arbitrated transfers (kept for <= 32 accelerators)
+  // communication links of the arbitrated transfers
   for (int s = 0; s < D; ++s)
     for (int e = 0; e < D; ++e) {
       const size_t k = (size_t)s * D + e;
       const int64_t id = d->link_id ? d->link_id[k] : (int64_t)k;
       if (s != e && (id < 0 || id >= (int64_t)D * D)) return GMG_EINVAL;
     }
-  if (D <= 32) {
+  {
     b.linkid.resize((size_t)D * D);
     std::vector<int> uses((size_t)D * D, 0);
     for (size_t k = 0; k < b.linkid.size(); ++k) {
@@ -416,7 +417,7 @@ struct gmg {
   gmg_info_t info;
   int64_t queue_bound;
   int64_t log_bound;
-  const uint16_t* linkid;  // device [D*D] (NULL above 32 accelerators)
+  const uint16_t* linkid;  // device [D*D]
   int32_t shared_links;    // 1 if two distinct ordered pairs share a link id
   int64_t xfer_bound;
 };
@@ -606,10 +607,85 @@ int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams&
   return GMG_OK;
 }
 
-cudaError_t launch_arb_batch(const gmg* g, Launch& L, ArbParams& A, cudaStream_t st) {
-  A.P = L.P;
-  return launch_arb(g->dg.t32 != 0, g->dg.ntypes >= 2, A, L.grid, 32 * L.wpb, L.smem, st);
+// Arbitrated transfers on 33..256 accelerators: per-accelerator transfer
+// state in tables.  Op ids below 2^24 (an intent packs op << 8 | destination).
+int plan_arbw(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbWParams& A) {
+  const DevGmg& G = g->dg;
+  if (G.D <= 32 || G.D > 256 || !g->linkid) return GMG_EINVAL;
+  if (!G.dev_key || G.n >= (1 << 24)) return GMG_ERANGE;
+  const int64_t xcap = std::max<int64_t>(g->xfer_bound, 1);
+  if (xcap > (int64_t(1) << 29)) return GMG_ERANGE;
+  int rc = plan_launch(g, K, o, false, L);
+  if (rc) return rc;
+  std::memset(&A, 0, sizeof(A));
+  SimParams& P = L.P;
+  size_t o2 = (size_t)P.slot_bytes;
+  auto take = [&](size_t bytes) {
+    const size_t at = o2;
+    o2 = align_up(o2 + std::max<size_t>(bytes, 1), 256);
+    return (int64_t)at;
+  };
+  const size_t n = (size_t)G.n, D = (size_t)G.D, DD = D * D, tsz = G.t32 ? 4 : 8;
+  A.xcap = (int32_t)xcap;
+  A.shared_links = g->shared_links;
+  A.words = (int32_t)((D + 31) / 32);
+  A.off_cnt = take(4 * n);
+  A.off_rmax = take(tsz * n);
+  A.off_refs = take(4 * n);
+  A.off_nextop = take(4 * n);
+  A.off_xent = take(4 * (size_t)xcap);
+  A.off_xnext = take(4 * (size_t)xcap);
+  A.off_qhead = take(4 * DD);
+  A.off_qtail = take(4 * DD);
+  A.off_xd = take(tsz * D);
+  A.off_xp = take(4 * D);
+  A.off_xe = take(4 * D);
+  A.off_fh = take(4 * D);
+  A.off_ft = take(4 * D);
+  A.off_fa = take(tsz * D);
+  A.off_pm = take(4 * D * (size_t)A.words);
+  A.off_lb = take(4 * ((DD + 31) / 32));
+  P.slot_bytes = (int64_t)o2;
+  A.smem_arb = 128;  // four 8-word bit sets
+  A.smem_std = (int64_t)L.smem;
+  L.smem += (size_t)L.wpb * (size_t)A.smem_arb;
+  const int sms = device_sms();
+  if (sms <= 0) return GMG_ECUDA;
+  int bps = 0;
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, arbw_kernel_ptr(G.t32 != 0, G.ntypes >= 2), 32 * L.wpb,
+                                                    L.smem) != cudaSuccess)
+    return GMG_ECUDA;
+  bps = std::max(bps, 1);
+  const int64_t need = (std::max<int64_t>(K, 1) + L.wpb - 1) / L.wpb;
+  L.grid = (int)std::min<int64_t>(need, (int64_t)sms * bps);
+  L.slots = (int64_t)L.grid * L.wpb;
+  A.link = g->linkid;
+  return GMG_OK;
 }
+
+// Either arbitrated kernel, by accelerator count.
+struct ArbPlan {
+  bool wide = false;
+  ArbParams A;
+  ArbWParams AW;
+};
+
+int plan_arb_any(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbPlan& Q) {
+  Q.wide = g->dg.D > 32;
+  return Q.wide ? plan_arbw(g, K, o, L, Q.AW) : plan_arb(g, K, o, L, Q.A);
+}
+
+cudaError_t launch_arb_any(const gmg* g, Launch& L, ArbPlan& Q, const int32_t* pre_status, cudaStream_t st) {
+  if (Q.wide) {
+    Q.AW.P = L.P;
+    Q.AW.pre_status = pre_status;
+    return launch_arbw(g->dg.t32 != 0, g->dg.ntypes >= 2, Q.AW, L.grid, 32 * L.wpb, L.smem, st);
+  }
+  Q.A.P = L.P;
+  Q.A.pre_status = pre_status;
+  return launch_arb(g->dg.t32 != 0, g->dg.ntypes >= 2, Q.A, L.grid, 32 * L.wpb, L.smem, st);
+}
+
 
 struct BasePlan {
   size_t off_row, off_rb, off_fb, off_status, off_res, off_peak, off_creq, off_cktime,
@@ -774,8 +850,8 @@ size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
   if (!g || K < 0) return 0;
   Launch L;
   if (arbitrated(opts)) {
-    ArbParams A;
-    if (plan_arb(g, K, opts, L, A)) return 0;
+    ArbPlan Q;
+    if (plan_arb_any(g, K, opts, L, Q)) return 0;
   } else if (plan_launch(g, K, opts, false, L)) {
     return 0;
   }
@@ -790,9 +866,9 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   if (K == 0) return GMG_OK;
   if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
   Launch L;
-  ArbParams A;
+  ArbPlan Q;
   const bool arb = arbitrated(opts);
-  rc = arb ? plan_arb(g, K, opts, L, A) : plan_launch(g, K, opts, false, L);
+  rc = arb ? plan_arb_any(g, K, opts, L, Q) : plan_launch(g, K, opts, false, L);
   if (rc) return rc;
   if (!d_scratch || !aligned(d_scratch, 256) ||
       scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
@@ -804,7 +880,7 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   P.K = K;
   P.scratch = static_cast<uint8_t*>(d_scratch);
   const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = arb ? launch_arb_batch(g, L, A, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
+  cudaError_t e = arb ? launch_arb_any(g, L, Q, nullptr, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 
@@ -855,9 +931,9 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   if (K == 0) return GMG_OK;
   if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
   Launch L;
-  ArbParams A;
+  ArbPlan Q;
   const bool arb = arbitrated(opts);
-  rc = arb ? plan_arb(g, K, opts, L, A) : plan_launch(g, K, opts, false, L);
+  rc = arb ? plan_arb_any(g, K, opts, L, Q) : plan_launch(g, K, opts, false, L);
   if (rc) return rc;
   // As many warp slots as the fixed buffer holds (each warp then takes more
   // candidates in turn); a graph whose single slot does not fit is refused.
@@ -866,7 +942,7 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   if (fit < L.wpb) {
     sim_opts_t one = opts ? *opts : sim_opts_t{};
     one.warps_per_block = 1;
-    rc = arb ? plan_arb(g, K, &one, L, A) : plan_launch(g, K, &one, false, L);
+    rc = arb ? plan_arb_any(g, K, &one, L, Q) : plan_launch(g, K, &one, false, L);
     if (rc) return rc;
   }
   L.grid = (int)std::min<int64_t>(L.grid, fit / L.wpb);
@@ -880,7 +956,7 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   P.K = K;
   P.scratch = scratch;
   const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  const cudaError_t e = arb ? launch_arb_batch(g, L, A, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
+  const cudaError_t e = arb ? launch_arb_any(g, L, Q, nullptr, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 
@@ -952,8 +1028,8 @@ void base_destroy(gmg_base_t* b) { delete b; }
 // Arbitrated incremental candidates: [moved rows K x ld | move statuses K | slots].
 static size_t arb_inc_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts, size_t* off_status, size_t* off_slots) {
   Launch L;
-  ArbParams A;
-  if (plan_arb(g, K, opts, L, A)) return 0;
+  ArbPlan Q;
+  if (plan_arb_any(g, K, opts, L, Q)) return 0;
   const size_t ld = align_up((size_t)std::max(g->dg.n, 1), 16);
   const size_t os = align_up((size_t)K * ld, 256);
   const size_t oz = os + align_up(4 * (size_t)std::max(K, 1), 256);
@@ -985,14 +1061,14 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
     const size_t need = arb_inc_bytes(g, K, opts, &os, &oz);
     if (need == 0) {
       Launch L0;
-      ArbParams A0;
-      const int prc = plan_arb(g, K, opts, L0, A0);
+      ArbPlan Q0;
+      const int prc = plan_arb_any(g, K, opts, L0, Q0);
       return prc ? prc : GMG_EINVAL;
     }
     if (!d_scratch || !aligned(d_scratch, 256) || scratch_bytes < need) return GMG_EWS;
     Launch L;
-    ArbParams A;
-    rc = plan_arb(g, K, opts, L, A);
+    ArbPlan Q;
+    rc = plan_arb_any(g, K, opts, L, Q);
     if (rc) return rc;
     uint8_t* sc = static_cast<uint8_t*>(d_scratch);
     const int32_t ld = b->db.ld;
@@ -1006,8 +1082,8 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
     P.ld = ld;
     P.K = K;
     P.scratch = sc + oz;
-    A.pre_status = reinterpret_cast<const int32_t*>(sc + os);
-    return launch_arb_batch(g, L, A, st) == cudaSuccess ? GMG_OK : GMG_ECUDA;
+    return launch_arb_any(g, L, Q, reinterpret_cast<const int32_t*>(sc + os), st) == cudaSuccess ? GMG_OK
+                                                                                                : GMG_ECUDA;
   }
   Launch L;
   rc = plan_launch(g, K, opts, true, L);
