@@ -186,8 +186,8 @@ def prepare(config: int, rank: int, device, cap=None, arbitrated=False, structur
     p.wl = wl
     p.arb = arbitrated
     p.structured = structured
-    if arbitrated and (wl.n_full == 0 or wl.desc.n_dev > 32):
-        raise SystemExit("--arbitrated needs a workload of full placements on at most 32 accelerators")
+    if arbitrated and wl.desc.n_dev > 256:
+        raise SystemExit("--arbitrated needs at most 256 accelerators")
     if structured and (wl.n_full == 0 or wl.moves is not None):
         raise SystemExit("--placements structured needs a workload of full placements only")
     p.g = G.gmg_create(wl.desc, device=device)
@@ -240,7 +240,7 @@ def run_step(p, kernel_events=None):
         o = _views(p.out, p.n_full, p.K)
         if kernel_events and not p.n_full:
             kernel_events[0].record()
-        G.sim_incremental(p.g, b, *p.moves, out=o, scratch=p.scratch)
+        G.sim_incremental(p.g, b, *p.moves, out=o, scratch=p.scratch, arbitrated=p.arb)
         if kernel_events and not p.n_full:
             kernel_events[1].record()
         p._base = b  # keep alive until the stream has used it
@@ -771,7 +771,8 @@ def main():
     pk = peaks()
     # the timed kernel: the full-placement simulation if the batch has one,
     # else the incremental one
-    kern = ("sim_arb_kernel" if p.arb else "sim_full_kernel") if p.n_full else "sim_inc_kernel"
+    arb_kern = "sim_arb_kernel" if wl.desc.n_dev <= 32 else "sim_arbw_kernel"
+    kern = (arb_kern if p.arb else "sim_full_kernel") if p.n_full else (arb_kern if p.arb else "sim_inc_kernel")
     kcand = p.n_full if p.n_full else p.n_inc
     out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
     if p.n_full:
