@@ -225,6 +225,23 @@ def test_transfer_tables_obey_the_arbitration_rule(seed):
     _check_table(d, place, r)
 
 
+@pytest.mark.parametrize("seed,D", [(0, 40), (1, 64)])
+def test_transfer_tables_obey_the_rule_on_many_accelerators(seed, D):
+    """The same rule checks with more accelerators than a warp has lanes
+    (the library's wide arbitrated kernel), with pair-shared links."""
+    g = np.random.default_rng(200 + seed)
+    d = random_desc(300 + seed, 240, D, dur_hi=40, bytes_hi=600)
+    d.bw[:] = g.integers(5, 60, D * D)
+    d.lat[:] = g.integers(1, 8, D * D)
+    a, b = np.meshgrid(np.arange(D), np.arange(D), indexing="ij")
+    d.link_id = (np.minimum(a, b) * D + np.maximum(a, b)).astype(np.int32).reshape(-1)
+    # few accelerators per op neighbourhood so that transfers compete
+    place = g.integers(0, 6, 240) * (D // 6)
+    r = _arb(d, place)
+    assert r["status"] == 0 and r["transfers"].shape[0] > 50
+    _check_table(d, place, r)
+
+
 def test_rejects_bad_link_ids():
     d = mk([[], [0]], [1, 1], n_dev=2)
     d.link_id = np.array([0, 4, 1, 0], np.int32)   # 4 >= D*D
