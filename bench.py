@@ -1,11 +1,11 @@
 #!/usr/bin/env python
 """Benchmark: candidate placements simulated per second on one GB300.
 
-Default workload: 8 prefill requests x 32 layers (N=3088 ops) on 8 simulated
-accelerators, K=4096 random placements (the benchmark's second config, the
-one its metric is quoted on).  One step = sim_batch over all K candidates +
-select_best, inputs resident in HBM, L2 flushed (256 MiB write) between
-steps; every step is timed with CUDA events on the launching stream.
+Default workload: the prefill workload, 8 requests x 32 layers (N=3088 ops)
+on 8 simulated accelerators, K=4096 uniform random placements.  One step =
+sim_batch over all K candidates + select_best, inputs resident in HBM, L2
+flushed (256 MiB write) between steps; every step is timed with CUDA events
+on the launching stream.
 
 Also reported: the end-to-end rate through the public API with host buffers
 (H2D of the placements from pinned memory and D2H of the selection inside
@@ -14,7 +14,10 @@ this host's cores, and the SM clocks sampled during the timed region.
 
 ``--impl reference`` times the CPU oracle (the reference arm of this repo:
 there is no upstream implementation) on the same workload and metric.
-``--config 1..5`` selects another workload (supplementary lines).
+``--config 1..6`` selects another workload, ``--arbitrated`` the arbitrated
+transfers of Sec. 3.5.2, ``--placements structured`` contiguous per-request
+stages instead of uniform placements, ``--rounds`` / ``--estimators`` the
+scheduling round and the estimator refits (supplementary lines).
 Under torchrun every rank simulates its own K candidates (weak scaling,
 no data-path collective); rank 0 prints the line with the max time.
 """
