@@ -169,6 +169,17 @@ def test_tick_stepped_arbitration_equals_oracle(block):
         assert r["req_done"].tolist() == want["req_done"], seed
 
 
+def test_tick_stepped_arbitration_equals_oracle_on_larger_graphs():
+    for seed in range(1000, 1040):
+        d, place = _rand(seed, n_hi=40, d_hi=6, dur_hi=10)
+        rd, st, fi, xs = refsim.tick_sim_arb(d, place)
+        r = _arb(d, place)
+        assert r["finish"].tolist() == fi and r["start"].tolist() == st and r["ready"].tolist() == rd, seed
+        assert _xt(r) == [(x["p"], x["e"], x["intent"], x["start"], x["done"]) for x in xs], seed
+        want = refsim.summarize(d, place, st, fi, transfers=xs)
+        assert r["peak"].tolist() == want["peak"] and r["viol_time"] == want["viol_time"], seed
+
+
 def _check_table(d, place, r):
     """Every property the arbitration rule fixes, on one transfer table
     (transfers of nonzero length only)."""
