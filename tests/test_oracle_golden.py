@@ -1,9 +1,11 @@
 """Hand-derived worked examples (tests/golden/*.json, each with the passages
-it follows and its step-by-step derivation) pin the oracle's arithmetic."""
+it follows and its step-by-step derivation) pin the oracle's arithmetic,
+with pure-latency or (transfer_mode 1) arbitrated transfers."""
 import glob
 import json
 import os
 
+import numpy as np
 import pytest
 
 from helpers import mk, row
@@ -21,7 +23,12 @@ def test_golden(path):
         d = mk(g["preds"], g["dur"], g["out_bytes"], n_dev=g["n_dev"], bw=g["bw"], lat=g["lat"],
                release=g.get("release"), avail0=g.get("avail0"), req_id=g.get("req_id"),
                deadline=g.get("deadline"), cap=case["cap"])
-        r = O.simulate(d, row(fx["place"]))
+        arb = g.get("transfer_mode", 0) == 1
+        if g.get("link_id") is not None:
+            d.link_id = np.asarray(g["link_id"], np.int32)
+        r = O.simulate(d, row(fx["place"]), arbitrated=arb)
+        if "transfers" in case:
+            assert r["transfers"].tolist() == case["transfers"]
         assert r["ready"].tolist() == case["ready"]
         assert r["start"].tolist() == case["start"]
         assert r["finish"].tolist() == case["finish"]
