@@ -3,7 +3,9 @@
 Usage: ``python oracle/build.py``.  Produces ``oracle/liboracle_sim.so`` next
 to this file.  Plain C++17, no CUDA, nothing shared with the product library.
 """
+import hashlib
 import os
+import platform
 import subprocess
 import sys
 
@@ -12,13 +14,31 @@ SRC = os.path.join(HERE, "sim_ref.cpp")
 OUT = os.path.join(HERE, "liboracle_sim.so")
 
 
+FLAGS = ["-O2", "-std=c++17", "-shared", "-fPIC", "-pthread", "-Wall"]
+STAMP = OUT + ".stamp"
+
+
+def stamp() -> str:
+    """SHA-256 over the source, the flags and the machine type: the library is
+    rebuilt whenever it differs from the stamp stored beside it."""
+    h = hashlib.sha256()
+    with open(SRC, "rb") as f:
+        h.update(f.read())
+    h.update(" ".join(FLAGS).encode() + platform.machine().encode())
+    return h.hexdigest()
+
+
 def build(force: bool = False) -> str:
-    if not force and os.path.exists(OUT) and os.path.getmtime(OUT) >= os.path.getmtime(SRC):
-        return OUT
+    want = stamp()
+    if not force and os.path.exists(OUT) and os.path.exists(STAMP):
+        with open(STAMP) as f:
+            if f.read().strip() == want:
+                return OUT
     tmp = OUT + ".tmp%d" % os.getpid()
-    cmd = ["g++", "-O2", "-std=c++17", "-shared", "-fPIC", "-pthread", "-Wall", SRC, "-o", tmp]
-    subprocess.check_call(cmd)
+    subprocess.check_call(["g++"] + FLAGS + [SRC, "-o", tmp])
     os.replace(tmp, OUT)
+    with open(STAMP, "w") as f:
+        f.write(want + "\n")
     return OUT
 
 

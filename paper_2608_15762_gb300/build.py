@@ -1,9 +1,17 @@
 """Build ``libgmgsim.so`` (the C-ABI library) for sm_103a with nvcc, in-tree.
 
-The two translation units compile in parallel, then link into one shared
-library next to this file.  ``python -m paper_2608_15762_gb300.build``.
+The translation units compile in parallel, then link into one shared library
+next to this file.  ``python -m paper_2608_15762_gb300.build``.
+
+A rebuild happens when the library is missing or when the stamp stored beside
+it (a SHA-256 over every source and header, the nvcc flags, the nvcc version
+and the host machine type) differs from the current one; file times are not
+consulted, so a library copied in from elsewhere is never trusted on its
+modification time alone.
 """
+import hashlib
 import os
+import platform
 import subprocess
 import sys
 
@@ -23,17 +31,42 @@ def nvcc() -> str:
     return cand if os.path.exists(cand) else "nvcc"
 
 
-def _stale() -> bool:
-    if not os.path.exists(OUT):
+STAMP = OUT + ".stamp"
+
+
+def _nvcc_version() -> str:
+    try:
+        return subprocess.run([nvcc(), "--version"], capture_output=True, text=True).stdout
+    except OSError:
+        return "no nvcc"
+
+
+def stamp() -> str:
+    """SHA-256 over the sources, headers, flags, compiler version and machine."""
+    h = hashlib.sha256()
+    for name in SOURCES + HEADERS:
+        with open(os.path.join(CSRC, name), "rb") as f:
+            h.update(name.encode() + b"\0" + f.read() + b"\0")
+    h.update(" ".join(ARCH + FLAGS).encode())
+    h.update(_nvcc_version().encode())
+    h.update(platform.machine().encode())
+    return h.hexdigest()
+
+
+def _stale(want: str) -> bool:
+    if not os.path.exists(OUT) or not os.path.exists(STAMP):
         return True
-    t = os.path.getmtime(OUT)
-    deps = [os.path.join(CSRC, s) for s in SOURCES + HEADERS] + [os.path.abspath(__file__)]
-    return any(os.path.getmtime(d) > t for d in deps)
+    with open(STAMP) as f:
+        return f.read().strip() != want
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
-    if not force and not _stale():
+    want = stamp()
+    if not force and not _stale(want):
+        if verbose:
+            print("libgmgsim.so up to date (stamp %s)" % want[:12])
         return OUT
+    print("building libgmgsim.so (stamp %s)" % want[:12], file=sys.stderr)
     objdir = os.path.join(HERE, "_build")
     os.makedirs(objdir, exist_ok=True)
     procs, objs = [], []
@@ -53,6 +86,8 @@ def build(force: bool = False, verbose: bool = False) -> str:
     tmp = OUT + ".tmp%d" % os.getpid()
     subprocess.check_call([nvcc()] + ARCH + ["-shared", "-o", tmp] + objs)
     os.replace(tmp, OUT)
+    with open(STAMP, "w") as f:
+        f.write(want + "\n")
     return OUT
 
 

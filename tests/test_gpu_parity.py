@@ -1,5 +1,9 @@
 """GPU parity: the CUDA path through the C ABI against the CPU oracle, bit for
 bit on every output field (all times and sizes are int64)."""
+import glob
+import json
+import os
+
 import numpy as np
 import pytest
 
@@ -92,27 +96,40 @@ def test_bad_device_rows_and_empty_graph():
     assert oe.status.cpu().tolist() == [0] * 4 and oe.score.cpu().tolist() == [0] * 4
 
 
-def test_golden_examples_on_gpu():
-    import json, glob, os
-    for path in sorted(glob.glob(os.path.join(os.path.dirname(__file__), "golden", "*.json"))):
-        fx = json.load(open(path))
-        gr = fx["graph"]
-        for case in fx["cases"]:
-            d = mk(gr["preds"], gr["dur"], gr["out_bytes"], n_dev=gr["n_dev"], bw=gr["bw"],
-                   lat=gr["lat"], release=gr.get("release"), avail0=gr.get("avail0"),
-                   req_id=gr.get("req_id"), deadline=gr.get("deadline"), cap=case["cap"])
-            g = G.gmg_create(d)
-            rows = row(fx["place"])[None, :]
-            tk = torch.tensor([0], dtype=torch.int32, device="cuda")
-            out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk).to_numpy()
-            assert out["trace_start"][0].tolist() == case["start"]
-            assert out["trace_finish"][0].tolist() == case["finish"]
-            assert out["peak"][0].tolist() == case["peak"]
-            assert out["makespan"][0] == case["makespan"] and out["score"][0] == case["score"]
-            viol = None if not out["viol_flag"][0] else [int(out["viol_time"][0]),
-                                                         int(out["viol_op"][0]),
-                                                         int(out["viol_dev"][0])]
-            assert viol == case["viol"]
+GOLDEN = sorted(glob.glob(os.path.join(os.path.dirname(__file__), "golden", "*.json")))
+
+
+@pytest.mark.parametrize("path", GOLDEN, ids=[os.path.basename(p) for p in GOLDEN])
+def test_golden_examples_on_gpu(path):
+    """Each hand-derived worked example, with the transfer model and link
+    table the fixture names, through the C ABI: start/finish of every op,
+    peaks, makespan, score, SLA, request completions and the first violation."""
+    with open(path) as f:
+        fx = json.load(f)
+    gr = fx["graph"]
+    arb = gr.get("transfer_mode", 0) == 1
+    for case in fx["cases"]:
+        d = mk(gr["preds"], gr["dur"], gr["out_bytes"], n_dev=gr["n_dev"], bw=gr["bw"],
+               lat=gr["lat"], release=gr.get("release"), avail0=gr.get("avail0"),
+               req_id=gr.get("req_id"), deadline=gr.get("deadline"), cap=case["cap"])
+        if gr.get("link_id") is not None:
+            d.link_id = np.asarray(gr["link_id"], np.int32)
+        g = G.gmg_create(d)
+        rows = row(fx["place"])[None, :]
+        tk = torch.tensor([0], dtype=torch.int32, device="cuda")
+        out = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk,
+                          arbitrated=arb).to_numpy()
+        assert out["status"][0] == 0
+        assert out["trace_start"][0].tolist() == case["start"]
+        assert out["trace_finish"][0].tolist() == case["finish"]
+        assert out["peak"][0].tolist() == case["peak"]
+        assert out["makespan"][0] == case["makespan"] and out["score"][0] == case["score"]
+        assert out["sla_miss"][0] == case["sla_miss"]
+        assert out["req_done"][0].tolist() == case["req_done"]
+        viol = None if not out["viol_flag"][0] else [int(out["viol_time"][0]),
+                                                     int(out["viol_op"][0]),
+                                                     int(out["viol_dev"][0])]
+        assert viol == case["viol"]
 
 
 def test_queue_capacity_status():
