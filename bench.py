@@ -1,16 +1,22 @@
 #!/usr/bin/env python
 """Benchmark: candidate placements simulated per second on one GB300.
 
-Default workload: the prefill workload, 8 requests x 32 layers (N=3088 ops)
-on 8 simulated accelerators, K=4096 uniform random placements.  One step =
-sim_batch over all K candidates + select_best, inputs resident in HBM, L2
-flushed (256 MiB write) between steps; every step is timed with CUDA events
-on the launching stream.
+Default workload: the large workload -- 128 tenants with 16/32/80-layer
+decoder graphs and Poisson request arrivals (N=213,568 ops) on 256 simulated
+accelerators, K=65,536 candidates: 32,768 uniform random full placements and
+32,768 incremental candidates of 1-64 moves against a base placement.  One
+step = base_create + sim_incremental over the move lists (side stream)
+concurrently with sim_batch over the full placements (current stream), then
+select_best over both halves; inputs resident in HBM, L2 flushed (256 MiB
+write) between steps; every step and every kernel timed with CUDA events on
+the stream it runs on.
 
 Also reported: the end-to-end rate through the public API with host buffers
-(H2D of the placements from pinned memory and D2H of the selection inside
-the timed region), the dominant kernel's roofline, the CPU oracle timed on
-this host's cores, and the SM clocks sampled during the timed region.
+(H2D of the placements, base row and move lists from pinned memory and D2H
+of the selection inside the timed region), the dominant kernel's roofline
+and every kernel's issue fraction, the CPU oracle timed on this host's cores
+on a sample of each half (scaled to the whole mix), and the SM clocks sampled
+during the timed region.
 
 ``--impl reference`` times the CPU oracle (the reference arm of this repo:
 there is no upstream implementation) on the same workload and metric.
@@ -18,8 +24,10 @@ there is no upstream implementation) on the same workload and metric.
 transfers of Sec. 3.5.2, ``--placements structured`` contiguous per-request
 stages instead of uniform placements, ``--rounds`` / ``--estimators`` the
 scheduling round and the estimator refits (supplementary lines).
-Under torchrun every rank simulates its own K candidates (weak scaling,
-no data-path collective); rank 0 prints the line with the max time.
+Under torchrun the workload's candidates are partitioned: every rank takes a
+contiguous block of each half (strong scaling, no data-path collective; the
+graph and the base row are replicated); rank 0 prints the line with the max
+time, each candidate counted once.
 """
 import argparse
 import hashlib
@@ -179,7 +187,11 @@ def rows_of(wl, ks, structured=False):
     return wl.structured_full_rows(ks) if structured else wl.full_rows(ks)
 
 
-def prepare(config: int, rank: int, device, cap=None, arbitrated=False, structured=False):
+def prepare(config: int, rank: int, world: int, device, cap=None, arbitrated=False, structured=False):
+    """Inputs of one rank, resident on its device: its contiguous block of
+    the full placements and of the incremental move lists (the base row and
+    the graph are replicated), outputs, two scratch buffers (the two halves
+    run on two streams) and the side stream."""
     import numpy as np
     import torch
     from paper_2608_15762_gb300 import gmgsim as G
@@ -194,31 +206,35 @@ def prepare(config: int, rank: int, device, cap=None, arbitrated=False, structur
     if structured and (wl.n_full == 0 or wl.moves is not None):
         raise SystemExit("--placements structured needs a workload of full placements only")
     p.g = G.gmg_create(wl.desc, device=device)
-    p.n_full = wl.n_full
-    p.n_inc = 0 if wl.moves is None else wl.moves.n_cand
-    moves = wl.moves
+    n_full = wl.n_full
+    n_inc = 0 if wl.moves is None else wl.moves.n_cand
     if cap is not None:
         # profiling captures: the first `cap` candidates of each half
-        p.n_full = min(p.n_full, cap)
-        if p.n_inc > cap:
-            moves = moves.subset(np.arange(cap))
-            p.n_inc = cap
+        n_full, n_inc = min(n_full, cap), min(n_inc, cap)
+    p.n_full_total, p.n_inc_total = n_full, n_inc
+    p.full_ks = G.shard_block(rank, world, n_full)
+    p.inc_ks = G.shard_block(rank, world, n_inc)
+    p.n_full, p.n_inc = len(p.full_ks), len(p.inc_ks)
     p.K = p.n_full + p.n_inc
+    p.to_global = G.two_half_index(p.n_full, p.full_ks.start, n_full, p.inc_ks.start)
     p.host_place = None
     if p.n_full:
-        ks = range(p.n_full) if cap is not None else G.shard_range(rank, p.n_full)
-        rows = rows_of(wl, ks, structured)
+        rows = rows_of(wl, p.full_ks, structured)
         p.host_place = torch.from_numpy(rows).pin_memory()
         p.place = p.host_place.to(device)
     if p.n_inc:
+        moves = wl.moves.subset(p.inc_ks)
         p.host_base = torch.from_numpy(np.ascontiguousarray(wl.base_place)).pin_memory()
         p.base_place = p.host_base.to(device)
         p.host_moves = [torch.from_numpy(np.ascontiguousarray(a)).pin_memory()
                         for a in (moves.off, moves.op, moves.dev)]
         p.moves = [t.to(device) for t in p.host_moves]
-    p.out = G.SimOut.empty(p.K, wl.desc.n_dev, wl.desc.n_req, device)
+    p.out = G.SimOut.empty(max(p.K, 1), wl.desc.n_dev, wl.desc.n_req, device)
     p.scratch = G.Scratch(device)
+    p.scratch_inc = G.Scratch(device)
+    p.side = torch.cuda.Stream(device)
     p.best = torch.empty(2, dtype=torch.int64, device=device)
+    p._base = None
     return p
 
 
@@ -227,27 +243,42 @@ def _views(out, a, b):
     return G.SimOut(**{k: (None if v is None else v[a:b]) for k, v in out.__dict__.items()})
 
 
-def run_step(p, kernel_events=None):
-    """One pass of the hot path over the batch; returns kernel launches."""
+def run_step(p, ev=None):
+    """One pass of the hot path over this rank's batch: the base snapshot and
+    the incremental candidates on the side stream, the full placements on the
+    current stream (the two run concurrently; the base's single warp is
+    launched first so that it is not queued behind the full grid), then the
+    selection over both halves.  ``ev``: optional dict of CUDA event pairs
+    recorded around each kernel on the stream it runs on.  Returns the
+    number of this library's kernel launches."""
+    import torch
     from paper_2608_15762_gb300 import gmgsim as G
     launches = 0
+    main = torch.cuda.current_stream()
+    if p.n_inc:
+        p.side.wait_stream(main)
+        with torch.cuda.stream(p.side):
+            if ev:
+                ev["base"][0].record()
+            b = G.base_create(p.g, p.base_place, stream=p.side)
+            if ev:
+                ev["base"][1].record()
+                ev["inc"][0].record()
+            G.sim_incremental(p.g, b, *p.moves, out=_views(p.out, p.n_full, p.K), scratch=p.scratch_inc,
+                              arbitrated=p.arb, stream=p.side)
+            if ev:
+                ev["inc"][1].record()
+        p._base = b  # keep alive until the stream has used it
+        launches += 2 if not p.arb else 3
     if p.n_full:
-        if kernel_events:
-            kernel_events[0].record()
+        if ev:
+            ev["full"][0].record()
         G.sim_batch(p.g, p.place, out=_views(p.out, 0, p.n_full), scratch=p.scratch, arbitrated=p.arb)
-        if kernel_events:
-            kernel_events[1].record()
+        if ev:
+            ev["full"][1].record()
         launches += 1
     if p.n_inc:
-        b = G.base_create(p.g, p.base_place)
-        o = _views(p.out, p.n_full, p.K)
-        if kernel_events and not p.n_full:
-            kernel_events[0].record()
-        G.sim_incremental(p.g, b, *p.moves, out=o, scratch=p.scratch, arbitrated=p.arb)
-        if kernel_events and not p.n_full:
-            kernel_events[1].record()
-        p._base = b  # keep alive until the stream has used it
-        launches += 2
+        main.wait_stream(p.side)
     G.select_best(p.out, p.K, best=p.best)
     launches += 2
     return launches
@@ -275,55 +306,75 @@ def h2d_bytes(p):
     return b
 
 
-def cpu_baseline(wl, min_s=10.0, arbitrated=False, structured=False):
-    """The CPU oracle as it stands on this host's cores, on a bounded sample of
-    the same workload: up to ~3e8 op-events of candidates, repeated as whole
-    batches until at least min_s seconds of wall time."""
+def oracle_sample(wl, k_full, k_inc, nthreads, arbitrated=False, structured=False):
+    """Callables that run the CPU oracle, as it stands, on the first k_full
+    full placements and the first k_inc incremental candidates of the
+    workload (either may be 0)."""
+    from oracle import oracle as O
+    from paper_2608_15762_gb300.workloads import Moves
+    runs = []
+    if k_full:
+        rows = rows_of(wl, range(k_full), structured)
+        runs.append(("full", k_full, wl.n_full,
+                     lambda nt=nthreads, r=rows: O.simulate_batch(wl.desc, r, nthreads=nt, arbitrated=arbitrated),
+                     lambda k1, r=rows: O.simulate_batch(wl.desc, r[:k1], nthreads=1, arbitrated=arbitrated)))
+    if k_inc:
+        m = wl.moves
+        mv = Moves(m.off[:k_inc + 1].copy(), m.op[:m.off[k_inc]], m.dev[:m.off[k_inc]])
+        runs.append(("incremental", k_inc, m.n_cand,
+                     lambda nt=nthreads, v=mv: O.incremental_batch(wl.desc, wl.base_place, v, nthreads=nt,
+                                                                 arbitrated=arbitrated),
+                     lambda k1, v=mv: O.incremental_batch(wl.desc, wl.base_place, v.subset(range(k1)),
+                                                          nthreads=1, arbitrated=arbitrated)))
+    return runs
+
+
+def cpu_baseline(wl, min_s=10.0, arbitrated=False, structured=False, ev_budget=1.2e8):
+    """The CPU oracle as it stands on this host's cores, on a bounded sample
+    of each half of the workload (up to ~ev_budget op-events of candidates per
+    half, whole sample passes repeated until min_s seconds in all), scaled to
+    the workload's whole candidate mix: value = K / sum over halves of
+    (candidates of the half x measured seconds per candidate)."""
     from oracle import oracle as O
     nt = O.hw_threads()
-    budget = max(16, int(3e8 // max(wl.desc.n_ops, 1)))
-    if wl.n_full:
-        k = min(wl.n_full, budget)
-        rows = rows_of(wl, range(k), structured)
-
-        def run():
-            O.simulate_batch(wl.desc, rows, nthreads=nt, arbitrated=arbitrated)
-        what = "%d of %d full%s placements%s" % (k, wl.n_full, " structured" if structured else "",
-                                               ", arbitrated transfers" if arbitrated else "")
-    else:
-        from paper_2608_15762_gb300.workloads import Moves
-        k = min(wl.moves.n_cand, budget)
-        mv = Moves(wl.moves.off[:k + 1].copy(), wl.moves.op[:wl.moves.off[k]], wl.moves.dev[:wl.moves.off[k]])
-
-        def run():
-            O.incremental_batch(wl.desc, wl.base_place, mv, nthreads=nt)
-        what = "%d of %d incremental candidates" % (k, wl.moves.n_cand)
-    reps = 0
-    t0 = time.perf_counter()
-    while True:
-        run()
-        reps += 1
-        dt = time.perf_counter() - t0
-        if dt >= min_s:
-            break
-    value = reps * k / dt
-    # one core: a smaller sample of the same candidates, about 3 s of work
-    k1 = int(max(1, min(k, 3.0 * value / nt)))
-    t1 = time.perf_counter()
-    if wl.n_full:
-        O.simulate_batch(wl.desc, rows[:k1], nthreads=1, arbitrated=arbitrated)
-    else:
-        O.incremental_batch(wl.desc, wl.base_place, mv.subset(range(k1)), nthreads=1)
-    dt1 = time.perf_counter() - t1
-    return {"value": value, "unit": UNIT, "cores": nt, "kind": "oracle",
-            "sample": "%s, %d pass%s" % (what, reps, "" if reps == 1 else "es"), "seconds": round(dt, 3),
-            "op_events_per_s": reps * k * wl.desc.n_ops / dt if wl.n_full else None,
-            "single_core": {"value": k1 / dt1, "unit": UNIT, "cores": 1,
-                            "sample": "the first %d of those candidates, one pass" % k1}}
+    budget = max(16, int(ev_budget // max(wl.desc.n_ops, 1)))
+    n_inc = 0 if wl.moves is None else wl.moves.n_cand
+    runs = oracle_sample(wl, min(wl.n_full, budget), min(n_inc, budget), nt, arbitrated, structured)
+    total_s, total_s1, parts, wall = 0.0, 0.0, [], 0.0
+    for name, k, k_all, run, run1 in runs:
+        reps, t0 = 0, time.perf_counter()
+        while True:
+            run()
+            reps += 1
+            dt = time.perf_counter() - t0
+            if dt >= min_s / len(runs):
+                break
+        wall += dt
+        spc = dt / (reps * k)
+        # one core: a smaller sample of the same candidates, about 1.5 s of work
+        k1 = int(max(1, min(k, 1.5 / (spc * nt))))
+        t1 = time.perf_counter()
+        run1(k1)
+        spc1 = (time.perf_counter() - t1) / k1
+        total_s += k_all * spc
+        total_s1 += k_all * spc1
+        parts.append("%s: %d of %d candidates x %d pass%s, %.4g s/candidate (1 core: first %d, %.4g s)" % (
+            name, k, k_all, reps, "" if reps == 1 else "es", spc, k1, spc1))
+    K = sum(r[2] for r in runs)
+    scaled = any(r[1] < r[2] for r in runs)
+    return {"value": K / total_s, "unit": UNIT, "cores": nt, "kind": "oracle",
+            "sample": "; ".join(parts) + ("; scaled to all %d candidates" % K if scaled else ""),
+            "scaled": scaled, "seconds": round(wall, 3),
+            "op_events_per_s": wl.n_full * wl.desc.n_ops / total_s if wl.n_full and not n_inc else None,
+            "single_core": {"value": K / total_s1, "unit": UNIT, "cores": 1,
+                            "sample": "smaller samples of the same candidates, one pass each"}}
 
 
 def reference_arm(args):
-    """--impl reference: time the CPU oracle on the host cores."""
+    """--impl reference: time the CPU oracle, as it stands, on the host cores,
+    on the same workload, metric and unit.  Each step is a bounded sample of
+    the workload with the workload's own mix of full placements and
+    incremental candidates (about 3e7 op-events of candidates per step)."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
@@ -331,18 +382,16 @@ def reference_arm(args):
     from paper_2608_15762_gb300 import workloads as W
     wl = W.make_workload(args.config)
     nt = O.hw_threads()
-    k = min(wl.n_full or wl.moves.n_cand, max(16, int(3e7 // max(wl.desc.n_ops, 1))))
-    if wl.n_full:
-        rows = rows_of(wl, range(k), args.placements == "structured")
+    n_inc = 0 if wl.moves is None else wl.moves.n_cand
+    K = wl.n_full + n_inc
+    k = min(K, max(16, int(3e7 // max(wl.desc.n_ops, 1))))
+    kf = min(wl.n_full, (k * wl.n_full + K - 1) // K)
+    ki = min(n_inc, k - kf) if n_inc else 0
+    runs = oracle_sample(wl, kf, ki, nt, args.arbitrated, args.placements == "structured")
 
-        def step():
-            O.simulate_batch(wl.desc, rows, nthreads=nt, arbitrated=args.arbitrated)
-    else:
-        mv = W.Moves(wl.moves.off[:k + 1].copy(), wl.moves.op[:wl.moves.off[k]],
-                     wl.moves.dev[:wl.moves.off[k]])
-
-        def step():
-            O.incremental_batch(wl.desc, wl.base_place, mv, nthreads=nt)
+    def step():
+        for r in runs:
+            r[3]()
     for _ in range(args.warmup):
         step()
     times = []
@@ -351,15 +400,17 @@ def reference_arm(args):
         step()
         times.append(time.perf_counter() - t0)
     ms = 1000 * statistics.mean(times)
-    v = k / (ms / 1000)
+    v = (kf + ki) / (ms / 1000)
     line = {"metric": METRIC, "value": v, "unit": UNIT, "n_gpus": args.gpus, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "strong",
             "vs_baseline": None, "dtype": "int64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": wl.name, "candidates_per_step": k, "n_ops": wl.desc.n_ops,
+            "config": {"workload": wl.name, "candidates_per_step": kf + ki, "full_per_step": kf,
+                       "incremental_per_step": ki, "n_ops": wl.desc.n_ops,
                        "transfers": "arbitrated" if args.arbitrated else "latency",
                        "placements": args.placements},
             "cpu_baseline": {"value": v, "unit": UNIT, "cores": nt, "kind": "oracle",
-                             "sample": "%d candidates per step" % k},
+                             "sample": "the first %d full placements and %d incremental candidates of the "
+                                       "workload per step (its own mix)" % (kf, ki)},
             "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line))
     return 0
@@ -674,7 +725,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--config", type=int, default=2, choices=[1, 2, 3, 4, 5, 6])
+    ap.add_argument("--config", type=int, default=5, choices=[1, 2, 3, 4, 5, 6])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--rounds", action="store_true",
                     help="time scheduling rounds (Algorithm 1) instead of the candidate simulation")
@@ -710,7 +761,7 @@ def main():
 
     from paper_2608_15762_gb300 import build as lib_build
     lib_build.build()
-    p = prepare(args.config, rank, device, cap=args.candidates, arbitrated=args.arbitrated,
+    p = prepare(args.config, rank, world, device, cap=args.candidates, arbitrated=args.arbitrated,
                 structured=args.placements == "structured")
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
 
@@ -720,6 +771,13 @@ def main():
             torch.distributed.barrier()
             torch.cuda.synchronize()
 
+    def max_over_ranks(x):
+        if world == 1:
+            return x
+        t = torch.tensor([x], dtype=torch.float64, device=device)
+        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+        return float(t.item())
+
     for _ in range(args.warmup):
         run_step(p)
     barrier()
@@ -728,94 +786,120 @@ def main():
     time.sleep(0.3)
     step_ev, kern_ev = [], []
     launches = 0
+    names = [n for n, on in (("full", p.n_full), ("base", p.n_inc), ("inc", p.n_inc)) if on]
     for _ in range(args.steps):
         flush.fill_(1)
-        e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+        ke = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in names}
         e[0].record()
-        launches += run_step(p, kernel_events=(e[2], e[3]))
+        launches += run_step(p, ev=ke)
         e[1].record()
         step_ev.append((e[0], e[1]))
-        kern_ev.append((e[2], e[3]))
+        kern_ev.append(ke)
     barrier()
     clocks = sampler.stop()
     step_ms = [a.elapsed_time(b) for a, b in step_ev]
-    kern_ms = [a.elapsed_time(b) for a, b in kern_ev]
-    ms = statistics.mean(step_ms)
-    if world > 1:
-        t = torch.tensor([ms], dtype=torch.float64, device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        ms = float(t.item())
+    kern_ms = {n: statistics.mean(ke[n][0].elapsed_time(ke[n][1]) for ke in kern_ev) for n in names}
+    ms = max_over_ranks(statistics.mean(step_ms))
 
-    # end-to-end through the public API with host buffers
-    for _ in range(2):
-        run_e2e_step(p)
+    # end to end through the public API with host buffers (fewer steps when a
+    # step is long: at least 3, about a minute of work)
+    e2e_steps = max(3, min(args.steps, int(60000 // max(ms, 1e-3))))
+    run_e2e_step(p)
     barrier()
     t0 = time.perf_counter()
-    for _ in range(args.steps):
+    for _ in range(e2e_steps):
         run_e2e_step(p)
     barrier()
-    e2e_ms = 1000 * (time.perf_counter() - t0) / args.steps
-    if world > 1:
-        t = torch.tensor([e2e_ms], dtype=torch.float64, device=device)
-        torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
-        e2e_ms = float(t.item())
+    e2e_ms = max_over_ranks(1000 * (time.perf_counter() - t0) / e2e_steps)
 
     wl = p.wl
-    K, N, D = p.K, wl.desc.n_ops, wl.desc.n_dev
-    inc_events = int(p.out.events[p.n_full:].sum().item()) if p.n_inc else 0
+    N, D = wl.desc.n_ops, wl.desc.n_dev
+    K_all = p.n_full_total + p.n_inc_total      # every rank's candidates, each counted once
+    inc_events = int(p.out.events[p.n_full:p.K].sum().item()) if p.n_inc else 0
+    ev_local = p.n_full * N + inc_events
+    ev_all = ev_local
     if world > 1:
+        t = torch.tensor([ev_local], dtype=torch.int64, device=device)
+        torch.distributed.all_reduce(t)
+        ev_all = int(t.item())
         from paper_2608_15762_gb300 import gmgsim as G
-        best = list(G.select_best_across_ranks(p.best, rank * p.n_full))
+        best = list(G.select_best_across_ranks(p.best, p.to_global))
     else:
         best = p.best.cpu().tolist()
-    value = world * K / (ms / 1000)
-    kms = statistics.mean(kern_ms)
-    # Roofline of the dominant kernel (the candidate simulation).
+        if best[0] >= 0:
+            best[0] = p.to_global(best[0])
+    value = K_all / (ms / 1000)
     pk = peaks()
-    # the timed kernel: the full-placement simulation if the batch has one,
-    # else the incremental one
-    arb_kern = "sim_arb_kernel" if wl.desc.n_dev <= 32 else "sim_arbw_kernel"
-    kern = (arb_kern if p.arb else "sim_full_kernel") if p.n_full else (arb_kern if p.arb else "sim_inc_kernel")
-    kcand = p.n_full if p.n_full else p.n_inc
-    out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
-    if p.n_full:
-        alg_bytes = p.n_full * (W_ld(N) + out_bytes_per_cand)
-    else:
-        alg_bytes = sum(t.numel() * t.element_size() for t in p.host_moves) + p.n_inc * out_bytes_per_cand
-    hbm_gbs = alg_bytes / (kms / 1000) / 1e9
     props = torch.cuda.get_device_properties(device)
     issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
-    ppath = profile_path(kern, wl.name + ("-structured" if p.structured else ""))
-    prof = read_profile(ppath, ARB_SOURCES if p.arb else ())
+    arb_kern = "sim_arb_kernel" if D <= 32 else "sim_arbw_kernel"
+    kname = {"full": arb_kern if p.arb else "sim_full_kernel", "inc": arb_kern if p.arb else "sim_inc_kernel",
+             "base": "sim_base_kernel"}
+    kcount = {"full": p.n_full, "inc": p.n_inc, "base": 1}
+    out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
+    alg_bytes = {"full": p.n_full * (W_ld(N) + out_bytes_per_cand),
+                 "inc": (sum(t.numel() * t.element_size() for t in p.host_moves) + p.n_inc * out_bytes_per_cand)
+                 if p.n_inc else 0,
+                 "base": W_ld(N) + 16 * N}
+    wname = wl.name + ("-structured" if p.structured else "")
+    kernels = {}
+    for n in names:
+        ppath = profile_path(kname[n], wname)
+        prof = read_profile(ppath, ARB_SOURCES if (p.arb and n != "base") else ())
+        kd = {"kernel": kname[n], "launch_ms": kern_ms[n], "units": kcount[n],
+              "hbm_gbs": alg_bytes[n] / (kern_ms[n] / 1000) / 1e9, "inst_per_launch": None, "issue_frac": None,
+              "dram_bytes_per_launch": None}
+        if prof:
+            inst = prof["inst_per_cand"] * kcount[n]
+            kd.update(inst_per_launch=inst, issue_frac=inst / (kern_ms[n] / 1000) / 1e9 / issue_peak,
+                      dram_bytes_per_launch=prof["dram_per_cand"] * kcount[n],
+                      inst_src="%s (ncu on %d units, scaled to %d)" % (os.path.relpath(ppath, ROOT),
+                                                                      prof["captured"], kcount[n]))
+        kernels[n] = kd
+    dom = max(names, key=lambda n: kern_ms[n])
+    kd = kernels[dom]
     roof = {"bound": "alu", "unit": "Ginst/s", "peak": issue_peak,
             "peak_src": "%d SMs x 4 issue slots x %.0f MHz (%s sm_max_mhz)" % (
                 props.multi_processor_count, pk["sm_max_mhz"], pk["src"]),
-            "achieved": None, "frac": None, "traffic": None, "kernel": kern, "kernel_ms": kms}
-    if prof:
-        inst = prof["inst_per_cand"] * kcand
-        ach = inst / (kms / 1000) / 1e9
-        roof.update(achieved=ach, frac=ach / issue_peak, traffic=prof["dram_per_cand"] * kcand,
-                    inst_per_launch=inst, inst_src="%s (ncu on %d candidates, scaled to %d)" % (
-                        os.path.relpath(ppath, ROOT), prof["captured"], kcand))
+            "achieved": None, "frac": None, "traffic": kd["dram_bytes_per_launch"], "kernel": kd["kernel"],
+            "kernel_ms": kd["launch_ms"]}
+    if kd["inst_per_launch"] is not None:
+        ach = kd["inst_per_launch"] / (kd["launch_ms"] / 1000) / 1e9
+        roof.update(achieved=ach, frac=ach / issue_peak, inst_per_launch=kd["inst_per_launch"],
+                    inst_src=kd["inst_src"],
+                    inst_per_op_event=kd["inst_per_launch"] / max(kcount[dom] * N if dom == "full" else 1, 1)
+                    if dom == "full" else None)
+    if all(kernels[n]["inst_per_launch"] is not None for n in names):
+        tot = sum(kernels[n]["inst_per_launch"] for n in names)
+        roof["step"] = {"inst_per_step": tot, "issue_frac": tot / (ms / 1000) / 1e9 / issue_peak,
+                        "inst_per_op_event": tot / max(ev_local, 1),
+                        "note": "every kernel of the step (instructions from the committed ncu summaries) over "
+                                "the whole step time"}
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
-        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+        "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "strong",
         "vs_baseline": None, "dtype": "int64", "data": "synthetic",
         "ms_per_step_best": min(step_ms), "ms_per_step_median": statistics.median(step_ms),
-        "config": {"workload": wl.name, "candidates": K, "n_ops": N, "n_dev": D,
+        "config": {"workload": wl.name, "candidates": K_all, "full_placements": p.n_full_total,
+                   "incremental_candidates": p.n_inc_total, "n_ops": N, "n_dev": D,
                    "transfers": "arbitrated" if p.arb else "latency",
                    "placements": "structured" if p.structured else "uniform",
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
-                   "parallelism": "dp%d over candidates" % world},
+                   "parallelism": "dp%d over candidates (contiguous blocks of each half per rank)" % world},
         # full placements simulate every op; an incremental candidate re-simulates
         # the ops its `events` output counts (read after the timed region)
-        "op_events_per_s": world * (p.n_full * N + inc_events) / (ms / 1000),
+        "op_events_per_s": ev_all / (ms / 1000),
         "roofline": roof,
-        "hbm": {"achieved": hbm_gbs, "peak": pk["hbm_gbs"], "unit": "GB/s",
-                "frac": hbm_gbs / pk["hbm_gbs"], "algorithmic_bytes_per_launch": alg_bytes,
+        "kernels": kernels,
+        "hbm": {"achieved": kd["hbm_gbs"], "peak": pk["hbm_gbs"], "unit": "GB/s",
+                "frac": kd["hbm_gbs"] / pk["hbm_gbs"], "algorithmic_bytes_per_launch": alg_bytes[dom],
+                "dram_bytes_per_candidate": (kd["dram_bytes_per_launch"] / kcount[dom])
+                if kd["dram_bytes_per_launch"] else None,
+                "algorithmic_bytes_per_candidate": alg_bytes[dom] / max(kcount[dom], 1),
                 "note": "placement bytes read + per-candidate outputs written; the kernel is issue/latency-bound"},
-        "e2e": {"value": world * K / (e2e_ms / 1000), "unit": UNIT, "ms_per_step": e2e_ms,
-                "h2d_bytes_per_step": h2d_bytes(p), "d2h_bytes_per_step": 16},
+        "e2e": {"value": K_all / (e2e_ms / 1000), "unit": UNIT, "ms_per_step": e2e_ms, "steps": e2e_steps,
+                "h2d_bytes_per_step": h2d_bytes(p) * world, "d2h_bytes_per_step": 16 * world},
         "gpu_launches": launches,
         "clocks": clocks,
         "best": best,

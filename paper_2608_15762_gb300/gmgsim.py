@@ -440,23 +440,26 @@ def select_best(out: SimOut, K: Optional[int] = None, score_mode: int = 0, best=
     return best
 
 
-def shard_range(rank: int, per_rank: int):
-    """Global candidate indices of one rank when every rank simulates its own
-    block of per_rank candidates (candidates are independent: no exchange)."""
-    return range(rank * per_rank, (rank + 1) * per_rank)
+def shard_block(rank: int, world: int, total: int) -> range:
+    """The contiguous block of ``total`` independent candidates that ``rank``
+    of ``world`` simulates (block sizes differ by at most one; no exchange on
+    the data path)."""
+    return range(total * rank // world, total * (rank + 1) // world)
 
 
-def select_best_across_ranks(best, k_offset: int, group=None):
+def select_best_across_ranks(best, to_global, group=None):
     """Combine the ranks' select_best results into the best over all ranks'
     candidates (lowest global index on ties; (-1, INT64_MAX) if none).
 
-    best: int64[2] (local index or -1, score) on this rank's device.  One
-    all_gather of 16 bytes per rank; call outside any timed region."""
+    best: int64[2] (local index or -1, score) on this rank's device;
+    to_global: maps this rank's local candidate index to its global index.
+    One all_gather of 16 bytes per rank; call outside any timed region."""
     import torch
     import torch.distributed as dist
-    loc = best.detach().to(torch.int64).reshape(2).clone()
+    loc = best.detach().to(torch.int64).reshape(2).cpu().clone()
     if int(loc[0]) >= 0:
-        loc[0] += k_offset
+        loc[0] = int(to_global(int(loc[0])))
+    loc = loc.to(best.device)
     world = dist.get_world_size(group)
     bufs = [torch.empty_like(loc) for _ in range(world)]
     dist.all_gather(bufs, loc, group=group)
@@ -465,6 +468,16 @@ def select_best_across_ranks(best, k_offset: int, group=None):
         return -1, int(np.iinfo(np.int64).max)
     sc, k = min(cands)
     return k, sc
+
+
+def two_half_index(n_full_local: int, full_lo: int, n_full_total: int, inc_lo: int):
+    """Local-to-global candidate index of a rank that simulates full
+    placements [full_lo, full_lo + n_full_local) and incremental candidates
+    [inc_lo, ...) of a workload whose K candidates list all full placements
+    first, then all incremental ones."""
+    def f(k: int) -> int:
+        return full_lo + k if k < n_full_local else n_full_total + inc_lo + (k - n_full_local)
+    return f
 
 
 def ceil_div_host(n: int, d: int) -> int:
