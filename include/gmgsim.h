@@ -156,6 +156,9 @@ typedef struct {
   int32_t uniform_links; /* 1 if every off-diagonal link has the same bw and latency */
   int64_t time_bound;    /* proven upper bound of every simulated time */
   int64_t default_queue_cap;
+  int32_t batched_sweep; /* 1 if the simulation kernels start READY ops in batches (graphs on
+                            more than 32 accelerators whose keys have room for a duration class) */
+  int32_t t32;           /* 1 if the kernels carry times as 32-bit integers (time_bound < 2^31) */
 } gmg_info_t;
 
 /* ---------------------------------------------------------------------- */

@@ -82,6 +82,7 @@ struct DevGmg {
                               // consumer of that predecessor (kSibNone / kSibMany)}
   const uint32_t* cons;
   const uint64_t* root_keys;  // READY keys of ops without predecessors, ascending
+  const uint64_t* root_keys_q;// the same keys with the duration class below them (batched sweep)
   const int64_t* cap;
   const int64_t* base;
   const int64_t* avail0;
@@ -98,7 +99,12 @@ struct DevGmg {
   const int64_t* durt;        // [N*ntypes] duration of op i on type t at i*ntypes + t
   const uint8_t* dtype;       // [D] type of each accelerator
   int32_t uniform;
+  int32_t batch;              // 1: the kernels take READY keys in batches (keys carry kQB class bits)
 };
+
+// Batched sweep: a READY key is followed by kQB bits holding floor(log2) of a
+// lower bound of the op's duration (31 at most).
+constexpr int kQB = 5;
 
 // Packed event key: time << (ib + 2) | class << ib | op.  Classes at equal
 // times: READY (an op's last input arrived) < FREE < ALLOC.
@@ -161,8 +167,9 @@ struct SimParams {
   int32_t ms;            // HBM event log slots in shared memory per warp
   int32_t mcap;          // HBM event log slots per warp
   int32_t sortcap;       // sort area entries per warp (power of two, >= max(32, n_dev))
-  int32_t drain_trigger; // (unused by the drain schedule; kept for layout stability)
-  int32_t opcap;         // ops started between HBM-event generations (<= 32)
+  int32_t drain_trigger; // batched sweep: ops started before an HBM-event generation
+  int32_t opcap;         // ops started between HBM-event generations (one at a time), or the
+                         // capacity of the list of started ops (batched: drain_trigger + 32)
   int32_t n_trace;
   const int32_t* trace_k;
   const int32_t* move_off;

@@ -17,8 +17,8 @@
 namespace gsim {
 // launchers (gmgsim_kernels.cu)
 size_t select_rank_bytes();
-const void* full_kernel_ptr(bool reg, bool key, bool t32, bool types);
-const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types);
+const void* full_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch);
+const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch);
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
@@ -40,8 +40,8 @@ constexpr int64_t kDefaultQueueCap = 1 << 16;
 constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
 constexpr int kSortCap = 128;             // power of two; raised to n_dev's power of two
-constexpr int kDrainTrigger = 48;
 constexpr int kOpsPerGeneration = 24;     // ~85 HBM events per generation (prefill graphs)
+constexpr int kBatchMinDevices = 33;      // the batched sweep serves graphs on more accelerators
 constexpr int kCheckpoints = 256;
 constexpr int kCheckpointQueue = 4096;
 constexpr int kCheckpointLog = 8192;
@@ -49,7 +49,7 @@ constexpr int kCheckpointLog = 8192;
 size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
-  size_t off_ops, off_succ, off_pred, off_sib, off_cons, off_roots, off_cap, off_base, off_avail,
+  size_t off_ops, off_succ, off_pred, off_sib, off_cons, off_roots, off_roots_q, off_cap, off_base, off_avail,
       off_dl, off_links, off_durt, off_dtype, off_linkid, total;
 };
 
@@ -104,6 +104,7 @@ void plan(Built& b) {
   L.off_sib = take(8 * (size_t)b.E);
   L.off_cons = take(4 * (size_t)b.Ec);
   L.off_roots = take(8 * (size_t)b.nroots);
+  L.off_roots_q = take(8 * (size_t)b.nroots);
   L.off_cap = take(8 * (size_t)b.D);
   L.off_base = take(8 * (size_t)b.D);
   L.off_avail = take(8 * (size_t)b.D);
@@ -459,9 +460,11 @@ size_t smem_per_warp(const SimParams& P) {
 
 bool g_smem_set = false;
 
-// Slot layout and grid for K candidates of kind `inc`.
-int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& L) {
+// Slot layout and grid for K candidates of kind `inc` (sweep: the graph's
+// batched sweep if it has one; the arbitrated kernels take keys one at a time).
+int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& L, bool sweep_batch = true) {
   const DevGmg& G = g->dg;
+  const bool batch = G.batch && sweep_batch;
   L.reg = G.D <= 32;
   L.wpb = (o && o->warps_per_block > 0) ? o->warps_per_block : kDefaultWarpsPerBlock;
   if (L.wpb > 4) return GMG_EINVAL;
@@ -474,8 +477,8 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   P.ms = kSharedLogEntries;
   P.sortcap = kSortCap;
   while (P.sortcap < G.D) P.sortcap <<= 1;
-  P.drain_trigger = kDrainTrigger;
-  P.opcap = kOpsPerGeneration;
+  P.drain_trigger = kOpsPerGeneration;
+  P.opcap = batch ? kOpsPerGeneration + 32 : kOpsPerGeneration;
   L.smem = (size_t)L.wpb * smem_per_warp(P);
   size_t o2 = 0;
   auto take = [&](size_t bytes) {
@@ -501,13 +504,14 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     SimParams big = P;
     big.g.D = 256;
     big.sortcap = 256;
+    big.opcap = kOpsPerGeneration + 32;
     if (set_smem_limits(4 * (int)smem_per_warp(big)) != cudaSuccess) return GMG_ECUDA;
     g_smem_set = true;
   }
   int bps = 0;
   const bool types = G.ntypes >= 2;
-  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0, types)
-                       : full_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0, types);
+  const void* fn = inc ? inc_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0, types, batch)
+                       : full_kernel_ptr(L.reg, G.dev_key != 0, G.t32 != 0, types, batch);
   if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
     return GMG_ECUDA;
   bps = std::max(bps, 1);
@@ -566,7 +570,7 @@ int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams&
   if (!G.dev_key || G.n >= (1 << 27)) return GMG_ERANGE;
   const int64_t xcap = std::max<int64_t>(g->xfer_bound, 1);
   if (xcap > (int64_t(1) << 29)) return GMG_ERANGE;
-  int rc = plan_launch(g, K, o, false, L);
+  int rc = plan_launch(g, K, o, false, L, false);
   if (rc) return rc;
   std::memset(&A, 0, sizeof(A));
   SimParams& P = L.P;
@@ -615,7 +619,7 @@ int plan_arbw(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbWParam
   if (!G.dev_key || G.n >= (1 << 24)) return GMG_ERANGE;
   const int64_t xcap = std::max<int64_t>(g->xfer_bound, 1);
   if (xcap > (int64_t(1) << 29)) return GMG_ERANGE;
-  int rc = plan_launch(g, K, o, false, L);
+  int rc = plan_launch(g, K, o, false, L, false);
   if (rc) return rc;
   std::memset(&A, 0, sizeof(A));
   SimParams& P = L.P;
@@ -771,6 +775,27 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   }
   put(L.off_cons, b.cons.data(), 4 * b.cons.size());
   put(L.off_roots, b.roots.data(), 8 * b.roots.size());
+  // The batched sweep: graphs on more accelerators than a warp has lanes
+  // (accelerator state in shared memory) whose READY keys have room for the
+  // duration class; its root keys carry the class of the op's shortest
+  // duration over the accelerator types.
+  int tb = 1;
+  while (tb < 62 && (int64_t(1) << tb) <= b.time_bound) ++tb;
+  const bool dev_key = tb + b.ib + 2 + 8 <= 63;
+  const bool batch = b.D >= kBatchMinDevices && dev_key && tb + b.ib + 2 + kQB <= 63;
+  if (batch) {
+    std::vector<uint64_t> rq(b.roots.size());
+    for (size_t r = 0; r < b.roots.size(); ++r) {
+      const uint32_t i = (uint32_t)(b.roots[r] & ((uint64_t(1) << b.ib) - 1));
+      int64_t lo = b.ops[i].dur;
+      if (b.T)
+        for (int t = 0; t < b.T; ++t) lo = std::min(lo, b.durt[(size_t)i * b.T + t]);
+      uint32_t q = 0;
+      while (q < 31 && (int64_t(2) << q) <= lo) ++q;
+      rq[r] = (b.roots[r] << kQB) | q;
+    }
+    put(L.off_roots_q, rq.data(), 8 * rq.size());
+  }
   put(L.off_cap, b.cap.data(), 8 * b.cap.size());
   put(L.off_base, b.base.data(), 8 * b.base.size());
   put(L.off_avail, b.avail0.data(), 8 * b.avail0.size());
@@ -795,6 +820,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.predsib = reinterpret_cast<const uint2*>(w + L.off_sib);
   G.cons = reinterpret_cast<const uint32_t*>(w + L.off_cons);
   G.root_keys = reinterpret_cast<const uint64_t*>(w + L.off_roots);
+  G.root_keys_q = reinterpret_cast<const uint64_t*>(w + L.off_roots_q);
   G.cap = reinterpret_cast<const int64_t*>(w + L.off_cap);
   G.base = reinterpret_cast<const int64_t*>(w + L.off_base);
   G.avail0 = reinterpret_cast<const int64_t*>(w + L.off_avail);
@@ -810,9 +836,9 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.R = b.R;
   G.nroots = b.nroots;
   G.ib = b.ib;
-  G.tb = 1;
-  while (G.tb < 62 && (int64_t(1) << G.tb) <= b.time_bound) ++G.tb;
-  G.dev_key = (G.tb + G.ib + 2 + 8 <= 63) ? 1 : 0;
+  G.tb = tb;
+  G.dev_key = dev_key ? 1 : 0;
+  G.batch = batch ? 1 : 0;
   // every time < 2^tb fits int32; the 32-bit instances also take the
   // accelerator id from the event key
   G.t32 = (G.tb <= 31 && G.dev_key) ? 1 : 0;
@@ -834,6 +860,8 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   g->xfer_bound = b.xfer_bound;
   g->shared_links = b.shared_links ? 1 : 0;
   I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
+  I.batched_sweep = G.batch;
+  I.t32 = G.t32;
   *out = g;
   return GMG_OK;
 }

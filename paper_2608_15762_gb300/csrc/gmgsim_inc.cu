@@ -8,12 +8,12 @@ namespace {
 // ---------------------------------------------------------------------------
 // sim_incremental: K move lists against the base.
 // ---------------------------------------------------------------------------
-template <bool kReg, bool kKey, bool kT32, bool kTypes>
-__device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p);
+template <bool kReg, bool kKey, bool kT32, bool kTypes, bool kBatch>
+__device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, uint32_t p);
 
-template <bool kReg, bool kKey, bool kT32, bool kTypes>
-__device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimParams& P, int64_t k, uint8_t* crow) {
-  using tm_t = typename Sim<kReg, kInc, kKey, kT32, kTypes>::tm_t;
+template <bool kReg, bool kKey, bool kT32, bool kTypes, bool kBatch>
+__device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, const SimParams& P, int64_t k, uint8_t* crow) {
+  using tm_t = typename Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>::tm_t;
   const DevGmg& g = S.g;
   const DevBase& B = P.base;
   const unsigned lane = lane_id();
@@ -139,7 +139,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimP
   // times change; its predecessors all finished before T_c).
   for (int x = lane; x < qsz; x += 32) {
     uint64_t key = B.ck_qkey[(int64_t)c * B.ckq + x];
-    const uint32_t op = S.kc.op(key);
+    const uint32_t op = S.rq.op(key);
     if (crow[op] != B.row[op]) {
       const int dx = crow[op];
       const RelPred rp = op_relpred(g.ops, op);
@@ -152,7 +152,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimP
         if (dp != dx) a += S.xfer(dp, dx, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
         rx = a > rx ? a : rx;
       }
-      key = S.kc.make(rx, kReady, op);
+      key = S.rq.make(rx, op, kBatch ? dur_class(S.dur_of(op, dx, op_durbytes(g.ops, op).x)) : 0u);
     }
     *S.q.kp(x) = key;
   }
@@ -242,8 +242,8 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes>& S, const SimP
 // placement: receive copies on every remote accelerator of its successors
 // (allocated at f_p), and the releases that are already determined because
 // every listed consumer on that accelerator has finished.
-template <bool kReg, bool kKey, bool kT32, bool kTypes>
-__device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
+template <bool kReg, bool kKey, bool kT32, bool kTypes, bool kBatch>
+__device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, uint32_t p) {
   const DevGmg& g = S.g;
   const unsigned lane = lane_id();
   const int64_t fp = S.fb[p];
@@ -284,7 +284,7 @@ __device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
         const uint32_t c = __ldg(lst + u);
         if (S.row[c] != du) continue;
         const int64_t fc = S.fin(c);
-        if (fc == 0) {  // not started yet
+        if (fc <= 0) {  // not started yet
           rel = false;
           break;
         }
@@ -301,9 +301,9 @@ __device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
     if (t < nl) {
       const uint32_t c = __ldg(lst + t);
       if (S.row[c] == dp) {
-        const uint64_t fc = (uint64_t)S.fin(c);
-        if (fc == 0) pending = true;
-        else mx = fc > mx ? fc : mx;
+        const int64_t fc = S.fin(c);
+        if (fc <= 0) pending = true;
+        else mx = (uint64_t)fc > mx ? (uint64_t)fc : mx;
       }
     }
   }
@@ -312,13 +312,13 @@ __device__ void regen(Sim<kReg, kInc, kKey, kT32, kTypes>& S, uint32_t p) {
   S.log_event(lane == 0, S.kc.make(m > hm ? m : hm, kFree, p), dp);
 }
 
-template <bool kReg, bool kKey, bool kT32, bool kTypes>
+template <bool kReg, bool kKey, bool kT32, bool kTypes, bool kBatch>
 __global__ void __launch_bounds__(128, 7) sim_inc_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
   const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
-  Sim<kReg, kInc, kKey, kT32, kTypes> S(P);
+  Sim<kReg, kInc, kKey, kT32, kTypes, kBatch> S(P);
   setup_slot(S, P, wib, slot, smem);
   S.rb = P.base.rb;
   S.fb = P.base.fb;
@@ -329,19 +329,21 @@ __global__ void __launch_bounds__(128, 7) sim_inc_kernel(const __grid_constant__
 }  // namespace
 
 // Instances by (accelerator state in registers, accelerator id in the event
-// key, 32-bit times, accelerator types).  32-bit times are only chosen with
-// the accelerator id in the key.
-template <bool R, bool K, bool T32>
-const void* inc_ptr4(bool types) {
-  return types ? (const void*)sim_inc_kernel<R, K, T32, true> : (const void*)sim_inc_kernel<R, K, T32, false>;
+// key, 32-bit times, accelerator types, batched sweep).  32-bit times are only
+// chosen with the accelerator id in the key; the batched sweep only with
+// accelerator state in shared memory and the id in the key.
+template <bool R, bool K, bool T32, bool B>
+const void* inc_ptr5(bool types) {
+  return types ? (const void*)sim_inc_kernel<R, K, T32, true, B> : (const void*)sim_inc_kernel<R, K, T32, false, B>;
 }
-const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types) {
+const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch) {
   if (reg) {
-    if (!key) return inc_ptr4<true, false, false>(types);
-    return t32 ? inc_ptr4<true, true, true>(types) : inc_ptr4<true, true, false>(types);
+    if (!key) return inc_ptr5<true, false, false, false>(types);
+    return t32 ? inc_ptr5<true, true, true, false>(types) : inc_ptr5<true, true, false, false>(types);
   }
-  if (!key) return inc_ptr4<false, false, false>(types);
-  return t32 ? inc_ptr4<false, true, true>(types) : inc_ptr4<false, true, false>(types);
+  if (!key) return inc_ptr5<false, false, false, false>(types);
+  if (batch) return t32 ? inc_ptr5<false, true, true, true>(types) : inc_ptr5<false, true, false, true>(types);
+  return t32 ? inc_ptr5<false, true, true, false>(types) : inc_ptr5<false, true, false, false>(types);
 }
 
 }  // namespace gsim

@@ -8,10 +8,10 @@ namespace {
 // ---------------------------------------------------------------------------
 // base_create: simulate the base placement once, recording resume points.
 // ---------------------------------------------------------------------------
-template <bool kReg, bool kKey, bool kTypes>
+template <bool kReg, bool kKey, bool kTypes, bool kBatch>
 __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
-  Sim<kReg, kBase, kKey, false, kTypes> S(P);
+  Sim<kReg, kBase, kKey, false, kTypes, kBatch> S(P);
   setup_slot(S, P, 0, 0, smem);
   const DevBase& B = P.base;
   const unsigned lane = lane_id();
@@ -30,7 +30,7 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
   S.ck = 0;
   S.next_ck = 0;
   // checkpoint 0: the initial state, valid for every resume time >= 0
-  S.maybe_checkpoint(S.kc.make(0, kReady, 0));
+  S.maybe_checkpoint(S.rq.make(0, 0u, 0u));
   S.run();
   if (lane == 0) B.status[0] = S.status;
   if (S.status != GMG_SIM_OK) return;
@@ -132,29 +132,32 @@ __global__ void __launch_bounds__(256) select_final_kernel(const Rank* part, int
 // ---------------------------------------------------------------------------
 size_t select_rank_bytes() { return sizeof(Rank); }
 
-const void* full_kernel_ptr(bool reg, bool key, bool t32, bool types);  // gmgsim_full.cu
-const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types);   // gmgsim_inc.cu
+const void* full_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch);  // gmgsim_full.cu
+const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch);   // gmgsim_inc.cu
 
-template <bool R, bool K>
-const void* base_ptr3(bool types) {
-  return types ? (const void*)sim_base_kernel<R, K, true> : (const void*)sim_base_kernel<R, K, false>;
+template <bool R, bool K, bool B>
+const void* base_ptr4(bool types) {
+  return types ? (const void*)sim_base_kernel<R, K, true, B> : (const void*)sim_base_kernel<R, K, false, B>;
 }
-const void* base_kernel_ptr(bool reg, bool key, bool types) {
-  if (reg) return key ? base_ptr3<true, true>(types) : base_ptr3<true, false>(types);
-  return key ? base_ptr3<false, true>(types) : base_ptr3<false, false>(types);
+const void* base_kernel_ptr(bool reg, bool key, bool types, bool batch) {
+  if (reg) return key ? base_ptr4<true, true, false>(types) : base_ptr4<true, false, false>(types);
+  if (!key) return base_ptr4<false, false, false>(types);
+  return batch ? base_ptr4<false, true, true>(types) : base_ptr4<false, true, false>(types);
 }
 
 cudaError_t set_smem_limits(int smem) {
   for (int r = 0; r < 2; ++r)
     for (int k = 0; k < 2; ++k)
       for (int t = 0; t < 2; ++t)
-        for (int y = 0; y < 2; ++y) {
-          const void* fns[] = {full_kernel_ptr(r, k, t, y), inc_kernel_ptr(r, k, t, y), base_kernel_ptr(r, k, y)};
-          for (const void* f : fns) {
-            const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-            if (e != cudaSuccess) return e;
+        for (int y = 0; y < 2; ++y)
+          for (int b = 0; b < 2; ++b) {
+            const void* fns[] = {full_kernel_ptr(r, k, t, y, b), inc_kernel_ptr(r, k, t, y, b),
+                                 base_kernel_ptr(r, k, y, b)};
+            for (const void* f : fns) {
+              const cudaError_t e = cudaFuncSetAttribute(f, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+              if (e != cudaSuccess) return e;
+            }
           }
-        }
   return cudaSuccess;
 }
 
@@ -167,15 +170,17 @@ static cudaError_t launch_ptr(const void* fn, const SimParams& P, int grid, int 
 }
 
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
-  return launch_ptr(full_kernel_ptr(reg, P.g.dev_key != 0, P.g.t32 != 0, P.g.ntypes >= 2), P, grid, block, smem, st);
+  return launch_ptr(full_kernel_ptr(reg, P.g.dev_key != 0, P.g.t32 != 0, P.g.ntypes >= 2, P.g.batch != 0), P, grid,
+                    block, smem, st);
 }
 
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st) {
-  return launch_ptr(inc_kernel_ptr(reg, P.g.dev_key != 0, P.g.t32 != 0, P.g.ntypes >= 2), P, grid, block, smem, st);
+  return launch_ptr(inc_kernel_ptr(reg, P.g.dev_key != 0, P.g.t32 != 0, P.g.ntypes >= 2, P.g.batch != 0), P, grid,
+                    block, smem, st);
 }
 
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st) {
-  return launch_ptr(base_kernel_ptr(reg, P.g.dev_key != 0, P.g.ntypes >= 2), P, 1, 32, smem, st);
+  return launch_ptr(base_kernel_ptr(reg, P.g.dev_key != 0, P.g.ntypes >= 2, P.g.batch != 0), P, 1, 32, smem, st);
 }
 
 cudaError_t launch_select(const int32_t* status, const int32_t* viol, const int64_t* score,

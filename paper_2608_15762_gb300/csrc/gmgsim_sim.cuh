@@ -117,6 +117,36 @@ struct KeyCodec {
   __device__ __forceinline__ uint32_t op(uint64_t k) const { return (uint32_t)(k & mask); }
 };
 
+// READY keys as queued: the KeyCodec key with class READY, shifted up by qb
+// bits that hold the op's duration class (floor(log2) of a lower bound of its
+// duration) in the batched sweep; qb = 0 otherwise (then equal to the
+// KeyCodec key).  The class bits sit below the op id, so they never change
+// the order of two keys.
+struct ReadyCodec {
+  int ib, qb;
+  uint64_t mask;
+  template <typename TM>
+  __device__ __forceinline__ uint64_t make(TM t, uint32_t op, uint32_t q) const {
+    using U = typename std::make_unsigned<TM>::type;
+    return ((((uint64_t)(U)t << (ib + 2)) | (uint64_t)op) << qb) | (qb ? (uint64_t)q : 0ull);
+  }
+  __device__ __forceinline__ int64_t time(uint64_t k) const { return (int64_t)(k >> (ib + 2 + qb)); }
+  __device__ __forceinline__ uint32_t op(uint64_t k) const { return (uint32_t)((k >> qb) & mask); }
+  __device__ __forceinline__ uint32_t q(uint64_t k) const { return (uint32_t)k & ((1u << qb) - 1u); }
+};
+
+// floor(log2(dur)) for dur >= 1, at most 31: 2^class is a lower bound of dur.
+__device__ __forceinline__ uint32_t dur_class(int64_t dur) {
+  const uint32_t c = 63u - (uint32_t)__clzll((unsigned long long)dur);
+  return c < 31u ? c : 31u;
+}
+
+__device__ __forceinline__ int64_t warp_sum_i64(int64_t v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(kFullMask, v, o);
+  return v;
+}
+
 // ---------------------------------------------------------------------------
 // READY keys: warp-cooperative 32-ary min-heap.  Slots [0, qs) are in shared
 // memory (qs >= 33, so the root and its children always are), the rest in
@@ -327,13 +357,17 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
 // start, finish, free and arrival times are carried as int32 (bytes, scores
 // and outputs stay int64).
 // kTypes: the graph has several accelerator types (durations per (type, op)).
-template <bool kReg, int kMode, bool kKey, bool kT32 = false, bool kTypes = false>
+// kBatch: the batched sweep (run_batched), for accelerator state in shared
+// memory with the accelerator id in the event key.
+template <bool kReg, int kMode, bool kKey, bool kT32 = false, bool kTypes = false, bool kBatch = false>
 struct Sim {
   static_assert(!(kT32 && kMode == kBase), "the base snapshot keeps 64-bit times");
+  static_assert(!kBatch || (!kReg && kKey), "the batched sweep keeps accelerator state in shared memory");
   using tm_t = typename std::conditional<kT32, int32_t, int64_t>::type;
   const SimParams& P;
   const DevGmg& g;
-  KeyCodec kc;
+  KeyCodec kc;      // HBM log entries (and READY keys when qb = 0)
+  ReadyCodec rq;    // READY keys
   ReadyHeap q;      // READY keys beyond the register tier
   uint64_t rk_reg;  // register tier: one READY key per lane (kKeyMax = empty)
   MemLog log;
@@ -368,13 +402,17 @@ struct Sim {
   __device__ Sim(const SimParams& p) : P(p), g(p.g) {
     kc.ib = g.ib;
     kc.mask = (1ull << g.ib) - 1ull;
+    rq.ib = g.ib;
+    rq.mask = kc.mask;
+    rq.qb = kBatch ? kQB : 0;
     ds = g.ib + 2 + g.tb;
     lowmask = kKey ? (1ull << ds) - 1ull : kKeyMax;
   }
 
   // Started ops are those with a finish time (every finish time is >= 1;
-  // the finish array is zeroed per candidate).
-  __device__ __forceinline__ bool popped(uint32_t x) const { return fin(x) != 0; }
+  // the finish array is zeroed per candidate; the batched sweep marks an op
+  // whose READY key is queued with -1).
+  __device__ __forceinline__ bool popped(uint32_t x) const { return fin(x) > 0; }
   // Finish time of a simulated op (incremental: ops before the resume point
   // keep their base finish).
   // The low 32 bits of a base-snapshot time (little-endian int64).
@@ -426,7 +464,7 @@ struct Sim {
 
 
   __device__ __forceinline__ void load_root() {
-    rkey = rootptr < g.nroots ? __ldg(g.root_keys + rootptr) : kKeyMax;
+    rkey = rootptr < g.nroots ? __ldg((kBatch ? g.root_keys_q : g.root_keys) + rootptr) : kKeyMax;
   }
 
   // READY keys go to a free lane's register if there is one, else the heap.
@@ -543,7 +581,7 @@ struct Sim {
             const uint32_t p = __ldg(g.pred + jp.pred_off + k) & kIdMask;
             if (p == i) continue;
             tm_t a = fin(p);
-            if (a == 0) {  // not started yet
+            if (a <= 0) {  // not started yet
               rdy = false;
               break;
             }
@@ -664,7 +702,7 @@ struct Sim {
               rel = row[sb & ~kSibLater] != d;  // the other consumer finishes later
             } else if (sb != kSibMany) {
               const tm_t fs = fin(sb);
-              rel = !(row[sb] == d && !(fs != 0 && fs < f));
+              rel = !(row[sb] == d && !(fs > 0 && fs < f));
             } else {
               const XqSucc px = op_xqsucc(g.ops, p);
               const uint4 pls = make_uint4(px.succ_off, px.nsucc, 0u, 0u);
@@ -676,7 +714,7 @@ struct Sim {
               for (uint32_t w = 0; w < nl; ++w) {
                 const uint32_t c = __ldg(lst + w);
                 const tm_t fc = c != x ? fin(c) : 0;
-                if (c != x && row[c] == d && !(fc != 0 && fc < f)) {
+                if (c != x && row[c] == d && !(fc > 0 && fc < f)) {
                   rel = false;
                   break;
                 }
@@ -962,6 +1000,10 @@ struct Sim {
   // The event loop (Sec. 3.3.3).
   __device__ void run() {
     if (status) return;
+    if (kBatch) {
+      run_batched();
+      return;
+    }
     while (true) {
       const uint64_t top = q.top();
       const uint64_t rm = warp_min_u64(rk_reg);
@@ -990,6 +1032,171 @@ struct Sim {
       if (status) break;
     }
     if (!status) drain(kI64Max);
+  }
+
+  // -------------------------------------------------------------------------
+  // Batched sweep: the keys are taken in the same order as by run(), but
+  // consecutive keys are handled together, one op per lane.  Key k_m joins
+  // the batch k_1 < ... < k_{m-1} while time(k_m) < min_l (time(k_l) +
+  // 2^class(k_l)).  Every key pushed while handling k_l is at least
+  // (f_l, READY, .) with f_l >= r_l + dur_l >= r_l + 2^class(k_l) > r_m, so
+  // nothing a batch pushes can precede one of its keys: handling them
+  // together, each accelerator's ops in key order, gives the starts of
+  // handling them one at a time.  (Many tenants on many accelerators keep
+  // about a dozen keys per batch; the dependent loads of a batch's ops then
+  // overlap instead of following each other.)
+  // -------------------------------------------------------------------------
+  __device__ __forceinline__ uint64_t peek(uint64_t& rm) const {
+    const uint64_t top = q.top();
+    rm = warp_min_u64(rk_reg);
+    const uint64_t nk = rkey < top ? rkey : top;
+    return rm < nk ? rm : nk;
+  }
+  __device__ __forceinline__ void take(uint64_t nk, uint64_t rm) {
+    if (nk == rm) {
+      if (rk_reg == rm) rk_reg = kKeyMax;  // keys are unique
+    } else if (nk == rkey) {
+      ++rootptr;
+      load_root();
+    } else {
+      __syncwarp();
+      q.pop();
+    }
+  }
+  // An op whose inputs several ops of one batch complete is queued once: the
+  // first lane to mark its (zero) finish time with -1 queues it.
+  __device__ __forceinline__ bool claim(uint32_t j) {
+    if (kT32) return atomicCAS(reinterpret_cast<int*>(fbuf + j), 0, -1) == 0;
+    return atomicCAS(reinterpret_cast<unsigned long long*>(fbuf + j), 0ull, ~0ull) == 0ull;
+  }
+
+  __device__ void run_batched() {
+    const unsigned lane = lane_id();
+    while (true) {
+      uint64_t rm;
+      uint64_t nk = peek(rm);
+      if (kMode == kBase) maybe_checkpoint(nk);
+      if (nk == kKeyMax) break;
+      if (opn >= P.drain_trigger) drain(rq.time(nk));
+      uint64_t mine = kKeyMax;
+      int m = 0;
+      int64_t lim = 0;
+      while (true) {
+        const int64_t t = rq.time(nk);
+        take(nk, rm);
+        if ((int)lane == m) mine = nk;
+        const int64_t e = t + ((int64_t)1 << rq.q(nk));
+        lim = (m == 0 || e < lim) ? e : lim;
+        if (kMode == kBase) last_t = (tm_t)t;
+        if (++m == 32) break;
+        nk = peek(rm);
+        if (nk == kKeyMax || rq.time(nk) >= lim) break;
+      }
+      iters += m;
+      if (iters > (int32_t)g.max_iter) {
+        status = GMG_SIM_LOOP;
+        break;
+      }
+      start_batch(mine, m);
+      if (status) break;
+    }
+    if (!status) drain(kI64Max);
+  }
+
+  // Start the batch's ops (lane b < m holds key b), record them for HBM-event
+  // generation, and queue the successors they make ready.
+  __device__ void start_batch(uint64_t key, int m) {
+    const unsigned lane = lane_id();
+    const bool v = (int)lane < m;
+    uint32_t i = 0, succ_off = 0, nsucc = 0, flags = 0;
+    int32_t req = 0;
+    int d = 0;
+    tm_t r = 0, f = 0, dur = 0;
+    int64_t bytes = 0, xq = 0;
+    if (v) {
+      i = rq.op(key);
+      r = (tm_t)rq.time(key);
+      const longlong2 db = op_durbytes(g.ops, i);
+      const XqSucc xs = op_xqsucc(g.ops, i);
+      const uint4 cs = op_cons(g.ops, i);
+      bytes = db.y;
+      xq = xs.xq;
+      succ_off = xs.succ_off;
+      nsucc = xs.nsucc;
+      req = (int32_t)cs.z;
+      flags = cs.w;
+      d = row[i];
+      dur = (tm_t)dur_of(i, d, db.x);
+    }
+    // every accelerator starts its ops of the batch in key (= lane) order
+    bool todo = v;
+    while (__any_sync(kFullMask, todo)) {
+      const uint32_t grp = __match_any_sync(kFullMask, todo ? (uint32_t)d : 256u + lane);
+      if (todo && __ffs(grp) - 1 == (int)lane) {
+        const tm_t fd = (tm_t)dv.fr[d];
+        const tm_t s = r > fd ? r : fd;
+        f = s + dur;
+        dv.fr[d] = (int64_t)f;
+        todo = false;
+      }
+      __syncwarp();
+    }
+    if (v) {
+      fbuf[i] = f;
+      if (flags & kReqSink)
+        atomicMax(reinterpret_cast<unsigned long long*>(creq + req), (unsigned long long)f);
+      if (kMode == kBase) P.base.rb[i] = r;
+      oplog[opn + (int)lane] = i;
+    }
+    opn += m;
+    score += warp_sum_i64((v && (flags & kScored)) ? (int64_t)f : 0);
+    if (kMode == kBase) {
+      const tm_t mk = (tm_t)warp_max_u64(v ? (uint64_t)f : 0ull);
+      makespan = mk > makespan ? mk : makespan;
+      readypops += m;
+    }
+    if (kMode == kInc) nev += __popc(__ballot_sync(kFullMask, v && r >= T0));
+    __syncwarp();
+    // successors: ready once every predecessor has started; ready time = the
+    // latest arrival over all of them (Sec. 3.3.2)
+    const uint32_t maxs = __reduce_max_sync(kFullMask, nsucc);
+    for (uint32_t u = 0; u < maxs; ++u) {
+      uint32_t j = 0, qj = 0;
+      tm_t rj = 0;
+      bool rdy = false;
+      if (u < nsucc) {
+        j = __ldg(g.succ + succ_off + u);
+        const int dj = row[j];
+        tm_t arr = f;
+        if (dj != d) arr = f + xfer(d, dj, bytes, xq);
+        const RelPred jp = op_relpred(g.ops, j);
+        qj = dur_class(dur_of(j, dj, op_durbytes(g.ops, j).x));
+        const tm_t rel = (tm_t)jp.rel;
+        rj = rel > arr ? rel : arr;
+        rdy = true;
+        if (jp.npred > 1) {
+          for (uint32_t k = 0; k < jp.npred; ++k) {
+            const uint32_t p = __ldg(g.pred + jp.pred_off + k) & kIdMask;
+            if (p == i) continue;
+            tm_t a = fin(p);
+            if (a <= 0) {  // not started yet
+              rdy = false;
+              break;
+            }
+            const int dp = row[p];
+            if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
+            rj = a > rj ? a : rj;
+          }
+          if (rdy) rdy = claim(j);
+        }
+      }
+      uint32_t bm = __ballot_sync(kFullMask, rdy);
+      while (bm) {
+        const int src = __ffs(bm) - 1;
+        bm &= bm - 1;
+        push_ready(__shfl_sync(kFullMask, rq.make(rj, j, qj), src));
+      }
+    }
   }
 
   __device__ void write_invalid(int64_t k, int32_t st) {
@@ -1093,12 +1300,12 @@ struct Sim {
 // READY heap, event log, partial results; the ops started by then are those
 // with base ready time < T_c.  An incremental candidate whose resume time T0
 // is >= T_c restarts there.
-template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes>
-__device__ void Sim<kReg, kMode, kKey, kT32, kTypes>::maybe_checkpoint(uint64_t next_key) {
+template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes, bool kBatch>
+__device__ void Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>::maybe_checkpoint(uint64_t next_key) {
   if (kMode != kBase) return;
   const DevBase& B = P.base;
   if (next_key == kKeyMax || ck >= B.nck || readypops < next_ck) return;
-  const int64_t tn = kc.time(next_key);
+  const int64_t tn = rq.time(next_key);
   if (tn <= last_t) return;
   const unsigned lane = lane_id();
   generate();
@@ -1134,9 +1341,9 @@ __device__ void Sim<kReg, kMode, kKey, kT32, kTypes>::maybe_checkpoint(uint64_t 
   __syncwarp();
 }
 
-template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes>
-__device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes>& S, const SimParams& P, unsigned wib, int64_t slot,
-                           uint8_t* smem) {
+template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes, bool kBatch>
+__device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>& S, const SimParams& P, unsigned wib,
+                           int64_t slot, uint8_t* smem) {
   uint8_t* sl = P.scratch + slot * P.slot_bytes;
   const WarpSmem w = carve_smem(smem, P, wib);
   S.q.sk = w.heap;
@@ -1156,8 +1363,9 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes>& S, const SimPar
   S.oplog = w.oplog;
   S.opn = 0;
   S.sortcap = P.sortcap;
-  S.fbuf = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32, kTypes>::tm_t*>(sl + P.off_f);
-  S.holdb = reinterpret_cast<typename Sim<kReg, kMode, kKey, kT32, kTypes>::tm_t*>(sl + P.off_hold);
+  using tm_t = typename Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>::tm_t;
+  S.fbuf = reinterpret_cast<tm_t*>(sl + P.off_f);
+  S.holdb = reinterpret_cast<tm_t*>(sl + P.off_hold);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
   S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
   S.dv.setup(P.g, w.dev);

@@ -86,7 +86,8 @@ class _Info(C.Structure):
     _fields_ = [("n_ops", C.c_int32), ("n_edges", C.c_int32), ("n_dev", C.c_int32),
                 ("n_req", C.c_int32), ("n_roots", C.c_int32), ("id_bits", C.c_int32),
                 ("time_bits", C.c_int32), ("uniform_links", C.c_int32),
-                ("time_bound", C.c_int64), ("default_queue_cap", C.c_int64)]
+                ("time_bound", C.c_int64), ("default_queue_cap", C.c_int64),
+                ("batched_sweep", C.c_int32), ("t32", C.c_int32)]
 
 
 _LIB = None

@@ -662,14 +662,16 @@ def random_desc(seed: int, n_ops: int, n_dev: int, n_req: int = 2, max_pred: int
                 edge_p: float = 0.3, dur_hi: int = 50, bytes_hi: int = 1 << 12,
                 cap=None, explicit_cons: bool = False, with_release: bool = True,
                 with_avail0: bool = True, link_hetero: bool = True,
-                deadline: bool = True, n_types: int = 0) -> GmgDesc:
+                deadline: bool = True, n_types: int = 0, window: int = 12) -> GmgDesc:
     """A random topologically numbered DAG with small integer values (with
     n_types >= 2: accelerator types and per-type durations, drawn from a
-    stream of their own so the other fields match the one-type graph)."""
+    stream of their own so the other fields match the one-type graph).
+    Predecessors are drawn among the previous ``window`` ops: a wide window
+    gives many ops that are ready at once."""
     g = _rng(seed, 77)
     preds = []
     for i in range(n_ops):
-        cand = np.arange(max(0, i - 12), i)
+        cand = np.arange(max(0, i - window), i)
         if cand.size and g.random() < 0.9:
             k = int(g.integers(0, min(max_pred, cand.size) + 1))
             p = sorted(g.choice(cand, size=k, replace=False).tolist()) if k else []
