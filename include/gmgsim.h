@@ -229,8 +229,10 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld,
  *     the buffer (about 16 bytes per op plus queue spill space), other
  *     arguments and errors as sim_batch.
  *   - The first call on each device looks up the buffer's device address
- *     (with that device current); make that first call before any stream
- *     capture.
+ *     (with that device current) and keeps it for the life of the process;
+ *     make that first call before any stream capture, and do not call this
+ *     entry point again after a cudaDeviceReset of that device (the reset
+ *     unloads the library's module, so the kept address no longer holds).
  *   - All calls share the buffer and find the previous call's data in it;
  *     nothing needs clearing (the kernel initialises what it reads), but two
  *     calls that could run at the same time on the GPU race: order them. */

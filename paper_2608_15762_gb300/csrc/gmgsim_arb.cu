@@ -556,6 +556,7 @@ __global__ void __launch_bounds__(128, 7) sim_arb_kernel(const __grid_constant__
 
 // One warp per incremental candidate: check the move list (an op or device
 // out of range, then an op moved twice), copy the base row, apply the moves.
+// A base row with a device out of range makes every candidate BADBASE.
 __global__ void __launch_bounds__(128) expand_moves_kernel(const uint8_t* base_row, const int32_t* base_status,
                                                            int32_t ld, int32_t n, int32_t D, const int32_t* off,
                                                            const int32_t* op, const uint8_t* dev, int32_t K,
@@ -563,7 +564,11 @@ __global__ void __launch_bounds__(128) expand_moves_kernel(const uint8_t* base_r
   const unsigned lane = lane_id();
   const int64_t w0 = ((int64_t)blockIdx.x * blockDim.x + threadIdx.x) >> 5;
   const int64_t nw = ((int64_t)gridDim.x * blockDim.x) >> 5;
-  const bool base_ok = *base_status == GMG_SIM_OK;
+  // Only a base row with a device out of range invalidates the moved rows;
+  // the base's own (pure-latency) simulation status -- a queue or loop limit
+  // of that run -- says nothing about the arbitrated simulations of the
+  // moved placements, which run in full.
+  const bool base_ok = *base_status != GMG_SIM_BADDEV;
   for (int64_t k = w0; k < K; k += nw) {
     const int32_t a = off[k], b = off[k + 1];
     int32_t st = base_ok ? GMG_SIM_OK : GMG_SIM_BADBASE;

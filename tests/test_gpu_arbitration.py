@@ -279,3 +279,26 @@ def test_large_workload_subset_256_accelerators():
     ks = np.array([0, 1, 37, 100, 128, 200, 254, 255])
     s, pk, _ = O.simulate_batch(wl.desc, rows[ks], arbitrated=True)
     compare({k: (None if v is None else v[ks]) for k, v in got.items()}, s, pk)
+
+
+def test_incremental_arbitrated_ignores_a_base_queue_limit():
+    """A base snapshot whose own pure-latency run stopped at a queue limit
+    (queue_cap=2 on a graph with 120 successors of one op) cannot serve
+    resumed candidates (pure latency: every candidate BADBASE), but the
+    arbitrated candidates are full simulations of their moved rows and equal
+    the oracle's."""
+    n = 121
+    d = mk([[]] + [[0]] * 120, [5] * n, [1 << 10] * n, n_dev=4, bw=100, lat=1)
+    base = np.random.default_rng(3).integers(0, 4, n).astype(np.uint8)
+    mv = W.random_moves(3, 16, base, 4, max_moves=6)
+    g = G.gmg_create(d)
+    b = G.base_create(g, torch.from_numpy(base).cuda(), queue_cap=2)
+    off, op, dv = G.moves_to_device(mv, "cuda")
+    lat = G.sim_incremental(g, b, off, op, dv)
+    arb = G.sim_incremental(g, b, off, op, dv, req_done=True, arbitrated=True)
+    torch.cuda.synchronize()
+    st = lat.status.cpu().numpy()
+    assert (st == G.SIM_BADBASE).all()
+    s, pk, rq = O.incremental_batch(d, base, mv, arbitrated=True)
+    compare(arb.to_numpy(), s, pk, rq)
+    assert (arb.status.cpu().numpy() == 0).all()

@@ -52,6 +52,60 @@ def test_same_results_as_sim_batch_on_two_calls(which):
             assert np.array_equal(a[f], b[f]), f
 
 
+def _compare_calls(g, batches, **kw):
+    for place in batches:
+        tk = torch.tensor([0, place.shape[0] - 1], dtype=torch.int32, device="cuda")
+        ref = G.sim_batch(g, place, req_done=True, trace_k=tk, **kw)
+        got = G.sim_batch_noalloc(g, place, req_done=True, trace_k=tk, **kw)
+        torch.cuda.synchronize()
+        a, b = ref.to_numpy(), got.to_numpy()
+        for f in FIELDS:
+            assert np.array_equal(a[f], b[f]), f
+
+
+def test_arbitrated_transfers_on_two_calls():
+    """Arbitrated transfers (Sec. 3.5.2) through the fixed buffer: on 8 and on
+    40 accelerators (the two arbitrated kernels)."""
+    for D in (8, 40):
+        desc = W.random_desc(23 + D, 400, D)
+        _compare_calls(G.gmg_create(desc), [_rows(3, 97, 400, D), _rows(4, 33, 400, D)], arbitrated=True)
+
+
+def _chain(n, D, seed):
+    """A chain of n ops (each op feeds the next) with random sizes."""
+    g = np.random.default_rng(seed)
+    pred_off = np.arange(n + 1, dtype=np.int32) - 1
+    pred_off[0] = 0
+    return W.GmgDesc(n_dev=D, pred_off=pred_off, pred_idx=np.arange(n - 1, dtype=np.int32),
+                     dur=g.integers(1, 50, n).astype(np.int64), out_bytes=g.integers(0, 1 << 12, n).astype(np.int64),
+                     release=np.zeros(n, np.int64), req_id=np.full(n, -1, np.int32),
+                     scored=np.ones(n, np.uint8), deadline=np.zeros(0, np.int64),
+                     cap=np.full(D, 1 << 40, np.int64), base=np.zeros(D, np.int64),
+                     avail0=np.zeros(D, np.int64), bw=np.full(D * D, 7, np.int64),
+                     lat=np.full(D * D, 2, np.int64)).normalized()
+
+
+def test_fewer_slots_than_the_grid():
+    """A graph whose warp slot is about 1 MB: the fixed buffer holds a few
+    dozen slots, fewer than sim_batch's grid, so each warp takes several
+    candidates in turn."""
+    n = 60_000
+    g = G.gmg_create(_chain(n, 3, 5))
+    slot = G.sim_scratch_bytes(g, 1) // 4          # one block of 4 warps for one candidate
+    assert 4 * slot <= _noalloc_bytes() < G.sim_scratch_bytes(g, 4096)
+    _compare_calls(g, [_rows(5, 211, n, 3), _rows(6, 64, n, 3)])
+
+
+def test_one_warp_blocks_when_four_slots_do_not_fit():
+    """A graph whose warp slot is about 13 MB: fewer than four slots fit, so
+    the call re-plans with one-warp blocks."""
+    n = 800_000
+    g = G.gmg_create(_chain(n, 2, 7))
+    slot = G.sim_scratch_bytes(g, 1) // 4
+    assert slot <= _noalloc_bytes() < 4 * slot
+    _compare_calls(g, [_rows(7, 6, n, 2), _rows(8, 3, n, 2)])
+
+
 def _noalloc_bytes():
     """GMG_NOALLOC_SCRATCH_BYTES as include/gmgsim.h defines it."""
     import os
