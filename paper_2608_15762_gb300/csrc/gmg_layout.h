@@ -177,8 +177,10 @@ struct SimParams {
   const uint8_t* move_dev;
   uint8_t* scratch;
   int64_t slot_bytes;    // scratch bytes per warp slot
-  // byte offsets inside a slot
-  int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row;
+  int32_t dev_bytes;     // shared bytes of accelerator state per warp
+  int32_t pad_;
+  // byte offsets inside a slot (off_pk < 0: the peaks are in shared memory)
+  int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row, off_pk;
 };
 
 }  // namespace gsim

@@ -36,6 +36,7 @@ constexpr int64_t kI64Max = 0x7fffffffffffffffll;
 constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
 constexpr int kDefaultWarpsPerBlock = 4;
 constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
+constexpr int kSharedQueueEntriesBatch = 225;  // 1 + 32 * 7: the batched sweep's wider frontier
 constexpr int64_t kDefaultQueueCap = 1 << 16;
 constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
@@ -455,7 +456,15 @@ int log_cap(const gmg* g, const sim_opts_t* o) {
 
 size_t smem_per_warp(const SimParams& P) {
   return align_up((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 + (size_t)P.opcap * 4, 16) +
-         (size_t)P.g.D * 24;
+         (size_t)P.dev_bytes;
+}
+
+// Shared bytes of accelerator state per warp: live bytes; peaks unless they
+// are kept in global scratch (more than 32 accelerators); free times (of
+// tbytes each) unless lanes hold them in registers (at most 32).
+int dev_smem_bytes(int D, size_t tbytes) {
+  const bool reg = D <= 32;
+  return (int)align_up((size_t)D * 8 + (reg ? (size_t)D * 8 : 0) + (reg ? 0 : (size_t)D * tbytes), 16);
 }
 
 bool g_smem_set = false;
@@ -472,13 +481,15 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   std::memset(&P, 0, sizeof(P));
   P.g = G;
   P.qcap = queue_cap(g, o);
-  P.qs = kSharedQueueEntries;   // >= 33 (the root's children are always in shared memory)
+  P.qs = batch ? kSharedQueueEntriesBatch : kSharedQueueEntries;  // >= 33 (the root's children are
+                                                                     // always in shared memory)
   P.mcap = log_cap(g, o);
   P.ms = kSharedLogEntries;
   P.sortcap = kSortCap;
   while (P.sortcap < G.D) P.sortcap <<= 1;
   P.drain_trigger = kOpsPerGeneration;
   P.opcap = batch ? kOpsPerGeneration + 32 : kOpsPerGeneration;
+  P.dev_bytes = dev_smem_bytes(G.D, G.t32 ? 4 : 8);
   L.smem = (size_t)L.wpb * smem_per_warp(P);
   size_t o2 = 0;
   auto take = [&](size_t bytes) {
@@ -496,6 +507,7 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   P.off_mk = take(8 * (size_t)mspill);
   P.off_md = take((size_t)mspill);
   P.off_row = take(inc ? (size_t)align_up(std::max(G.n, 1), 16) : 0);
+  P.off_pk = L.reg ? -1 : take(8 * (size_t)G.D);
   P.slot_bytes = (int64_t)o2;
   const int sms = device_sms();
   if (sms <= 0) return GMG_ECUDA;
@@ -505,6 +517,8 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     big.g.D = 256;
     big.sortcap = 256;
     big.opcap = kOpsPerGeneration + 32;
+    big.qs = kSharedQueueEntriesBatch;
+    big.dev_bytes = 24 * 256;
     if (set_smem_limits(4 * (int)smem_per_warp(big)) != cudaSuccess) return GMG_ECUDA;
     g_smem_set = true;
   }
@@ -704,6 +718,7 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   int rc = plan_launch(g, 1, o, false, L);
   if (rc) return rc;
   L.wpb = 1;
+  L.P.dev_bytes = dev_smem_bytes(G.D, 8);  // the base snapshot keeps 64-bit times
   L.smem = smem_per_warp(L.P);
   B.nck = kCheckpoints;
   B.ckq = std::min(L.P.qcap, kCheckpointQueue);

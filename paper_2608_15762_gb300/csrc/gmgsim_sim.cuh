@@ -230,35 +230,38 @@ struct MemLog {
 
 // ---------------------------------------------------------------------------
 // Per-accelerator state.  Free times: with at most 32 accelerators lane d
-// holds accelerator d's in a register, else a shared array.  Live and peak
-// bytes: shared arrays (the drain updates them a batch at a time).
+// holds accelerator d's in a register, else a shared array of the kernel's
+// time type.  Live bytes: a shared array (the drain updates it a batch at a
+// time).  Peak bytes: a shared array, or with more than 32 accelerators an
+// array in the warp's global scratch (only raised by atomicMax and read at
+// the end, so its latency is never waited on).
 // ---------------------------------------------------------------------------
 template <bool kReg, typename TM>
 struct Devices {
   TM fr_reg;
-  int64_t* fr;  // shared [D] (when !kReg)
+  TM* fr;       // shared [D] (when !kReg)
   int64_t* lv;  // shared [D]
-  int64_t* pk;  // shared [D]
+  int64_t* pk;  // [D], shared or global
   int D;
-  __device__ void setup(const DevGmg& g, int64_t* sm) {
+  __device__ void setup(const DevGmg& g, uint8_t* sm, int64_t* pk_global) {
     D = g.D;
-    fr = sm;
-    lv = sm + (kReg ? 0 : D);
-    pk = lv + D;
+    lv = reinterpret_cast<int64_t*>(sm);
+    pk = pk_global ? pk_global : lv + D;
+    fr = reinterpret_cast<TM*>(pk_global ? lv + D : lv + 2 * D);
   }
   __device__ void reset(const DevGmg& g) {
     const unsigned l = lane_id();
     for (int d = l; d < D; d += 32) {
       lv[d] = g.base[d];
       pk[d] = g.base[d];
-      if (!kReg) fr[d] = g.avail0[d];
+      if (!kReg) fr[d] = (TM)g.avail0[d];
     }
     if (kReg) fr_reg = l < (unsigned)D ? (TM)g.avail0[l] : (TM)0;
     __syncwarp();
   }
   __device__ __forceinline__ TM get_free(int d) const {
     if (kReg) return __shfl_sync(kFullMask, fr_reg, d);
-    return (TM)fr[d];
+    return fr[d];
   }
   __device__ __forceinline__ void set_free(int d, TM v) {
     if (kReg) {
@@ -289,7 +292,7 @@ struct Devices {
   __device__ void save(int64_t* dst) const {
     const unsigned l = lane_id();
     for (int d = l; d < D; d += 32) {
-      if (!kReg) dst[d] = fr[d];
+      if (!kReg) dst[d] = (int64_t)fr[d];
       dst[D + d] = lv[d];
       dst[2 * D + d] = pk[d];
     }
@@ -298,7 +301,7 @@ struct Devices {
   __device__ void load(const int64_t* src) {
     const unsigned l = lane_id();
     for (int d = l; d < D; d += 32) {
-      if (!kReg) fr[d] = src[d];
+      if (!kReg) fr[d] = (TM)src[d];
       lv[d] = src[D + d];
       pk[d] = src[2 * D + d];
     }
@@ -310,7 +313,7 @@ struct Devices {
   __device__ int64_t max_busy(const DevGmg& g) const {
     uint64_t m = 0;
     for (int d = lane_id(); d < D; d += 32) {
-      const int64_t f = kReg ? (int64_t)fr_reg : fr[d];
+      const int64_t f = kReg ? (int64_t)fr_reg : (int64_t)fr[d];
       if (f > g.avail0[d]) m = (uint64_t)f > m ? (uint64_t)f : m;
     }
     return (int64_t)warp_max_u64(m);
@@ -329,7 +332,7 @@ struct WarpSmem {
   uint64_t* sortk;  // [sortcap]
   uint8_t* logd;    // [ms]
   uint8_t* sortd;   // [sortcap]
-  int64_t* dev;     // [3*D] (2*D used when free times are in registers)
+  uint8_t* dev;     // accelerator state (P.dev_bytes)
 };
 
 __device__ __forceinline__ size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
@@ -337,7 +340,7 @@ __device__ __forceinline__ size_t align16(size_t x) { return (x + 15) & ~(size_t
 __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P, unsigned wib) {
   const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 +
                               (size_t)P.opcap * 4);
-  const size_t per = head + (size_t)P.g.D * 24;
+  const size_t per = head + (size_t)P.dev_bytes;
   uint8_t* b = smem + per * wib;
   WarpSmem w;
   w.heap = reinterpret_cast<uint64_t*>(b);
@@ -346,7 +349,7 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
   w.logd = reinterpret_cast<uint8_t*>(w.sortk + P.sortcap);
   w.sortd = w.logd + P.ms;
   w.oplog = reinterpret_cast<uint32_t*>(w.sortd + P.sortcap);
-  w.dev = reinterpret_cast<int64_t*>(b + head);
+  w.dev = b + head;
   return w;
 }
 
@@ -1133,10 +1136,10 @@ struct Sim {
     while (__any_sync(kFullMask, todo)) {
       const uint32_t grp = __match_any_sync(kFullMask, todo ? (uint32_t)d : 256u + lane);
       if (todo && __ffs(grp) - 1 == (int)lane) {
-        const tm_t fd = (tm_t)dv.fr[d];
+        const tm_t fd = dv.fr[d];
         const tm_t s = r > fd ? r : fd;
         f = s + dur;
-        dv.fr[d] = (int64_t)f;
+        dv.fr[d] = f;
         todo = false;
       }
       __syncwarp();
@@ -1368,7 +1371,7 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>& S, cons
   S.holdb = reinterpret_cast<tm_t*>(sl + P.off_hold);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);
   S.creq = reinterpret_cast<int64_t*>(sl + P.off_creq);
-  S.dv.setup(P.g, w.dev);
+  S.dv.setup(P.g, w.dev, P.off_pk >= 0 ? reinterpret_cast<int64_t*>(sl + P.off_pk) : nullptr);
   S.T0 = -1;
   S.Tc = 0;
 }
