@@ -178,7 +178,7 @@ class Prepared:
     pass
 
 
-ARB_SOURCES = ("gmgsim_arb.cu", "gmg_arb.h")
+ARB_SOURCES = ("gmgsim_arb.cu", "gmg_arb.h", "gmg_arb_events.h")
 
 
 def rows_of(wl, ks, structured=False):
@@ -187,7 +187,8 @@ def rows_of(wl, ks, structured=False):
     return wl.structured_full_rows(ks) if structured else wl.full_rows(ks)
 
 
-def prepare(config: int, rank: int, world: int, device, cap=None, arbitrated=False, structured=False):
+def prepare(config: int, rank: int, world: int, device, cap=None, arbitrated=False, structured=False,
+            staging="default"):
     """Inputs of one rank, resident on its device: its contiguous block of
     the full placements and of the incremental move lists (the base row and
     the graph are replicated), outputs, two scratch buffers (the two halves
@@ -201,6 +202,7 @@ def prepare(config: int, rank: int, world: int, device, cap=None, arbitrated=Fal
     p.wl = wl
     p.arb = arbitrated
     p.structured = structured
+    p.staging = {"default": G.GMG_STAGING_DEFAULT, "shared": G.GMG_STAGING_SHARED, "l1": G.GMG_STAGING_L1}[staging]
     if arbitrated and wl.desc.n_dev > 256:
         raise SystemExit("--arbitrated needs at most 256 accelerators")
     if structured and (wl.n_full == 0 or wl.moves is not None):
@@ -273,7 +275,8 @@ def run_step(p, ev=None):
     if p.n_full:
         if ev:
             ev["full"][0].record()
-        G.sim_batch(p.g, p.place, out=_views(p.out, 0, p.n_full), scratch=p.scratch, arbitrated=p.arb)
+        G.sim_batch(p.g, p.place, out=_views(p.out, 0, p.n_full), scratch=p.scratch, arbitrated=p.arb,
+                    gmg_staging=p.staging)
         if ev:
             ev["full"][1].record()
         launches += 1
@@ -736,6 +739,9 @@ def main():
     ap.add_argument("--placements", default="uniform", choices=["uniform", "structured"],
                     help="full placement rows: uniform i.i.d. device ids, or contiguous per-request "
                          "stages on random accelerators")
+    ap.add_argument("--gmg-staging", default="default", choices=["default", "shared", "l1"],
+                    help="full placements: the GMG's hot fields staged in every CTA's shared memory, or read "
+                         "through the L1 path (default: the library's choice)")
     ap.add_argument("--candidates", type=int, default=None,
                     help="profiling aid: simulate only the first N candidates of each half "
                          "(the line then describes that smaller batch)")
@@ -762,7 +768,7 @@ def main():
     from paper_2608_15762_gb300 import build as lib_build
     lib_build.build()
     p = prepare(args.config, rank, world, device, cap=args.candidates, arbitrated=args.arbitrated,
-                structured=args.placements == "structured")
+                structured=args.placements == "structured", staging=args.gmg_staging)
     flush = torch.empty(256 << 20, dtype=torch.uint8, device=device)
 
     def barrier():
@@ -834,7 +840,8 @@ def main():
     props = torch.cuda.get_device_properties(device)
     issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
     arb_kern = "sim_arb_kernel" if D <= 32 else "sim_arbw_kernel"
-    kname = {"full": arb_kern if p.arb else "sim_full_kernel", "inc": arb_kern if p.arb else "sim_inc_kernel",
+    full_kern = "sim_full_staged_kernel" if p.staging == 1 else "sim_full_kernel"
+    kname = {"full": arb_kern if p.arb else full_kern, "inc": arb_kern if p.arb else "sim_inc_kernel",
              "base": "sim_base_kernel"}
     kcount = {"full": p.n_full, "inc": p.n_inc, "base": 1}
     out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
@@ -885,6 +892,7 @@ def main():
                    "incremental_candidates": p.n_inc_total, "n_ops": N, "n_dev": D,
                    "transfers": "arbitrated" if p.arb else "latency",
                    "placements": "structured" if p.structured else "uniform",
+                   "gmg_staging": args.gmg_staging,
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
                    "parallelism": "dp%d over candidates (contiguous blocks of each half per rank)" % world},
         # full placements simulate every op; an incremental candidate re-simulates

@@ -116,6 +116,20 @@ typedef struct {
 typedef struct gmg gmg_t;           /* opaque; host metadata + borrowed device workspace */
 typedef struct gmg_base gmg_base_t; /* opaque; base schedule snapshot for incremental runs */
 
+/* sim_opts_t.gmg_staging: where sim_batch's warps read the GMG's hot fields
+ * (durations, transfer sizes, flags, releases, both CSR lists) when they start
+ * ops and test successors.  GMG_STAGING_SHARED: each CTA (one per SM, up to 28
+ * warps) first copies a compact 16-byte record per op, the releases and both
+ * lists into shared memory with bulk copies; needs one accelerator type,
+ * uniform links, every time below 2^31 and the copy within the CTA's shared
+ * memory, else GMG_EINVAL.  GMG_STAGING_L1: 4-warp CTAs read the 64-byte op
+ * records through the read-only L1 path.  GMG_STAGING_DEFAULT picks
+ * GMG_STAGING_L1, the faster one on the prefill workload (Sec. 3.3.2
+ * simulator construction reads the same fields either way). */
+#define GMG_STAGING_DEFAULT 0
+#define GMG_STAGING_SHARED 1
+#define GMG_STAGING_L1 2
+
 /* sim_opts_t.transfer_mode */
 #define GMG_TRANSFER_LATENCY 0    /* a transfer starts when its producer finishes (Sec. 3.3.2) */
 #define GMG_TRANSFER_ARBITRATED 1 /* transfers wait for the arbiter (Sec. 3.5.2); sim_batch only */
@@ -127,7 +141,8 @@ typedef struct {
   int32_t queue_cap;        /* per-candidate event-queue entries; 0 = library default */
   int32_t warps_per_block;  /* 0 = library default (tuning knob) */
   int32_t transfer_mode;    /* GMG_TRANSFER_*; 0 = GMG_TRANSFER_LATENCY */
-  int32_t reserved[3];      /* must be 0 */
+  int32_t gmg_staging;      /* GMG_STAGING_*; sim_batch with pure-latency transfers only */
+  int32_t reserved[2];      /* must be 0 */
 } sim_opts_t;
 
 /* Caller-owned device output arrays for K candidates. */

@@ -20,7 +20,7 @@ CSRC = os.path.join(HERE, "csrc")
 OUT = os.path.join(HERE, "libgmgsim.so")
 SOURCES = ["gmgsim_host.cu", "gmgsim_kernels.cu", "gmgsim_full.cu", "gmgsim_inc.cu", "gmgsim_arb.cu",
            "gmgsim_arbw.cu", "gmgest.cu", "gmground.cu"]
-HEADERS = ["gmg_layout.h", "gmg_access.h", "gmg_arb.h", "gmg_arbw.h", "gmgsim_sim.cuh", os.path.join("..", "..", "include", "gmgsim.h"),
+HEADERS = ["gmg_layout.h", "gmg_access.h", "gmg_arb.h", "gmg_arbw.h", "gmg_arb_events.h", "gmgsim_sim.cuh", os.path.join("..", "..", "include", "gmgsim.h"),
            os.path.join("..", "..", "include", "gmgest.h"), os.path.join("..", "..", "include", "gmground.h")]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-Wall"]

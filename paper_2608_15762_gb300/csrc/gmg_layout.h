@@ -100,7 +100,25 @@ struct DevGmg {
   const uint8_t* dtype;       // [D] type of each accelerator
   int32_t uniform;
   int32_t batch;              // 1: the kernels take READY keys in batches (keys carry kQB class bits)
+  // The hot fields in the compact form a CTA stages into shared memory
+  // (sim_full_staged_kernel); present when stage_ok.
+  const uint4* st_hot;        // [N] {dur, xq | flags << 29, succ_off | nsucc << 24, pred_off | npred << 24}
+  const int32_t* st_rel;      // [N] release
+  int32_t stage_ok;           // 1: 32-bit times, one type, uniform links, lists and sizes fit the fields
+  int32_t n_edges;
 };
+
+// Bytes of the staged copy in shared memory: an mbarrier, then the four
+// arrays, each padded to 16 bytes (bulk copies move multiples of 16 bytes).
+#if defined(__CUDACC__)
+__host__ __device__
+#endif
+inline int64_t stage_smem_bytes(int64_t n, int64_t E) {
+  return 16 + 16 * n + (4 * n + 15) / 16 * 16 + 2 * ((4 * E + 15) / 16 * 16);
+}
+
+// The staged-GMG kernel's largest CTA (one per SM; 72 registers a thread).
+constexpr int kStageMaxWarps = 28;
 
 // Batched sweep: a READY key is followed by kQB bits holding floor(log2) of a
 // lower bound of the op's duration (31 at most).
@@ -178,7 +196,7 @@ struct SimParams {
   uint8_t* scratch;
   int64_t slot_bytes;    // scratch bytes per warp slot
   int32_t dev_bytes;     // shared bytes of accelerator state per warp
-  int32_t pad_;
+  int32_t stage_bytes;   // shared bytes of the staged GMG copy (sim_full_staged_kernel), else 0
   // byte offsets inside a slot (off_pk < 0: the peaks are in shared memory)
   int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row, off_pk;
 };

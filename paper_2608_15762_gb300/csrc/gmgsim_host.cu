@@ -19,7 +19,9 @@ namespace gsim {
 size_t select_rank_bytes();
 const void* full_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch);
 const void* inc_kernel_ptr(bool reg, bool key, bool t32, bool types, bool batch);
+const void* full_staged_kernel_ptr();
 cudaError_t launch_full(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
+cudaError_t launch_full_staged(const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_inc(bool reg, const SimParams& P, int grid, int block, size_t smem, cudaStream_t st);
 cudaError_t launch_base(bool reg, const SimParams& P, size_t smem, cudaStream_t st);
 cudaError_t set_smem_limits(int smem);
@@ -51,7 +53,7 @@ size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
 
 struct Layout {
   size_t off_ops, off_succ, off_pred, off_sib, off_cons, off_roots, off_roots_q, off_cap, off_base, off_avail,
-      off_dl, off_links, off_durt, off_dtype, off_linkid, total;
+      off_dl, off_links, off_durt, off_dtype, off_linkid, off_st_hot, off_st_rel, total;
 };
 
 // Everything gmg_create derives from a description.
@@ -69,6 +71,10 @@ struct Built {
   std::vector<uint16_t> linkid;  // [D*D] communication link of each ordered pair
   int64_t xfer_bound = 0;     // transfers of one placement at most: sum of min(successors, D-1)
   bool shared_links = false;  // two distinct ordered pairs share a link id
+  // compact hot records for a CTA's staged copy (sim_opts_t.gmg_staging = 1)
+  bool stage_ready = false;
+  std::vector<uint32_t> st_hot;  // [4n]
+  std::vector<int32_t> st_rel;   // [n]
   Layout L{};
 };
 
@@ -114,6 +120,8 @@ void plan(Built& b) {
   L.off_durt = take(8 * b.durt.size());
   L.off_dtype = take(b.dtype.size());
   L.off_linkid = take(2 * b.linkid.size());
+  L.off_st_hot = take(b.stage_ready ? 16 * (size_t)b.n : 0);
+  L.off_st_rel = take(b.stage_ready ? align_up(4 * (size_t)b.n, 16) : 0);
   L.total = o;
 }
 
@@ -401,6 +409,26 @@ int build(const gmg_desc_t* d, Built& b) {
       b.roots.push_back(((uint64_t)b.ops[i].release << (b.ib + 2)) | (uint64_t)i);
   std::sort(b.roots.begin(), b.roots.end());
   b.nroots = (int)b.roots.size();
+  // compact records for the staged copy: one accelerator type, uniform links,
+  // every time below 2^31, lists addressable in 24 bits with fewer than 256
+  // entries per op, transfer sizes (xq) below 2^29
+  b.stage_ready = !b.T && b.uniform && b.time_bound < (int64_t(1) << 31) && b.E < (1 << 24);
+  for (int i = 0; i < n && b.stage_ready; ++i) {
+    const OpRec& r = b.ops[i];
+    b.stage_ready = r.nsucc < 256 && r.npred < 256 && r.xq < (int64_t(1) << 29);
+  }
+  if (b.stage_ready) {
+    b.st_hot.resize(4 * (size_t)n);
+    b.st_rel.resize(n);
+    for (int i = 0; i < n; ++i) {
+      const OpRec& r = b.ops[i];
+      b.st_hot[4 * (size_t)i] = (uint32_t)r.dur;
+      b.st_hot[4 * (size_t)i + 1] = (uint32_t)r.xq | ((r.flags & 7u) << 29);
+      b.st_hot[4 * (size_t)i + 2] = r.succ_off | (r.nsucc << 24);
+      b.st_hot[4 * (size_t)i + 3] = r.pred_off | (r.npred << 24);
+      b.st_rel[i] = (int32_t)r.release;
+    }
+  }
   plan(b);
   return GMG_OK;
 }
@@ -550,7 +578,44 @@ int check_out(const sim_out_t* o, const sim_opts_t* opts) {
       if (r != 0) return GMG_EINVAL;
     if (opts->transfer_mode != GMG_TRANSFER_LATENCY && opts->transfer_mode != GMG_TRANSFER_ARBITRATED)
       return GMG_EINVAL;
+    if (opts->gmg_staging < GMG_STAGING_DEFAULT || opts->gmg_staging > GMG_STAGING_L1) return GMG_EINVAL;
   }
+  return GMG_OK;
+}
+
+bool staged(const sim_opts_t* o) { return o && o->gmg_staging == GMG_STAGING_SHARED; }
+
+bool g_stage_smem_set = false;
+
+// sim_batch with the GMG staged in shared memory: one CTA per SM with as many
+// warps (up to kStageMaxWarps) as fit beside the staged copy.
+int plan_staged(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L) {
+  const DevGmg& G = g->dg;
+  if (!G.stage_ok || (o && o->transfer_mode != GMG_TRANSFER_LATENCY)) return GMG_EINVAL;
+  int rc = plan_launch(g, K, o, false, L);
+  if (rc) return rc;
+  int dev = 0, optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess)
+    return GMG_ECUDA;
+  SimParams& P = L.P;
+  P.stage_bytes = (int32_t)stage_smem_bytes(G.n, G.n_edges);
+  const size_t spw = smem_per_warp(P);
+  const int64_t room = (int64_t)optin - P.stage_bytes;
+  const int w = (int)std::min<int64_t>(kStageMaxWarps, room > 0 ? room / (int64_t)spw : 0);
+  if (w < 1) return GMG_EINVAL;
+  if (!g_stage_smem_set) {
+    if (cudaFuncSetAttribute(full_staged_kernel_ptr(), cudaFuncAttributeMaxDynamicSharedMemorySize, optin) !=
+        cudaSuccess)
+      return GMG_ECUDA;
+    g_stage_smem_set = true;
+  }
+  const int sms = device_sms();
+  if (sms <= 0) return GMG_ECUDA;
+  L.wpb = w;
+  L.smem = (size_t)P.stage_bytes + (size_t)w * spw;
+  L.grid = (int)std::min<int64_t>(sms, ((int64_t)std::max(K, 1) + w - 1) / w);
+  L.slots = (int64_t)L.grid * w;
   return GMG_OK;
 }
 
@@ -821,6 +886,10 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
     put(L.off_dtype, b.dtype.data(), b.dtype.size());
   }
   put(L.off_linkid, b.linkid.data(), 2 * b.linkid.size());
+  if (b.stage_ready) {
+    put(L.off_st_hot, b.st_hot.data(), 4 * b.st_hot.size());
+    put(L.off_st_rel, b.st_rel.data(), 4 * b.st_rel.size());
+  }
   cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
   if (cudaMemcpyAsync(d_ws, host.data(), b.L.total, cudaMemcpyHostToDevice, st) != cudaSuccess)
     return GMG_ECUDA;
@@ -854,6 +923,10 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.tb = tb;
   G.dev_key = dev_key ? 1 : 0;
   G.batch = batch ? 1 : 0;
+  G.st_hot = reinterpret_cast<const uint4*>(w + L.off_st_hot);
+  G.st_rel = reinterpret_cast<const int32_t*>(w + L.off_st_rel);
+  G.stage_ok = (b.stage_ready && G.t32 && G.D <= 32) ? 1 : 0;
+  G.n_edges = b.E;
   // every time < 2^tb fits int32; the 32-bit instances also take the
   // accelerator id from the event key
   G.t32 = (G.tb <= 31 && G.dev_key) ? 1 : 0;
@@ -895,7 +968,7 @@ size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
   if (arbitrated(opts)) {
     ArbPlan Q;
     if (plan_arb_any(g, K, opts, L, Q)) return 0;
-  } else if (plan_launch(g, K, opts, false, L)) {
+  } else if (staged(opts) ? plan_staged(g, K, opts, L) : plan_launch(g, K, opts, false, L)) {
     return 0;
   }
   return (size_t)L.slots * (size_t)L.P.slot_bytes;
@@ -911,7 +984,9 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   Launch L;
   ArbPlan Q;
   const bool arb = arbitrated(opts);
-  rc = arb ? plan_arb_any(g, K, opts, L, Q) : plan_launch(g, K, opts, false, L);
+  const bool stg = staged(opts);
+  rc = arb ? (stg ? GMG_EINVAL : plan_arb_any(g, K, opts, L, Q))
+           : (stg ? plan_staged(g, K, opts, L) : plan_launch(g, K, opts, false, L));
   if (rc) return rc;
   if (!d_scratch || !aligned(d_scratch, 256) ||
       scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
@@ -923,7 +998,9 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   P.K = K;
   P.scratch = static_cast<uint8_t*>(d_scratch);
   const cudaStream_t st = reinterpret_cast<cudaStream_t>(stream);
-  cudaError_t e = arb ? launch_arb_any(g, L, Q, nullptr, st) : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
+  cudaError_t e = arb ? launch_arb_any(g, L, Q, nullptr, st)
+                      : stg ? launch_full_staged(P, L.grid, 32 * L.wpb, L.smem, st)
+                            : launch_full(L.reg, P, L.grid, 32 * L.wpb, L.smem, st);
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 
@@ -973,6 +1050,7 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
   if (rc) return rc;
   if (K == 0) return GMG_OK;
   if (!d_place || ld < g->dg.n || ld % 16 != 0 || !aligned(d_place, 16)) return GMG_EINVAL;
+  if (staged(opts)) return GMG_EINVAL;  // the staged copy's CTA shape is not planned for the fixed buffer
   Launch L;
   ArbPlan Q;
   const bool arb = arbitrated(opts);
@@ -1095,6 +1173,7 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
   if (!g || !b || b->g != g || K < 0) return GMG_EINVAL;
   int rc = check_out(d_out, opts);
   if (rc) return rc;
+  if (staged(opts)) return GMG_EINVAL;  // staging applies to sim_batch
   if (K == 0) return GMG_OK;
   if (!d_move_off) return GMG_EINVAL;
   if (arbitrated(opts)) {

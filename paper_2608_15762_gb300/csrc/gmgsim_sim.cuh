@@ -362,10 +362,15 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
 // kTypes: the graph has several accelerator types (durations per (type, op)).
 // kBatch: the batched sweep (run_batched), for accelerator state in shared
 // memory with the accelerator id in the event key.
-template <bool kReg, int kMode, bool kKey, bool kT32 = false, bool kTypes = false, bool kBatch = false>
+// kStage: the hot fields of the GMG (durations, transfer sizes, flags, both
+// CSR lists, releases) are read from the CTA's shared-memory copy (staged by
+// sim_full_staged_kernel) when starting ops and testing successors.
+template <bool kReg, int kMode, bool kKey, bool kT32 = false, bool kTypes = false, bool kBatch = false,
+          bool kStage = false>
 struct Sim {
   static_assert(!(kT32 && kMode == kBase), "the base snapshot keeps 64-bit times");
   static_assert(!kBatch || (!kReg && kKey), "the batched sweep keeps accelerator state in shared memory");
+  static_assert(!kStage || (kMode == kFull && kT32 && !kTypes && !kBatch), "staged GMG: 32-bit, one type");
   using tm_t = typename std::conditional<kT32, int32_t, int64_t>::type;
   const SimParams& P;
   const DevGmg& g;
@@ -401,6 +406,11 @@ struct Sim {
   int64_t vt;
   // base checkpoints
   int ck, next_ck;
+  // staged GMG (kStage): shared copies
+  const uint4* sh_hot;      // per op {dur, xq | flags << 29, succ_off | nsucc << 24, pred_off | npred << 24}
+  const int32_t* sh_rel;    // per op release
+  const uint32_t* sh_succ;  // successor lists
+  const uint32_t* sh_pred;  // predecessor lists (hold bits included)
 
   __device__ Sim(const SimParams& p) : P(p), g(p.g) {
     kc.ib = g.ib;
@@ -536,6 +546,10 @@ struct Sim {
   // generation, and push the successors it makes ready.
   // -------------------------------------------------------------------------
   __device__ void start_op(uint32_t i, tm_t r) {
+    if constexpr (kStage) {
+      start_op_staged(i, r);
+      return;
+    }
     const unsigned lane = lane_id();
     const longlong2 db = op_durbytes(g.ops, i);
     const XqSucc xs = op_xqsucc(g.ops, i);
@@ -590,6 +604,66 @@ struct Sim {
             }
             const int dp = row[p];
             if (dp != dj) a += xfer(dp, dj, op_durbytes(g.ops, p).y, op_xqsucc(g.ops, p).xq);
+            rj = a > rj ? a : rj;
+          }
+        }
+      }
+      uint32_t m = __ballot_sync(kFullMask, rdy);
+      while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        push_ready(__shfl_sync(kFullMask, kc.make(rj, kReady, j), src));
+      }
+    }
+  }
+
+  // start_op with the hot fields from the CTA's staged copy of the GMG (the
+  // links are uniform: a transfer takes xq + lat0).
+  __device__ void start_op_staged(uint32_t i, tm_t r) {
+    const unsigned lane = lane_id();
+    const uint4 h = sh_hot[i];
+    const uint32_t flags = h.y >> 29;
+    const tm_t xq = (tm_t)(h.y & 0x1fffffffu);
+    const uint32_t succ_off = h.z & 0xffffffu, nsucc = h.z >> 24;
+    const int d = row[i];
+    const tm_t fd = dv.get_free(d);
+    const tm_t s = r > fd ? r : fd;
+    const tm_t f = s + (tm_t)(int32_t)h.x;
+    dv.set_free(d, f);
+    if (lane == 0) {
+      fbuf[i] = f;
+      if (flags & kReqSink)
+        atomicMax(reinterpret_cast<unsigned long long*>(creq + (int32_t)op_cons(g.ops, i).z), (unsigned long long)f);
+      oplog[opn] = i;
+    }
+    ++opn;
+    if (flags & kScored) score += (int64_t)f;
+    __syncwarp();
+    const tm_t lat = (tm_t)g.lat0;
+    for (uint32_t c0 = 0; c0 < nsucc; c0 += 32) {
+      const uint32_t t = c0 + lane;
+      uint32_t j = 0;
+      tm_t rj = 0;
+      bool rdy = false;
+      if (t < nsucc) {
+        j = sh_succ[succ_off + t];
+        const int dj = row[j];
+        const tm_t arr = dj != d ? f + xq + lat : f;
+        const uint32_t po = sh_hot[j].w;
+        const uint32_t npred = po >> 24, pred_off = po & 0xffffffu;
+        const tm_t rel = (tm_t)sh_rel[j];
+        rj = rel > arr ? rel : arr;
+        rdy = true;
+        if (npred > 1) {
+          for (uint32_t k = 0; k < npred; ++k) {
+            const uint32_t p = sh_pred[pred_off + k] & kIdMask;
+            if (p == i) continue;
+            tm_t a = fin(p);
+            if (a <= 0) {  // not started yet
+              rdy = false;
+              break;
+            }
+            if (row[p] != dj) a += (tm_t)(sh_hot[p].y & 0x1fffffffu) + lat;
             rj = a > rj ? a : rj;
           }
         }
@@ -1303,8 +1377,8 @@ struct Sim {
 // READY heap, event log, partial results; the ops started by then are those
 // with base ready time < T_c.  An incremental candidate whose resume time T0
 // is >= T_c restarts there.
-template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes, bool kBatch>
-__device__ void Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>::maybe_checkpoint(uint64_t next_key) {
+template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes, bool kBatch, bool kStage>
+__device__ void Sim<kReg, kMode, kKey, kT32, kTypes, kBatch, kStage>::maybe_checkpoint(uint64_t next_key) {
   if (kMode != kBase) return;
   const DevBase& B = P.base;
   if (next_key == kKeyMax || ck >= B.nck || readypops < next_ck) return;
@@ -1344,8 +1418,8 @@ __device__ void Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>::maybe_checkpoint(u
   __syncwarp();
 }
 
-template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes, bool kBatch>
-__device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>& S, const SimParams& P, unsigned wib,
+template <bool kReg, int kMode, bool kKey, bool kT32, bool kTypes, bool kBatch, bool kStage>
+__device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes, kBatch, kStage>& S, const SimParams& P, unsigned wib,
                            int64_t slot, uint8_t* smem) {
   uint8_t* sl = P.scratch + slot * P.slot_bytes;
   const WarpSmem w = carve_smem(smem, P, wib);
@@ -1366,7 +1440,7 @@ __device__ void setup_slot(Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>& S, cons
   S.oplog = w.oplog;
   S.opn = 0;
   S.sortcap = P.sortcap;
-  using tm_t = typename Sim<kReg, kMode, kKey, kT32, kTypes, kBatch>::tm_t;
+  using tm_t = typename Sim<kReg, kMode, kKey, kT32, kTypes, kBatch, kStage>::tm_t;
   S.fbuf = reinterpret_cast<tm_t*>(sl + P.off_f);
   S.holdb = reinterpret_cast<tm_t*>(sl + P.off_hold);
   S.bits = reinterpret_cast<uint32_t*>(sl + P.off_bits);

@@ -73,7 +73,7 @@ class _Desc(C.Structure):
 class _Opts(C.Structure):
     _fields_ = [("score_mode", C.c_int32), ("n_trace", C.c_int32), ("d_trace_k", C.c_void_p),
                 ("queue_cap", C.c_int32), ("warps_per_block", C.c_int32),
-                ("transfer_mode", C.c_int32), ("reserved", C.c_int32 * 3)]
+                ("transfer_mode", C.c_int32), ("gmg_staging", C.c_int32), ("reserved", C.c_int32 * 2)]
 
 
 class _Out(C.Structure):
@@ -168,9 +168,14 @@ def gmg_workspace_bytes(desc) -> int:
     return int(lib().gmg_workspace_bytes(C.addressof(h.c)))
 
 
-def _opts(score_mode=0, trace_k=None, queue_cap=0, warps_per_block=0, arbitrated=False) -> _Opts:
+GMG_STAGING_DEFAULT, GMG_STAGING_SHARED, GMG_STAGING_L1 = 0, 1, 2
+
+
+def _opts(score_mode=0, trace_k=None, queue_cap=0, warps_per_block=0, arbitrated=False,
+          gmg_staging=GMG_STAGING_DEFAULT) -> _Opts:
     o = _Opts()
     o.transfer_mode = GMG_TRANSFER_ARBITRATED if arbitrated else GMG_TRANSFER_LATENCY
+    o.gmg_staging = int(gmg_staging)
     o.score_mode = score_mode
     o.n_trace = 0 if trace_k is None else int(trace_k.numel())
     o.d_trace_k = None if trace_k is None else trace_k.data_ptr()
@@ -317,16 +322,18 @@ class Scratch:
 @_traced("sim_batch")
 def sim_batch(g: Gmg, place, out: Optional[SimOut] = None, scratch: Optional[Scratch] = None,
               req_done=False, trace_k=None, queue_cap=0, warps_per_block=0, stream=None,
-              arbitrated=False) -> SimOut:
+              arbitrated=False, gmg_staging=GMG_STAGING_DEFAULT) -> SimOut:
     """Simulate every row of ``place`` (CUDA uint8 [K, ld], ld % 16 == 0);
-    ``arbitrated``: transfers go through the arbiter of Sec. 3.5.2."""
+    ``arbitrated``: transfers go through the arbiter of Sec. 3.5.2;
+    ``gmg_staging``: GMG_STAGING_SHARED stages the GMG's hot fields in every
+    CTA's shared memory, GMG_STAGING_L1 reads them through the L1 path."""
     import torch
     assert place.dtype == torch.uint8 and place.dim() == 2 and place.is_contiguous()
     K, ld = place.shape
     n_trace = 0 if trace_k is None else int(trace_k.numel())
     if out is None:
         out = SimOut.empty(K, g.n_dev, g.n_req, place.device, req_done, n_trace, g.n_ops)
-    o = _opts(0, trace_k, queue_cap, warps_per_block, arbitrated)
+    o = _opts(0, trace_k, queue_cap, warps_per_block, arbitrated, gmg_staging)
     need = lib().sim_scratch_bytes(g.handle, K, C.addressof(o))
     scratch = scratch or Scratch(place.device)
     buf = scratch.get(need)

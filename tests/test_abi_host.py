@@ -111,10 +111,14 @@ def test_link_id_validation_and_option_layout():
     assert G.gmg_workspace_bytes(linked([-7, 3, 2, 99])) > 0    # the diagonal is not read
     assert _create_rc(linked([0, 4, 1, 0])) == G.GMG_EINVAL     # id >= D*D
     assert _create_rc(linked([0, -1, 1, 0])) == G.GMG_EINVAL
-    # sim_opts_t: transfer_mode takes the first reserved word; the struct size is unchanged
+    # sim_opts_t: transfer_mode and gmg_staging take reserved words; the struct size is unchanged
     assert C.sizeof(G._Opts) == 40 and G._Opts.transfer_mode.offset == 24
+    assert G._Opts.gmg_staging.offset == 28 and G._Opts.reserved.offset == 32
     hdr = open(os.path.join(ROOT, "include", "gmgsim.h")).read()
-    assert re.search(r"int32_t transfer_mode;.*\n\s*int32_t reserved\[3\];", hdr)
+    assert re.search(r"int32_t transfer_mode;.*\n\s*int32_t gmg_staging;.*\n\s*int32_t reserved\[2\];", hdr)
+    for name, v in (("DEFAULT", 0), ("SHARED", 1), ("L1", 2)):
+        assert re.search(r"#define GMG_STAGING_%s %d\b" % (name, v), hdr)
+        assert getattr(G, "GMG_STAGING_" + name) == v
     assert "const int32_t* link_id;" in hdr and G._Desc.link_id.offset == C.sizeof(G._Desc) - 8
 
 

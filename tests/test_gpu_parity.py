@@ -247,3 +247,47 @@ def test_workload_large_full_size_sampled():
     si, pki, rqi = O.incremental_batch(wl.desc, wl.base_place, wl.moves.subset(ki))
     compare(goti, si, pki, rqi, ks=ki)
     assert best.cpu().tolist()[1] == int(got["score"].min())
+
+
+# ---------------------------------------------------------------------------
+# The GMG staged in shared memory (sim_opts_t.gmg_staging)
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("which", ["tiny", "prefill", "random", "random_wide"])
+def test_staged_gmg_bit_exact(which):
+    """sim_batch with each CTA's warps reading the hot GMG fields from a
+    shared-memory copy made with bulk copies: every candidate against the
+    oracle, and the same bytes as the L1 path."""
+    if which in ("tiny", "prefill"):
+        wl = W.config1() if which == "tiny" else W.config2()
+        d, rows = wl.desc, wl.all_full_rows()
+    else:
+        D = 6 if which == "random" else 32
+        d = W.random_desc(61 if which == "random" else 62, 700, D, link_hetero=False, explicit_cons=True,
+                          window=12 if which == "random" else 200)
+        rows = _random_case(61, 700, D, link_hetero=False)[1]
+        rows = np.concatenate([rows] * 40)[:1000]
+    g = G.gmg_create(d)
+    tk = torch.tensor([0, rows.shape[0] - 1], dtype=torch.int32, device="cuda")
+    st = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk, gmg_staging=G.GMG_STAGING_SHARED)
+    l1 = G.sim_batch(g, torch_place(rows), req_done=True, trace_k=tk, gmg_staging=G.GMG_STAGING_L1)
+    torch.cuda.synchronize()
+    got = st.to_numpy()
+    s, pk, rq = oracle_rows(d, rows)
+    compare(got, s, pk, rq)
+    ref = l1.to_numpy()
+    for f in ("trace_start", "trace_finish", "peak", "req_done", "score", "makespan"):
+        assert np.array_equal(got[f], ref[f]), f
+
+
+def test_staging_refused_where_it_does_not_apply():
+    """Two accelerator types, per-pair links or arbitrated transfers: the
+    compact staged record does not hold them, and the call says so."""
+    rows = np.zeros((4, 320), np.uint8)
+    for d, arb in ((W.random_desc(63, 300, 4, n_types=2, link_hetero=False), False),
+                   (W.random_desc(64, 300, 4, link_hetero=True), False),
+                   (W.random_desc(65, 300, 4, link_hetero=False), True)):
+        g = G.gmg_create(d)
+        with pytest.raises(G.GmgError) as e:
+            G.sim_batch(g, torch_place(rows), gmg_staging=G.GMG_STAGING_SHARED, arbitrated=arb)
+        assert e.value.code == G.GMG_EINVAL
