@@ -840,7 +840,8 @@ def main():
     props = torch.cuda.get_device_properties(device)
     issue_peak = props.multi_processor_count * 4 * pk["sm_max_mhz"] * 1e6 / 1e9  # Ginst/s
     arb_kern = "sim_arb_kernel" if D <= 32 else "sim_arbw_kernel"
-    full_kern = "sim_full_staged_kernel" if p.staging == 1 else "sim_full_kernel"
+    staged_run = p.staging == 1 or (p.staging == 0 and p.g.info["stageable"] == 1 and not p.arb)
+    full_kern = "sim_full_staged_kernel" if staged_run else "sim_full_kernel"
     kname = {"full": arb_kern if p.arb else full_kern, "inc": arb_kern if p.arb else "sim_inc_kernel",
              "base": "sim_base_kernel"}
     kcount = {"full": p.n_full, "inc": p.n_inc, "base": 1}
@@ -892,7 +893,7 @@ def main():
                    "incremental_candidates": p.n_inc_total, "n_ops": N, "n_dev": D,
                    "transfers": "arbitrated" if p.arb else "latency",
                    "placements": "structured" if p.structured else "uniform",
-                   "gmg_staging": args.gmg_staging,
+                   "gmg_staging": "shared memory (bulk-copied once per CTA)" if staged_run else "L1 path",
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",
                    "parallelism": "dp%d over candidates (contiguous blocks of each half per rank)" % world},
         # full placements simulate every op; an incremental candidate re-simulates

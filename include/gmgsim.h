@@ -121,11 +121,12 @@ typedef struct gmg_base gmg_base_t; /* opaque; base schedule snapshot for increm
  * ops and test successors.  GMG_STAGING_SHARED: each CTA (one per SM, up to 28
  * warps) first copies a compact 16-byte record per op, the releases and both
  * lists into shared memory with bulk copies; needs one accelerator type,
- * uniform links, every time below 2^31 and the copy within the CTA's shared
- * memory, else GMG_EINVAL.  GMG_STAGING_L1: 4-warp CTAs read the 64-byte op
- * records through the read-only L1 path.  GMG_STAGING_DEFAULT picks
- * GMG_STAGING_L1, the faster one on the prefill workload (Sec. 3.3.2
- * simulator construction reads the same fields either way). */
+ * uniform links, every time below 2^31, at most 32 accelerators and the copy
+ * within the CTA's shared memory, else GMG_EINVAL.  GMG_STAGING_L1: 4-warp
+ * CTAs read the 64-byte op records through the read-only L1 path.
+ * GMG_STAGING_DEFAULT stages wherever staging applies (measured faster on the
+ * prefill workload) and takes the L1 path elsewhere; sim_batch_noalloc always
+ * takes the L1 path (and refuses GMG_STAGING_SHARED). */
 #define GMG_STAGING_DEFAULT 0
 #define GMG_STAGING_SHARED 1
 #define GMG_STAGING_L1 2
@@ -174,6 +175,9 @@ typedef struct {
   int32_t batched_sweep; /* 1 if the simulation kernels start READY ops in batches (graphs on
                             more than 32 accelerators whose keys have room for a duration class) */
   int32_t t32;           /* 1 if the kernels carry times as 32-bit integers (time_bound < 2^31) */
+  int32_t stageable;     /* 1 if sim_batch can stage this graph's hot fields in shared memory
+                            (GMG_STAGING_SHARED; the default then does, with pure-latency transfers) */
+  int32_t reserved_;
 } gmg_info_t;
 
 /* ---------------------------------------------------------------------- */

@@ -38,7 +38,19 @@ constexpr int64_t kI64Max = 0x7fffffffffffffffll;
 constexpr int kMaxOpsLog2 = 28;          // op ids must fit the packed key
 constexpr int kDefaultWarpsPerBlock = 4;
 constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
-constexpr int kSharedQueueEntriesBatch = 225;  // 1 + 32 * 7: the batched sweep's wider frontier
+// The batched sweep's sizes (compile-time overridable for tuning sweeps).
+#ifndef GMG_BATCH_QUEUE_SHARED
+#define GMG_BATCH_QUEUE_SHARED 225  // 1 + 32 * 7: the wider frontier of many tenants
+#endif
+#ifndef GMG_BATCH_OPS_PER_GENERATION
+#define GMG_BATCH_OPS_PER_GENERATION 24
+#endif
+#ifndef GMG_BATCH_LOG_SHARED
+#define GMG_BATCH_LOG_SHARED 192
+#endif
+constexpr int kSharedQueueEntriesBatch = GMG_BATCH_QUEUE_SHARED;
+constexpr int kBatchOpsPerGeneration = GMG_BATCH_OPS_PER_GENERATION;
+constexpr int kSharedLogEntriesBatch = GMG_BATCH_LOG_SHARED;
 constexpr int64_t kDefaultQueueCap = 1 << 16;
 constexpr int kSharedLogEntries = 192;
 constexpr int64_t kDefaultLogCap = 1 << 17;
@@ -512,11 +524,11 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   P.qs = batch ? kSharedQueueEntriesBatch : kSharedQueueEntries;  // >= 33 (the root's children are
                                                                      // always in shared memory)
   P.mcap = log_cap(g, o);
-  P.ms = kSharedLogEntries;
+  P.ms = batch ? kSharedLogEntriesBatch : kSharedLogEntries;
   P.sortcap = kSortCap;
   while (P.sortcap < G.D) P.sortcap <<= 1;
-  P.drain_trigger = kOpsPerGeneration;
-  P.opcap = batch ? kOpsPerGeneration + 32 : kOpsPerGeneration;
+  P.drain_trigger = batch ? kBatchOpsPerGeneration : kOpsPerGeneration;
+  P.opcap = batch ? kBatchOpsPerGeneration + 32 : kOpsPerGeneration;
   P.dev_bytes = dev_smem_bytes(G.D, G.t32 ? 4 : 8);
   L.smem = (size_t)L.wpb * smem_per_warp(P);
   size_t o2 = 0;
@@ -544,8 +556,9 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     SimParams big = P;
     big.g.D = 256;
     big.sortcap = 256;
-    big.opcap = kOpsPerGeneration + 32;
-    big.qs = kSharedQueueEntriesBatch;
+    big.opcap = std::max(kOpsPerGeneration, kBatchOpsPerGeneration + 32);
+    big.qs = std::max(kSharedQueueEntries, kSharedQueueEntriesBatch);
+    big.ms = std::max(kSharedLogEntries, kSharedLogEntriesBatch);
     big.dev_bytes = 24 * 256;
     if (set_smem_limits(4 * (int)smem_per_warp(big)) != cudaSuccess) return GMG_ECUDA;
     g_smem_set = true;
@@ -584,6 +597,7 @@ int check_out(const sim_out_t* o, const sim_opts_t* opts) {
 }
 
 bool staged(const sim_opts_t* o) { return o && o->gmg_staging == GMG_STAGING_SHARED; }
+bool l1_path(const sim_opts_t* o) { return o && o->gmg_staging == GMG_STAGING_L1; }
 
 bool g_stage_smem_set = false;
 
@@ -602,21 +616,39 @@ int plan_staged(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L) {
   P.stage_bytes = (int32_t)stage_smem_bytes(G.n, G.n_edges);
   const size_t spw = smem_per_warp(P);
   const int64_t room = (int64_t)optin - P.stage_bytes;
-  const int w = (int)std::min<int64_t>(kStageMaxWarps, room > 0 ? room / (int64_t)spw : 0);
-  if (w < 1) return GMG_EINVAL;
+  const int64_t fit = std::min<int64_t>(kStageMaxWarps, room > 0 ? room / (int64_t)spw : 0);
+  if (fit < 1) return GMG_EINVAL;
+  // as many warps per CTA as spread the candidates over every SM (few
+  // candidates: small CTAs on many SMs; many: up to what fits beside the copy)
+  const int sms = device_sms();
+  if (sms <= 0) return GMG_ECUDA;
+  const int w = (int)std::min<int64_t>(fit, std::max<int64_t>(1, ((int64_t)std::max(K, 1) + sms - 1) / sms));
   if (!g_stage_smem_set) {
     if (cudaFuncSetAttribute(full_staged_kernel_ptr(), cudaFuncAttributeMaxDynamicSharedMemorySize, optin) !=
         cudaSuccess)
       return GMG_ECUDA;
     g_stage_smem_set = true;
   }
-  const int sms = device_sms();
-  if (sms <= 0) return GMG_ECUDA;
   L.wpb = w;
   L.smem = (size_t)P.stage_bytes + (size_t)w * spw;
   L.grid = (int)std::min<int64_t>(sms, ((int64_t)std::max(K, 1) + w - 1) / w);
   L.slots = (int64_t)L.grid * w;
   return GMG_OK;
+}
+
+// Full placements with pure-latency transfers: the staged-GMG kernel when the
+// caller asks for it (an error if it cannot serve the graph) or by default
+// when it can, else the L1 path.  *stg tells which.
+int plan_full(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, bool* stg) {
+  *stg = false;
+  if (l1_path(o)) return plan_launch(g, K, o, false, L);
+  const int rc = plan_staged(g, K, o, L);
+  if (rc == GMG_OK) {
+    *stg = true;
+    return GMG_OK;
+  }
+  if (staged(o) || rc != GMG_EINVAL) return rc;
+  return plan_launch(g, K, o, false, L);
 }
 
 bool arbitrated(const sim_opts_t* o) { return o && o->transfer_mode == GMG_TRANSFER_ARBITRATED; }
@@ -894,7 +926,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   if (cudaMemcpyAsync(d_ws, host.data(), b.L.total, cudaMemcpyHostToDevice, st) != cudaSuccess)
     return GMG_ECUDA;
   if (cudaStreamSynchronize(st) != cudaSuccess) return GMG_ECUDA;
-  gmg* g = new (std::nothrow) gmg;
+  gmg* g = new (std::nothrow) gmg();
   if (!g) return GMG_ENOMEM;
   uint8_t* w = static_cast<uint8_t*>(d_ws);
   DevGmg& G = g->dg;
@@ -925,11 +957,11 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.batch = batch ? 1 : 0;
   G.st_hot = reinterpret_cast<const uint4*>(w + L.off_st_hot);
   G.st_rel = reinterpret_cast<const int32_t*>(w + L.off_st_rel);
-  G.stage_ok = (b.stage_ready && G.t32 && G.D <= 32) ? 1 : 0;
   G.n_edges = b.E;
   // every time < 2^tb fits int32; the 32-bit instances also take the
   // accelerator id from the event key
   G.t32 = (G.tb <= 31 && G.dev_key) ? 1 : 0;
+  G.stage_ok = (b.stage_ready && G.t32 && G.D <= 32) ? 1 : 0;
   G.uniform = b.uniform ? 1 : 0;
   gmg_info_t& I = g->info;
   std::memset(&I, 0, sizeof(I));
@@ -950,6 +982,7 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
   I.batched_sweep = G.batch;
   I.t32 = G.t32;
+  I.stageable = G.stage_ok;
   *out = g;
   return GMG_OK;
 }
@@ -968,8 +1001,9 @@ size_t sim_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
   if (arbitrated(opts)) {
     ArbPlan Q;
     if (plan_arb_any(g, K, opts, L, Q)) return 0;
-  } else if (staged(opts) ? plan_staged(g, K, opts, L) : plan_launch(g, K, opts, false, L)) {
-    return 0;
+  } else {
+    bool stg = false;
+    if (plan_full(g, K, opts, L, &stg)) return 0;
   }
   return (size_t)L.slots * (size_t)L.P.slot_bytes;
 }
@@ -984,9 +1018,8 @@ int sim_batch(const gmg_t* g, const uint8_t* d_place, int32_t K, int32_t ld, con
   Launch L;
   ArbPlan Q;
   const bool arb = arbitrated(opts);
-  const bool stg = staged(opts);
-  rc = arb ? (stg ? GMG_EINVAL : plan_arb_any(g, K, opts, L, Q))
-           : (stg ? plan_staged(g, K, opts, L) : plan_launch(g, K, opts, false, L));
+  bool stg = false;
+  rc = arb ? (staged(opts) ? GMG_EINVAL : plan_arb_any(g, K, opts, L, Q)) : plan_full(g, K, opts, L, &stg);
   if (rc) return rc;
   if (!d_scratch || !aligned(d_scratch, 256) ||
       scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)

@@ -87,7 +87,8 @@ class _Info(C.Structure):
                 ("n_req", C.c_int32), ("n_roots", C.c_int32), ("id_bits", C.c_int32),
                 ("time_bits", C.c_int32), ("uniform_links", C.c_int32),
                 ("time_bound", C.c_int64), ("default_queue_cap", C.c_int64),
-                ("batched_sweep", C.c_int32), ("t32", C.c_int32)]
+                ("batched_sweep", C.c_int32), ("t32", C.c_int32), ("stageable", C.c_int32),
+                ("reserved_", C.c_int32)]
 
 
 _LIB = None
