@@ -1077,7 +1077,7 @@ struct Sim {
   // The event loop (Sec. 3.3.3).
   __device__ void run() {
     if (status) return;
-    if (kBatch) {
+    if constexpr (kBatch) {
       run_batched();
       return;
     }
