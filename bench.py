@@ -332,25 +332,38 @@ def oracle_sample(wl, k_full, k_inc, nthreads, arbitrated=False, structured=Fals
     return runs
 
 
-def cpu_baseline(wl, min_s=10.0, arbitrated=False, structured=False, ev_budget=1.2e8):
+def cpu_baseline(wl, min_s=10.0, arbitrated=False, structured=False):
     """The CPU oracle as it stands on this host's cores, on a bounded sample
-    of each half of the workload (up to ~ev_budget op-events of candidates per
-    half, whole sample passes repeated until min_s seconds in all), scaled to
-    the workload's whole candidate mix: value = K / sum over halves of
-    (candidates of the half x measured seconds per candidate)."""
+    of each half of the workload, scaled to the workload's whole candidate
+    mix: value = K / sum over halves of (candidates of the half x measured
+    seconds per candidate).  The sample of a half is sized from a short probe
+    pass so that its timed passes take about min_s / (number of halves)
+    seconds; whole sample passes repeat until then."""
     from oracle import oracle as O
     nt = O.hw_threads()
-    budget = max(16, int(ev_budget // max(wl.desc.n_ops, 1)))
     n_inc = 0 if wl.moves is None else wl.moves.n_cand
-    runs = oracle_sample(wl, min(wl.n_full, budget), min(n_inc, budget), nt, arbitrated, structured)
-    total_s, total_s1, parts, wall = 0.0, 0.0, [], 0.0
-    for name, k, k_all, run, run1 in runs:
+    halves = [h for h in ((wl.n_full, 0), (0, n_inc)) if h[0] or h[1]]
+    per_half = min_s / max(len(halves), 1)
+    total_s, total_s1, parts, wall, K, scaled = 0.0, 0.0, [], 0.0, 0, False
+    for kf, ki in halves:
+        k_all = kf or ki
+        if not k_all:
+            continue
+        K += k_all
+        k0 = min(k_all, 2 * nt)
+        probe = oracle_sample(wl, k0 if kf else 0, k0 if ki else 0, nt, arbitrated, structured)[0]
+        t0 = time.perf_counter()
+        probe[3]()
+        spc0 = (time.perf_counter() - t0) / k0
+        k = int(min(k_all, max(k0, per_half / max(spc0, 1e-9))))
+        name, k, _, run, run1 = oracle_sample(wl, k if kf else 0, k if ki else 0, nt, arbitrated, structured)[0]
+        scaled = scaled or k < k_all
         reps, t0 = 0, time.perf_counter()
         while True:
             run()
             reps += 1
             dt = time.perf_counter() - t0
-            if dt >= min_s / len(runs):
+            if dt >= per_half:
                 break
         wall += dt
         spc = dt / (reps * k)
@@ -363,8 +376,6 @@ def cpu_baseline(wl, min_s=10.0, arbitrated=False, structured=False, ev_budget=1
         total_s1 += k_all * spc1
         parts.append("%s: %d of %d candidates x %d pass%s, %.4g s/candidate (1 core: first %d, %.4g s)" % (
             name, k, k_all, reps, "" if reps == 1 else "es", spc, k1, spc1))
-    K = sum(r[2] for r in runs)
-    scaled = any(r[1] < r[2] for r in runs)
     return {"value": K / total_s, "unit": UNIT, "cores": nt, "kind": "oracle",
             "sample": "; ".join(parts) + ("; scaled to all %d candidates" % K if scaled else ""),
             "scaled": scaled, "seconds": round(wall, 3),

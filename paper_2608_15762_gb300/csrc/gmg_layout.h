@@ -197,6 +197,8 @@ struct SimParams {
   int64_t slot_bytes;    // scratch bytes per warp slot
   int32_t dev_bytes;     // shared bytes of accelerator state per warp
   int32_t stage_bytes;   // shared bytes of the staged GMG copy (sim_full_staged_kernel), else 0
+  int32_t no_side;       // 1: no side bytes in shared memory (the accelerator is inside the log entry)
+  int32_t pad_;
   // byte offsets inside a slot (off_pk < 0: the peaks are in shared memory)
   int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row, off_pk;
 };

@@ -495,7 +495,9 @@ int log_cap(const gmg* g, const sim_opts_t* o) {
 }
 
 size_t smem_per_warp(const SimParams& P) {
-  return align_up((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 + (size_t)P.opcap * 4, 16) +
+  const size_t side = P.no_side ? 0 : 1;
+  return align_up((size_t)P.qs * 8 + (size_t)P.ms * (8 + side) + (size_t)P.sortcap * (8 + side) + (size_t)P.opcap * 4,
+                  16) +
          (size_t)P.dev_bytes;
 }
 
@@ -530,6 +532,7 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
   P.drain_trigger = batch ? kBatchOpsPerGeneration : kOpsPerGeneration;
   P.opcap = batch ? kBatchOpsPerGeneration + 32 : kOpsPerGeneration;
   P.dev_bytes = dev_smem_bytes(G.D, G.t32 ? 4 : 8);
+  P.no_side = batch ? 1 : 0;  // the batched sweep keeps the accelerator inside the entry
   L.smem = (size_t)L.wpb * smem_per_warp(P);
   size_t o2 = 0;
   auto take = [&](size_t bytes) {
@@ -560,6 +563,7 @@ int plan_launch(const gmg* g, int32_t K, const sim_opts_t* o, bool inc, Launch& 
     big.qs = std::max(kSharedQueueEntries, kSharedQueueEntriesBatch);
     big.ms = std::max(kSharedLogEntries, kSharedLogEntriesBatch);
     big.dev_bytes = 24 * 256;
+    big.no_side = 0;
     if (set_smem_limits(4 * (int)smem_per_warp(big)) != cudaSuccess) return GMG_ECUDA;
     g_smem_set = true;
   }

@@ -170,7 +170,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, co
     bool keep = false;
     if (v) {
       e = B.ck_mkey[(int64_t)c * B.ckm + idx];
-      dv8 = B.ck_mdev[(int64_t)c * B.ckm + idx];
+      if (!kKey) dv8 = B.ck_mdev[(int64_t)c * B.ckm + idx];
       keep = true;
       const uint32_t cls = S.kc.cls(e), op = S.kc.op(e);
       const int dev = kKey ? (int)(e >> S.ds) : (int)dv8;
@@ -186,7 +186,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, co
     if (keep) {
       const int pos = outn + __popc(bal & lanes_below());
       *S.log.kp(pos) = e;
-      *S.log.dp(pos) = dv8;
+      if (!kKey) *S.log.dp(pos) = dv8;
     }
     outn += __popc(bal);
   }

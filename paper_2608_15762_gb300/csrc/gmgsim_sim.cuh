@@ -179,11 +179,60 @@ struct ReadyHeap {
     __syncwarp();
   }
 
+  // The same as sift_down while every slot in use is in shared memory.
+  __device__ void sift_down_shared(int pos, uint64_t x) {
+    const unsigned lane = lane_id();
+    while (true) {
+      const int c0 = pos * 32 + 1;
+      if (c0 >= size) break;
+      const int idx = c0 + (int)lane;
+      const uint64_t ck = idx < size ? sk[idx] : kKeyMax;
+      const uint64_t m = warp_min_u64(ck);
+      if (m >= x) break;
+      const int src = __ffs(__ballot_sync(kFullMask, ck == m)) - 1;
+      if (lane == 0) sk[pos] = m;
+      pos = c0 + src;
+    }
+    if (lane == 0) sk[pos] = x;
+    __syncwarp();
+  }
+
   __device__ void pop() {
     const int n = --size;
     if (n == 0) return;
     const uint64_t x = *kp(n);
     sift_down(0, x);
+  }
+
+  // pop / push with a branch for a heap held entirely in shared memory (the
+  // batched sweep's larger shared part makes that the common case)
+  __device__ void pop_fast() {
+    const int n = --size;
+    if (n == 0) return;
+    if (n < qs) {
+      sift_down_shared(0, sk[n]);
+      return;
+    }
+    const uint64_t x = *kp(n);
+    sift_down(0, x);
+  }
+
+  __device__ bool push_fast(uint64_t key) {
+    if (size >= cap) return false;
+    if (size < qs) {
+      int pos = size++;
+      while (pos > 0) {
+        const int par = (pos - 1) >> 5;
+        const uint64_t pk = sk[par];
+        if (pk <= key) break;
+        if (lane_id() == 0) sk[pos] = pk;
+        pos = par;
+      }
+      if (lane_id() == 0) sk[pos] = key;
+      __syncwarp();
+      return true;
+    }
+    return push(key);
   }
 
   __device__ bool push(uint64_t key) {
@@ -246,8 +295,13 @@ struct Devices {
   __device__ void setup(const DevGmg& g, uint8_t* sm, int64_t* pk_global) {
     D = g.D;
     lv = reinterpret_cast<int64_t*>(sm);
-    pk = pk_global ? pk_global : lv + D;
-    fr = reinterpret_cast<TM*>(pk_global ? lv + D : lv + 2 * D);
+    if (kReg) {  // peaks in shared memory (a compile-time fact for these instances)
+      pk = lv + D;
+      fr = nullptr;
+    } else {
+      pk = pk_global;
+      fr = reinterpret_cast<TM*>(lv + D);
+    }
   }
   __device__ void reset(const DevGmg& g) {
     const unsigned l = lane_id();
@@ -338,7 +392,10 @@ struct WarpSmem {
 __device__ __forceinline__ size_t align16(size_t x) { return (x + 15) & ~(size_t)15; }
 
 __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P, unsigned wib) {
-  const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * 9 + (size_t)P.sortcap * 9 +
+  // the side bytes (accelerator of a log entry) are left out where the
+  // accelerator is inside the entry and shared memory is tight (P.no_side)
+  const size_t side = P.no_side ? 0 : 1;
+  const size_t head = align16((size_t)P.qs * 8 + (size_t)P.ms * (8 + side) + (size_t)P.sortcap * (8 + side) +
                               (size_t)P.opcap * 4);
   const size_t per = head + (size_t)P.dev_bytes;
   uint8_t* b = smem + per * wib;
@@ -347,8 +404,8 @@ __device__ __forceinline__ WarpSmem carve_smem(uint8_t* smem, const SimParams& P
   w.logk = w.heap + P.qs;
   w.sortk = w.logk + P.ms;
   w.logd = reinterpret_cast<uint8_t*>(w.sortk + P.sortcap);
-  w.sortd = w.logd + P.ms;
-  w.oplog = reinterpret_cast<uint32_t*>(w.sortd + P.sortcap);
+  w.sortd = w.logd + P.ms * side;
+  w.oplog = reinterpret_cast<uint32_t*>(w.sortd + P.sortcap * side);
   w.dev = b + head;
   return w;
 }
@@ -485,7 +542,7 @@ struct Sim {
     const uint32_t freel = __ballot_sync(kFullMask, rk_reg == kKeyMax);
     if (freel) {
       if ((int)lane_id() == __ffs(freel) - 1) rk_reg = key;
-    } else if (!q.push(key)) {
+    } else if (!(kBatch ? q.push_fast(key) : q.push(key))) {
       status = GMG_SIM_QUEUE;
     }
   }
@@ -1137,7 +1194,7 @@ struct Sim {
       load_root();
     } else {
       __syncwarp();
-      q.pop();
+      q.pop_fast();
     }
   }
   // An op whose inputs several ops of one batch complete is queued once: the
@@ -1160,13 +1217,18 @@ struct Sim {
       int64_t lim = 0;
       while (true) {
         const int64_t t = rq.time(nk);
+        const bool from_reg = nk == rm;
         take(nk, rm);
         if ((int)lane == m) mine = nk;
         const int64_t e = t + ((int64_t)1 << rq.q(nk));
         lim = (m == 0 || e < lim) ? e : lim;
         if (kMode == kBase) last_t = (tm_t)t;
         if (++m == 32) break;
-        nk = peek(rm);
+        // the register tier's minimum only changes when its key was taken
+        if (from_reg) rm = warp_min_u64(rk_reg);
+        const uint64_t top = q.top();
+        nk = rkey < top ? rkey : top;
+        nk = rm < nk ? rm : nk;
         if (nk == kKeyMax || rq.time(nk) >= lim) break;
       }
       iters += m;
@@ -1408,7 +1470,7 @@ __device__ void Sim<kReg, kMode, kKey, kT32, kTypes, kBatch, kStage>::maybe_chec
     for (int x = lane; x < q.size; x += 32) B.ck_qkey[(int64_t)ck * B.ckq + x] = *q.kp(x);
     for (int x = lane; x < log.n; x += 32) {
       B.ck_mkey[(int64_t)ck * B.ckm + x] = *log.kp(x);
-      B.ck_mdev[(int64_t)ck * B.ckm + x] = *log.dp(x);
+      if (!kKey) B.ck_mdev[(int64_t)ck * B.ckm + x] = *log.dp(x);
     }
   } else if (lane == 0) {
     B.ck_time[ck] = kI64Max;
