@@ -179,6 +179,7 @@ class Prepared:
 
 
 ARB_SOURCES = ("gmgsim_arb.cu", "gmg_arb.h", "gmg_arb_events.h")
+ARBW_SOURCES = ("gmgsim_arbw.cu", "gmg_arbw.h", "gmg_arb_events.h")
 
 
 def rows_of(wl, ks, structured=False):
@@ -865,7 +866,8 @@ def main():
     kernels = {}
     for n in names:
         ppath = profile_path(kname[n], wname)
-        prof = read_profile(ppath, ARB_SOURCES if (p.arb and n != "base") else ())
+        extra = () if not p.arb or n == "base" else (ARB_SOURCES if D <= 32 else ARBW_SOURCES)
+        prof = read_profile(ppath, extra)
         kd = {"kernel": kname[n], "launch_ms": kern_ms[n], "units": kcount[n],
               "hbm_gbs": alg_bytes[n] / (kern_ms[n] / 1000) / 1e9, "inst_per_launch": None, "issue_frac": None,
               "dram_bytes_per_launch": None}
