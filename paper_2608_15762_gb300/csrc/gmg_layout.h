@@ -117,6 +117,13 @@ inline int64_t stage_smem_bytes(int64_t n, int64_t E) {
   return 16 + 16 * n + (4 * n + 15) / 16 * 16 + 2 * ((4 * E + 15) / 16 * 16);
 }
 
+// Resident 4-warp blocks per SM the batched kernels are compiled for (their
+// register budget; compile-time overridable for tuning sweeps).
+#ifndef GMG_BATCH_BLOCKS_PER_SM
+#define GMG_BATCH_BLOCKS_PER_SM 7
+#endif
+constexpr int kBatchBlocksPerSM = GMG_BATCH_BLOCKS_PER_SM;
+
 // The staged-GMG kernel's largest CTA (one per SM; 72 registers a thread).
 constexpr int kStageMaxWarps = 28;
 

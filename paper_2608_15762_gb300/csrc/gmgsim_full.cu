@@ -8,7 +8,7 @@ namespace {
 // sim_batch: K full placements.
 // ---------------------------------------------------------------------------
 template <bool kReg, bool kKey, bool kT32, bool kTypes, bool kBatch>
-__global__ void __launch_bounds__(128, 7) sim_full_kernel(const __grid_constant__ SimParams P) {
+__global__ void __launch_bounds__(128, kBatch ? kBatchBlocksPerSM : 7) sim_full_kernel(const __grid_constant__ SimParams P) {
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;

@@ -40,13 +40,13 @@ constexpr int kDefaultWarpsPerBlock = 4;
 constexpr int kSharedQueueEntries = 97;  // 1 + 32 * 3: root, its children, two more groups
 // The batched sweep's sizes (compile-time overridable for tuning sweeps).
 #ifndef GMG_BATCH_QUEUE_SHARED
-#define GMG_BATCH_QUEUE_SHARED 225  // 1 + 32 * 7: the wider frontier of many tenants
+#define GMG_BATCH_QUEUE_SHARED 161  // 1 + 32 * 5 (with the log below: 28 warps per SM at 256 accelerators)
 #endif
 #ifndef GMG_BATCH_OPS_PER_GENERATION
 #define GMG_BATCH_OPS_PER_GENERATION 24
 #endif
 #ifndef GMG_BATCH_LOG_SHARED
-#define GMG_BATCH_LOG_SHARED 192
+#define GMG_BATCH_LOG_SHARED 128
 #endif
 constexpr int kSharedQueueEntriesBatch = GMG_BATCH_QUEUE_SHARED;
 constexpr int kBatchOpsPerGeneration = GMG_BATCH_OPS_PER_GENERATION;
