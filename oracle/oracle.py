@@ -60,7 +60,7 @@ def lib():
         L.orc_simulate.restype = C.c_int
         L.orc_simulate_batch.argtypes = [vp, vp, i64, i32, i32, vp, vp, vp]
         L.orc_simulate_batch.restype = C.c_int
-        L.orc_incremental_batch.argtypes = [vp, vp, vp, vp, vp, i32, i32, vp, vp, vp]
+        L.orc_incremental_batch.argtypes = [vp, vp, vp, vp, vp, i32, i32, vp, vp, vp, i32]
         L.orc_incremental_batch.restype = C.c_int
         L.orc_select_best.argtypes = [vp, i32, i32, vp]
         L.orc_select_best.restype = i64
@@ -156,7 +156,11 @@ def simulate_batch(desc, place, nthreads: int = 0, arbitrated=False):
     return s, peak, req[:, :d.n_req]
 
 
-def incremental_batch(desc, base_place, moves, nthreads: int = 0, arbitrated=False):
+def incremental_batch(desc, base_place, moves, nthreads: int = 0, arbitrated=False, resumed=False):
+    """Move lists against a base placement.  Results are the simulation of
+    each moved placement; with arbitrated transfers `resumed` selects what
+    `events` counts: False -- every op (the moved placement simulated in
+    full); True -- the ops whose arbitrated base ready time is >= T0."""
     h = _GraphHolder(desc, arbitrated)
     d = h.desc
     base = np.ascontiguousarray(base_place, dtype=np.uint8)
@@ -171,7 +175,8 @@ def incremental_batch(desc, base_place, moves, nthreads: int = 0, arbitrated=Fal
     rc = lib().orc_incremental_batch(C.addressof(h.g), base.ctypes.data, off.ctypes.data,
                                      op.ctypes.data if op.size else None,
                                      dv.ctypes.data if dv.size else None, K, nt, s.ctypes.data,
-                                     peak.ctypes.data, req.ctypes.data if d.n_req else None)
+                                     peak.ctypes.data, req.ctypes.data if d.n_req else None,
+                                     1 if resumed else 0)
     if rc:
         raise ValueError("oracle rejected the input: %d" % rc)
     return s, peak, req[:, :d.n_req]

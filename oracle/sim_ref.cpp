@@ -695,10 +695,17 @@ int orc_simulate_batch(const orc_graph* in, const uint8_t* place, int64_t ld, in
   return 0;
 }
 
-// K candidates given as move lists against a base placement.
+// K candidates given as move lists against a base placement.  With
+// arbitrated transfers, `resumed` says what `events` counts: 0 -- the
+// candidate's moved placement simulated in full (events = n); 1 -- resumed at
+// T0 from the arbitrated base (events = ops whose arbitrated base ready time
+// is >= T0, as with pure-latency transfers; every intent, transfer and buffer
+// of a moved op's predecessors happens at or after their finish, so nothing
+// before T0 changes).
 int orc_incremental_batch(const orc_graph* in, const uint8_t* base_place, const int32_t* move_off,
                           const int32_t* move_op, const uint8_t* move_dev, int32_t K,
-                          int32_t nthreads, orc_summary* out, int64_t* peak, int64_t* req_done) {
+                          int32_t nthreads, orc_summary* out, int64_t* peak, int64_t* req_done,
+                          int32_t resumed) {
   Graph g;
   int rc = build(in, g);
   if (rc) return rc;
@@ -742,7 +749,7 @@ int orc_incremental_batch(const orc_graph* in, const uint8_t* base_place, const 
     }
     simulate(g, place.data(), res);
     int64_t ev = 0;
-    if (g.mode == 1) {
+    if (g.mode == 1 && !resumed) {
       ev = g.n;  // arbitrated transfers: the moved placement is simulated in full
     } else if (t0 != kI64Max) {
       for (int i = 0; i < g.n; ++i) ev += base.ready[i] >= t0 ? 1 : 0;

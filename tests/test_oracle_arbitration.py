@@ -282,3 +282,74 @@ def test_incremental_is_the_full_arbitrated_simulation_of_the_moved_placement():
         r = _arb(d, pl)
         assert (r["score"], r["makespan"], r["viol_flag"]) == (s["score"][k], s["makespan"][k], s["viol_flag"][k])
         assert r["peak"].tolist() == pk[k].tolist() and s["events"][k] == d.n_ops
+
+
+# ---------------------------------------------------------------------------
+# Resuming arbitrated incremental candidates at T0
+# ---------------------------------------------------------------------------
+
+def _inc_helpers():
+    import test_oracle_incremental as TI
+    return TI._t0, TI._applied
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_arbitrated_prefix_before_t0_is_unchanged(seed):
+    """What resuming an arbitrated candidate at T0 relies on: with T0 taken
+    from the arbitrated base's finish times, every op whose arbitrated base
+    ready time is < T0 keeps its ready, start and finish times in the moved
+    placement's arbitrated schedule, every other op is ready at or after T0,
+    and so is every transfer that touches a moved op's predecessors."""
+    from paper_2608_15762_gb300.workloads import random_desc, random_moves
+    t0f, applied = _inc_helpers()
+    g = np.random.default_rng(900 + seed)
+    n = int(g.integers(5, 150))
+    D = int(g.integers(2, 7))
+    d = random_desc(7000 + seed, n, D, explicit_cons=bool(seed % 2), dur_hi=300)
+    if seed % 3 == 2:
+        d.link_id = np.asarray([(min(s, e) * D + max(s, e)) for s in range(D) for e in range(D)], np.int32)
+    base = g.integers(0, D, n).astype(np.uint8)
+    mv = random_moves(300 + seed, 30, base, D, max_moves=5, allow_noop=False)
+    rb = O.simulate(d, base, arbitrated=True)
+    checked = 0
+    for k in range(30):
+        t0 = t0f(d, base, mv, k, rb["finish"].tolist())
+        if t0 is None:
+            continue
+        rc = O.simulate(d, applied(base, mv, k), arbitrated=True)
+        early = rb["ready"] < t0
+        assert np.array_equal(rc["ready"][early], rb["ready"][early])
+        assert np.array_equal(rc["start"][early], rb["start"][early])
+        assert np.array_equal(rc["finish"][early], rb["finish"][early])
+        assert (rc["ready"][~early] >= t0).all()
+        checked += 1
+    assert checked > 0
+
+
+@pytest.mark.parametrize("seed", range(6))
+def test_resumed_event_count(seed):
+    """resumed=True changes only `events`: the ops whose arbitrated base ready
+    time is >= T0 (0 without an effective move); every other field is the
+    moved placement's full arbitrated simulation."""
+    from paper_2608_15762_gb300.workloads import random_desc, random_moves
+    t0f, _ = _inc_helpers()
+    g = np.random.default_rng(60 + seed)
+    n = int(g.integers(20, 120))
+    D = int(g.integers(2, 6))
+    d = random_desc(7100 + seed, n, D, dur_hi=200)
+    base = g.integers(0, D, n).astype(np.uint8)
+    mv = random_moves(400 + seed, 24, base, D, max_moves=4)
+    full, pf, rf = O.incremental_batch(d, base, mv, arbitrated=True)
+    res, pr, rr = O.incremental_batch(d, base, mv, arbitrated=True, resumed=True)
+    rb = O.simulate(d, base, arbitrated=True)
+    for f in full.dtype.names:
+        if f not in ("events", "reserved"):
+            assert np.array_equal(full[f], res[f]), f
+    assert np.array_equal(pf, pr) and np.array_equal(rf, rr)
+    assert (full["events"][full["status"] == 0] == n).all()
+    for k in range(24):
+        if res["status"][k]:
+            continue
+        t0 = t0f(d, base, mv, k, rb["finish"].tolist())
+        want = 0 if t0 is None else int((rb["ready"] >= t0).sum())
+        assert res["events"][k] == want
