@@ -10,6 +10,21 @@
 
 namespace gsim {
 
+// An arbitrated base snapshot keeps, beside the simulation state of every
+// checkpoint (DevBase), the arbiter's state at that instant in one arena per
+// checkpoint: the per-op input counters, latest arrivals, holds, remote sets,
+// FIFO links and hold times, the arrived intents, the pair queues, every
+// lane's sending transfer and FIFO head, and the endpoint and link sets.
+struct ArbCk {
+  uint8_t* arena;         // [nck][bytes]
+  int64_t bytes;          // per checkpoint
+  int64_t off_cnt, off_rmax, off_refs, off_rmask, off_nextop, off_hold;  // per op (times as int64)
+  int64_t off_xent, off_xnext;  // [xcap]
+  int64_t off_qhead, off_qtail; // [D*D]
+  int64_t off_lanes;      // [32][7] int64: pm, xd, xdp, xde, fh, ft, fa
+  int64_t off_warp;       // int64 nx, xev, sendm, recvm; then uint32 lbits[32]
+};
+
 struct ArbParams {
   SimParams P;            // the full simulation's parameters (slot offsets inside P too)
   const uint16_t* link;   // [D*D] link id of each ordered accelerator pair (< D*D)
@@ -29,6 +44,7 @@ struct ArbParams {
   int64_t off_qhead;      // int32 [D*D]  first pending intent of each pair (-1: none), when not shared
   int64_t off_qtail;      // int32 [D*D]
   const int32_t* pre_status;  // [K] optional: a nonzero entry is the candidate's status, not simulated
+  ArbCk ck;               // arbitrated base snapshot (base and resumed incremental launches)
 };
 
 // Incremental candidates under arbitrated transfers: row k = the base row with
@@ -42,5 +58,13 @@ cudaError_t launch_expand_moves(const uint8_t* base_row, const int32_t* base_sta
 const void* arb_kernel_ptr(bool t32, bool types);
 cudaError_t launch_arb(bool t32, bool types, const ArbParams& A, int grid, int block, size_t smem,
                        cudaStream_t st);
+
+// The arbitrated base snapshot (one warp) and the incremental candidates
+// resumed from it (at most 32 accelerators).
+const void* arb_base_kernel_ptr(bool types);
+const void* arb_inc_kernel_ptr(bool t32, bool types);
+cudaError_t launch_arb_base(bool types, const ArbParams& A, size_t smem, cudaStream_t st);
+cudaError_t launch_arb_inc(bool t32, bool types, const ArbParams& A, int grid, int block, size_t smem,
+                           cudaStream_t st);
 
 }  // namespace gsim

@@ -54,9 +54,11 @@
 namespace gsim {
 namespace {
 
-template <bool kT32, bool kTypes>
-struct ArbSim : ArbEvents<ArbSim<kT32, kTypes>, Sim<true, kFull, true, kT32, kTypes>> {
-  using Base = ArbEvents<ArbSim<kT32, kTypes>, Sim<true, kFull, true, kT32, kTypes>>;
+// kMode: kFull (sim_batch), kBase (the arbitrated base snapshot: records
+// ready and finish times and checkpoints), kInc (candidates resumed from it).
+template <bool kT32, bool kTypes, int kMode = kFull>
+struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT32, kTypes>> {
+  using Base = ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT32, kTypes>>;
   using tm_t = typename Base::tm_t;
   using U = typename std::make_unsigned<tm_t>::type;
   using Base::g;
@@ -166,10 +168,16 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes>, Sim<true, kFull, true, kT32, kTy
       this->fbuf[i] = f;
       if (cs.w & kReqSink)
         atomicMax(reinterpret_cast<unsigned long long*>(this->creq + (int32_t)cs.z), (unsigned long long)f);
+      if (kMode == kBase) P.base.rb[i] = r;
       this->oplog[this->opn] = i;
     }
     ++this->opn;
     if (cs.w & kScored) this->score += (int64_t)f;
+    if (kMode == kBase) {
+      this->makespan = f > this->makespan ? f : this->makespan;
+      ++this->readypops;
+    }
+    if (kMode == kInc && r >= this->T0) ++this->nev;
     __syncwarp();
     uint32_t remote = 0u;
     for (uint32_t c0 = 0; c0 < xs.nsucc; c0 += 32) {
@@ -242,7 +250,7 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes>, Sim<true, kFull, true, kT32, kTy
         fa = kNever;
       } else {
         fh = nextop()[fh];
-        fa = this->fbuf[fh];
+        fa = this->fin((uint32_t)fh);
       }
     }
     __syncwarp();
@@ -375,12 +383,14 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes>, Sim<true, kFull, true, kT32, kTy
         }
         if (td == tx) transfer_done(__ffs(__ballot_sync(kFullMask, xd == td)) - 1, td);
         else intents_arrive((uint32_t)(ik & this->kc.mask));
+        if (kMode == kBase) this->last_t = tx;
         arb_due = true;
         t_arb = tx;
         if (status) break;
         continue;
       }
       if (nk == kKeyMax) break;
+      if (kMode == kBase) arb_checkpoint(nk);
       if (this->opn >= P.opcap) drain(this->kc.time(nk));
       if (nk == rm) {
         if (this->rk_reg == rm) this->rk_reg = kKeyMax;
@@ -395,10 +405,406 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes>, Sim<true, kFull, true, kT32, kTy
         status = GMG_SIM_LOOP;
         break;
       }
+      if (kMode == kBase) this->last_t = (tm_t)this->kc.time(nk);
       start_op(this->kc.op(nk), (tm_t)this->kc.time(nk));
       if (status) break;
     }
     if (!status) drain(kI64Max);
+  }
+
+  // -------------------------------------------------------------------------
+  // Arbitrated base snapshot.  A checkpoint is taken right before a READY key
+  // whose time T_c is past every event handled so far: every transfer event
+  // and arbitration before T_c is done (transfer events at a time come before
+  // READY keys at that time, and the arbiter runs before the next later
+  // event), nothing at T_c or later is.  The simulation part is the base
+  // snapshot's (Sim::maybe_checkpoint, after this simulator's own event
+  // generation); the arbiter's part goes to the checkpoint's arena.
+  // -------------------------------------------------------------------------
+  __device__ void arb_checkpoint(uint64_t next_key) {
+    const DevBase& B = P.base;
+    if (this->ck >= B.nck || this->readypops < this->next_ck) return;
+    if (this->kc.time(next_key) <= (int64_t)this->last_t) return;
+    generate();  // the simulation checkpoint then finds no started op left to generate
+    const int c = this->ck;
+    this->maybe_checkpoint(next_key);
+    if (this->ck > c && B.ck_time[c] != kI64Max) save_arb(c);
+  }
+
+  __device__ uint8_t* arena(int c) const { return A.ck.arena + (int64_t)c * A.ck.bytes; }
+
+  __device__ void save_arb(int c) {
+    const unsigned lane = lane_id();
+    uint8_t* a = arena(c);
+    const ArbCk& K = A.ck;
+    for (int x = lane; x < g.n; x += 32) {
+      reinterpret_cast<int32_t*>(a + K.off_cnt)[x] = cnt()[x];
+      reinterpret_cast<int64_t*>(a + K.off_rmax)[x] = (int64_t)rmax()[x];
+      reinterpret_cast<int32_t*>(a + K.off_refs)[x] = refs()[x];
+      reinterpret_cast<uint32_t*>(a + K.off_rmask)[x] = rmask()[x];
+      reinterpret_cast<int32_t*>(a + K.off_nextop)[x] = nextop()[x];
+      reinterpret_cast<int64_t*>(a + K.off_hold)[x] = (int64_t)this->holdb[x];
+    }
+    for (int x = lane; x < nx; x += 32) {
+      reinterpret_cast<uint32_t*>(a + K.off_xent)[x] = xent()[x];
+      reinterpret_cast<int32_t*>(a + K.off_xnext)[x] = xnext()[x];
+    }
+    for (int x = lane; x < g.D * g.D; x += 32) {
+      reinterpret_cast<int32_t*>(a + K.off_qhead)[x] = qhead()[x];
+      reinterpret_cast<int32_t*>(a + K.off_qtail)[x] = qtail()[x];
+    }
+    int64_t* ls = reinterpret_cast<int64_t*>(a + K.off_lanes) + 7 * lane;
+    ls[0] = pm;
+    ls[1] = (int64_t)xd;
+    ls[2] = xdp;
+    ls[3] = xde;
+    ls[4] = fh;
+    ls[5] = ft;
+    ls[6] = (int64_t)fa;
+    int64_t* w = reinterpret_cast<int64_t*>(a + K.off_warp);
+    if (lane == 0) {
+      w[0] = nx;
+      w[1] = xev;
+      w[2] = sendm;
+      w[3] = recvm;
+    }
+    reinterpret_cast<uint32_t*>(w + 4)[lane] = lbits()[lane];
+    __syncwarp();
+  }
+
+  // A base time (int64) in this kernel's time type; the base's "never" maps
+  // to this kernel's.
+  static __device__ __forceinline__ tm_t narrow_time(int64_t v) {
+    return v >= (int64_t)kNever ? kNever : (tm_t)v;
+  }
+
+  __device__ void restore_arb(int c) {
+    const unsigned lane = lane_id();
+    const uint8_t* a = arena(c);
+    const ArbCk& K = A.ck;
+    for (int x = lane; x < g.n; x += 32) {
+      cnt()[x] = reinterpret_cast<const int32_t*>(a + K.off_cnt)[x];
+      rmax()[x] = narrow_time(reinterpret_cast<const int64_t*>(a + K.off_rmax)[x]);
+      refs()[x] = reinterpret_cast<const int32_t*>(a + K.off_refs)[x];
+      rmask()[x] = reinterpret_cast<const uint32_t*>(a + K.off_rmask)[x];
+      nextop()[x] = reinterpret_cast<const int32_t*>(a + K.off_nextop)[x];
+      this->holdb[x] = narrow_time(reinterpret_cast<const int64_t*>(a + K.off_hold)[x]);
+    }
+    const int64_t* w = reinterpret_cast<const int64_t*>(a + K.off_warp);
+    nx = (int32_t)w[0];
+    xev = (int32_t)w[1];
+    sendm = (uint32_t)w[2];
+    recvm = (uint32_t)w[3];
+    lbits()[lane] = reinterpret_cast<const uint32_t*>(w + 4)[lane];
+    for (int x = lane; x < nx; x += 32) {
+      xent()[x] = reinterpret_cast<const uint32_t*>(a + K.off_xent)[x];
+      xnext()[x] = reinterpret_cast<const int32_t*>(a + K.off_xnext)[x];
+    }
+    for (int x = lane; x < g.D * g.D; x += 32) {
+      qhead()[x] = reinterpret_cast<const int32_t*>(a + K.off_qhead)[x];
+      qtail()[x] = reinterpret_cast<const int32_t*>(a + K.off_qtail)[x];
+    }
+    const int64_t* ls = reinterpret_cast<const int64_t*>(a + K.off_lanes) + 7 * lane;
+    pm = (uint32_t)ls[0];
+    xd = narrow_time(ls[1]);
+    xdp = (uint32_t)ls[2];
+    xde = (int)ls[3];
+    fh = (int32_t)ls[4];
+    ft = (int32_t)ls[5];
+    fa = narrow_time(ls[6]);
+    arb_due = false;
+    t_arb = 0;
+    __syncwarp();
+  }
+
+  // Remote accelerators of p's successors under placement rw (uniform).
+  __device__ uint32_t remote_set(uint32_t p, const uint8_t* rw) const {
+    const XqSucc xs = op_xqsucc(g.ops, p);
+    const int dp = rw[p];
+    uint32_t m = 0u;
+    for (uint32_t u = lane_id(); u < xs.nsucc; u += 32) {
+      const int dj = rw[__ldg(g.succ + xs.succ_off + u)];
+      if (dj != dp) m |= 1u << dj;
+    }
+    return __reduce_or_sync(kFullMask, m);
+  }
+
+  // A listed consumer of p on p's accelerator under placement rw (uniform).
+  __device__ bool local_consumer(uint32_t p, const uint8_t* rw) const {
+    const uint4 cs = op_cons(g.ops, p);
+    const XqSucc xs = op_xqsucc(g.ops, p);
+    const bool all = (cs.w & kAllCons) != 0;
+    const uint32_t* lst = all ? g.succ + xs.succ_off : g.cons + cs.x;
+    const uint32_t nl = all ? xs.nsucc : cs.y;
+    const int dp = rw[p];
+    bool f = false;
+    for (uint32_t u = lane_id(); u < nl; u += 32) f |= rw[__ldg(lst + u)] == dp;
+    return __any_sync(kFullMask, f);
+  }
+
+  // Op p (started before the resume point, finishing at or after it) in the
+  // FIFO of coming intents of its accelerator d, kept in finish order: insert
+  // (want) or remove.  The list runs from the head to the tail through
+  // nextop (the tail's link is not kept).  Uniform call; lane d owns the head
+  // and tail.
+  __device__ void fifo_set(uint32_t p, int d, bool want) {
+    const unsigned lane = lane_id();
+    int32_t h = __shfl_sync(kFullMask, fh, d);
+    int32_t t = __shfl_sync(kFullMask, ft, d);
+    int32_t* nxp = nextop();
+    const tm_t fp = this->fin(p);
+    int32_t prev = -1, cur = h;
+    bool found = false;
+    for (int guard = 0; cur >= 0 && guard <= g.n; ++guard) {
+      if (cur == (int32_t)p) {
+        found = true;
+        break;
+      }
+      if (this->fin((uint32_t)cur) > fp) break;
+      prev = cur;
+      cur = cur == t ? -1 : nxp[cur];
+    }
+    if (want == found) return;
+    if (want) {  // link p between prev and cur
+      if (lane == 0) {
+        nxp[p] = cur;
+        if (prev >= 0) nxp[prev] = (int32_t)p;
+      }
+      if (prev < 0) h = (int32_t)p;
+      if (cur < 0) t = (int32_t)p;
+    } else {  // unlink p (cur == p)
+      const int32_t after = (int32_t)p == t ? -1 : nxp[p];
+      if (lane == 0 && prev >= 0) nxp[prev] = after;
+      if (prev < 0) h = after;
+      if (t == (int32_t)p) t = prev;
+    }
+    __syncwarp();
+    if ((int)lane == d) {
+      fh = h;
+      ft = h < 0 ? -1 : t;
+      fa = h < 0 ? kNever : this->fin((uint32_t)h);
+    }
+    __syncwarp();
+  }
+
+  // One incremental candidate resumed from the arbitrated base snapshot.
+  // Results equal the full arbitrated simulation of the moved placement
+  // (Sec. 3.5.2); the fix-ups below are what the moves change in the state
+  // at the checkpoint T_c <= T0: a moved op's inputs counted so far (only
+  // predecessors local under the new placement and already started count; no
+  // remote one has finished) and its READY key; and for every predecessor p
+  // of a moved op that started before T_c (it finishes at or after T0, so
+  // none of its intents, transfers or receive buffers exist yet): its remote
+  // set, the holds on its copy, its place in its accelerator's FIFO of coming
+  // intents, and whether its copy's release is already logged.
+  __device__ void inc_candidate(int64_t k, uint8_t* crow) {
+    const DevBase& B = P.base;
+    const unsigned lane = lane_id();
+    const int32_t m0 = P.move_off[k], m1 = P.move_off[k + 1];
+    const int32_t nm = m1 - m0;
+    // validate the move list (range, then an op moved twice)
+    bool bad = false, dup = false;
+    for (int32_t m = m0 + (int32_t)lane; m < m1; m += 32)
+      bad |= P.move_op[m] < 0 || P.move_op[m] >= g.n || P.move_dev[m] >= g.D;
+    bad = __any_sync(kFullMask, bad);
+    if (!bad)
+      for (int32_t m = m0 + (int32_t)lane; m < m1; m += 32)
+        for (int32_t m2 = m + 1; m2 < m1 && !dup; ++m2) dup = P.move_op[m2] == P.move_op[m];
+    dup = __any_sync(kFullMask, dup);
+    if (B.status[0] != GMG_SIM_OK) {
+      this->write_invalid(k, GMG_SIM_BADBASE);
+      return;
+    }
+    if (bad || dup) {
+      this->write_invalid(k, bad ? GMG_SIM_MOVE_RANGE : GMG_SIM_MOVE_DUP);
+      return;
+    }
+    for (int c = lane * 16; c < B.ld; c += 512)
+      *reinterpret_cast<uint4*>(crow + c) = *reinterpret_cast<const uint4*>(B.row + c);
+    __syncwarp();
+    uint64_t t0 = kKeyMax;
+    for (int t = lane; t < nm; t += 32) {
+      const int32_t op = P.move_op[m0 + t];
+      const uint8_t dvc = P.move_dev[m0 + t];
+      crow[op] = dvc;
+      if (dvc != B.row[op]) {
+        const RelPred rp = op_relpred(g.ops, (uint32_t)op);
+        uint64_t tx = (uint64_t)rp.rel;
+        if (rp.npred) {
+          tx = kKeyMax;
+          for (uint32_t u = 0; u < rp.npred; ++u) {
+            const uint64_t fp = (uint64_t)B.fb[__ldg(g.pred + rp.pred_off + u) & kIdMask];
+            tx = fp < tx ? fp : tx;
+          }
+        }
+        t0 = tx < t0 ? tx : t0;
+      }
+    }
+    t0 = warp_min_u64(t0);
+    __syncwarp();
+    row = crow;
+    const DevOut& o = P.out;
+    if (t0 == kKeyMax) {  // no effective move: the base results
+      const int64_t* rs = B.res_scalars;
+      if (lane == 0) {
+        o.makespan[k] = rs[0];
+        o.score[k] = rs[1];
+        o.status[k] = GMG_SIM_OK;
+        o.viol_flag[k] = (int32_t)rs[2];
+        o.viol_op[k] = (int32_t)rs[3];
+        o.viol_dev[k] = (int32_t)rs[4];
+        o.viol_time[k] = rs[5];
+        o.sla_miss[k] = (int32_t)rs[6];
+        o.events[k] = 0;
+      }
+      for (int d = lane; d < g.D; d += 32) o.peak[k * g.D + d] = B.res_peak[d];
+      if (o.req_done)
+        for (int r = lane; r < g.R; r += 32) o.req_done[k * g.R + r] = B.res_creq[r];
+      const int ts = this->trace_slot(k);
+      if (ts >= 0)
+        for (int x = lane; x < g.n; x += 32) {
+          o.trace_finish[(int64_t)ts * g.n + x] = B.fb[x];
+          o.trace_start[(int64_t)ts * g.n + x] =
+              B.fb[x] - this->dur_of((uint32_t)x, B.row[x], op_durbytes(g.ops, (uint32_t)x).x);
+        }
+      return;
+    }
+    this->T0 = (tm_t)t0;
+    int best = -1;
+    for (int c = lane; c < B.nck; c += 32)
+      if (B.ck_time[c] <= (int64_t)t0) best = c;
+    const int c = __reduce_max_sync(kFullMask, best);
+    const int64_t* sc = B.ck_scalars + (int64_t)c * 8;
+    const int qsz = (int)sc[0];
+    const int msz = (int)sc[7];
+    if (qsz + nm > this->q.cap || msz + nm > this->log.cap) {
+      this->write_invalid(k, GMG_SIM_QUEUE);
+      return;
+    }
+    // the simulation state of checkpoint c
+    this->Tc = (tm_t)B.ck_time[c];
+    this->rootptr = (int)sc[1];
+    this->load_root();
+    this->score = sc[2];
+    this->makespan = (tm_t)sc[3];
+    this->vflag = (int32_t)sc[4];
+    this->vt = sc[5];
+    this->vop = (int32_t)(sc[6] >> 32);
+    this->vdev = (int32_t)(sc[6] & 0xffffffff);
+    this->iters = 0;
+    this->nev = 0;
+    this->readypops = 0;
+    this->last_t = -1;
+    status = GMG_SIM_OK;
+    this->rk_reg = kKeyMax;
+    this->opn = 0;
+    this->dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
+    for (int r = lane; r < g.R; r += 32) this->creq[r] = B.ck_creq[(int64_t)c * g.R + r];
+    this->zero_fin();
+    restore_arb(c);
+    // READY keys, except those of moved ops (recomputed below)
+    int nq = 0;
+    for (int c0 = 0; c0 < qsz; c0 += 32) {
+      const int x = c0 + (int)lane;
+      const bool v = x < qsz;
+      const uint64_t key = v ? B.ck_qkey[(int64_t)c * B.ckq + x] : 0ull;
+      const uint32_t op = this->kc.op(key);
+      const bool keep = v && crow[op] == B.row[op];
+      const uint32_t bal = __ballot_sync(kFullMask, keep);
+      if (keep) *this->q.kp(nq + __popc(bal & lanes_below())) = key;
+      nq += __popc(bal);
+    }
+    // logged HBM events, except the release of a moved op's predecessor's own
+    // copy (regenerated below if it is due)
+    int outn = 0;
+    for (int c0 = 0; c0 < msz; c0 += 32) {
+      const int x = c0 + (int)lane;
+      const bool v = x < msz;
+      const uint64_t e = v ? B.ck_mkey[(int64_t)c * B.ckm + x] : 0ull;
+      bool keep = v;
+      if (v && this->kc.cls(e) == kFree) {
+        const uint32_t op = this->kc.op(e);
+        const int dev = (int)(e >> this->ds);
+        if (dev == B.row[op]) {
+          const XqSucc xs = op_xqsucc(g.ops, op);
+          for (uint32_t u = 0; u < xs.nsucc && keep; ++u) {
+            const uint32_t j = __ldg(g.succ + xs.succ_off + u);
+            keep = crow[j] == B.row[j];
+          }
+        }
+      }
+      const uint32_t bal = __ballot_sync(kFullMask, keep);
+      if (keep) *this->log.kp(outn + __popc(bal & lanes_below())) = e;
+      outn += __popc(bal);
+    }
+    this->log.n = outn;
+    __syncwarp();
+    // every effective move: the moved op's inputs, its predecessors' state
+    for (int32_t t = 0; t < nm; ++t) {
+      const uint32_t x = (uint32_t)P.move_op[m0 + t];
+      if (crow[x] == B.row[x]) continue;
+      const RelPred rp = op_relpred(g.ops, x);
+      // inputs of x present so far: started predecessors local under crow
+      int32_t cx = 0;
+      uint64_t rx = 0;
+      for (uint32_t u = lane; u < rp.npred; u += 32) {
+        const uint32_t p = __ldg(g.pred + rp.pred_off + u) & kIdMask;
+        if (this->base_time(this->rb, p) < this->Tc && crow[p] == crow[x]) {
+          ++cx;
+          const uint64_t fp = (uint64_t)this->base_time(this->fb, p);
+          rx = fp > rx ? fp : rx;
+        }
+      }
+      cx = (int32_t)__reduce_add_sync(kFullMask, (uint32_t)cx);
+      rx = warp_max_u64(rx);
+      if (lane == 0) {
+        cnt()[x] = cx;
+        rmax()[x] = (tm_t)rx;
+      }
+      if (rp.npred > 0 && (uint32_t)cx == rp.npred) {
+        const tm_t rel = (tm_t)rp.rel;
+        const tm_t rj = rel > (tm_t)rx ? rel : (tm_t)rx;
+        if (lane == 0) *this->q.kp(nq) = this->kc.make(rj, kReady, x);
+        ++nq;
+      }
+      // started predecessors: remote set, holds, FIFO, own copy's release;
+      // each predecessor once, by its first moved successor in this list
+      for (uint32_t u = 0; u < rp.npred; ++u) {
+        const uint32_t p = __ldg(g.pred + rp.pred_off + u) & kIdMask;
+        if (this->base_time(this->rb, p) >= this->Tc) continue;
+        bool first = true;
+        for (int32_t t2 = 0; t2 < t && first; ++t2) {
+          const uint32_t x2 = (uint32_t)P.move_op[m0 + t2];
+          if (crow[x2] == B.row[x2]) continue;
+          const RelPred r2 = op_relpred(g.ops, x2);
+          for (uint32_t u2 = 0; u2 < r2.npred; ++u2)
+            if ((__ldg(g.pred + r2.pred_off + u2) & kIdMask) == p) {
+              first = false;
+              break;
+            }
+        }
+        if (!first) continue;
+        const uint32_t rc = remote_set(p, crow);
+        const bool lc = local_consumer(p, crow);
+        const int dp = crow[p];
+        const int32_t holds = 1 + __popc(rc) - (lc ? 0 : 1);
+        const tm_t fp = this->fin(p);
+        if (lane == 0) {
+          rmask()[p] = rc;
+          refs()[p] = holds;
+          this->holdb[p] = fp;
+        }
+        __syncwarp();
+        fifo_set(p, dp, rc != 0u);
+        this->log_event(lane == 0 && holds == 0, this->kc.make(fp, kFree, p), dp);
+      }
+    }
+    this->q.size = nq;
+    this->q.heapify();
+    refresh_done();
+    refresh_intent();
+    run();
+    this->finish(k);
   }
 };
 
@@ -428,6 +834,70 @@ __global__ void __launch_bounds__(128, 7) sim_arb_kernel(const __grid_constant__
     S.run();
     S.finish(k);
   }
+}
+
+// The arbitrated base snapshot: the base placement simulated once (64-bit
+// times) with checkpoints of the simulation and the arbiter.
+template <bool kTypes>
+__global__ void __launch_bounds__(32) sim_arb_base_kernel(const __grid_constant__ ArbParams A) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  ArbSim<false, kTypes, kBase> S(A);
+  setup_slot(S, A.P, 0, 0, smem);
+  S.setup_arb(0, smem + A.smem_std);
+  const DevBase& B = A.P.base;
+  const unsigned lane = lane_id();
+  for (int c = lane * 16; c < B.ld; c += 512)
+    *reinterpret_cast<uint4*>(B.row + c) = *reinterpret_cast<const uint4*>(A.P.place + c);
+  for (int c = lane; c < B.nck; c += 32) B.ck_time[c] = kI64Max;
+  S.fbuf = B.fb;
+  S.row = A.P.place;
+  __syncwarp();
+  if (S.row_has_bad_device(A.P.place)) {
+    if (lane == 0) B.status[0] = GMG_SIM_BADDEV;
+    return;
+  }
+  S.reset_arb();
+  S.ck = 0;
+  S.next_ck = 0;
+  S.arb_checkpoint(S.kc.make(0, kReady, 0));  // checkpoint 0: the initial state
+  S.run();
+  if (lane == 0) B.status[0] = S.status;
+  if (S.status != GMG_SIM_OK) return;
+  int32_t miss = 0;
+  for (int r = lane; r < S.g.R; r += 32) {
+    const int64_t c = S.creq[r];
+    B.res_creq[r] = c;
+    miss += c > __ldg(S.g.deadline + r) ? 1 : 0;
+  }
+  miss = (int32_t)__reduce_add_sync(kFullMask, (unsigned)miss);
+  S.dv.write_peak(B.res_peak);
+  if (lane == 0) {
+    int64_t* rs = B.res_scalars;
+    rs[0] = S.makespan;
+    rs[1] = S.vflag ? kI64Max : S.score;
+    rs[2] = S.vflag;
+    rs[3] = S.vop;
+    rs[4] = S.vdev;
+    rs[5] = S.vt;
+    rs[6] = miss;
+    rs[7] = S.ck;
+  }
+}
+
+// Incremental candidates resumed from the arbitrated base snapshot.
+template <bool kT32, bool kTypes>
+__global__ void __launch_bounds__(128, 7) sim_arb_inc_kernel(const __grid_constant__ ArbParams A) {
+  extern __shared__ __align__(16) uint8_t smem[];
+  const unsigned wib = threadIdx.x >> 5;
+  const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
+  const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
+  ArbSim<kT32, kTypes, kInc> S(A);
+  setup_slot(S, A.P, wib, slot, smem);
+  S.setup_arb(slot, smem + A.smem_std + (size_t)wib * A.smem_arb);
+  S.rb = A.P.base.rb;
+  S.fb = A.P.base.fb;
+  uint8_t* crow = A.P.scratch + slot * A.P.slot_bytes + A.P.off_row;
+  for (int64_t k = slot; k < A.P.K; k += nslots) S.inc_candidate(k, crow);
 }
 
 // One warp per incremental candidate: check the move list (an op or device
@@ -490,6 +960,26 @@ cudaError_t launch_arb(bool t32, bool types, const ArbParams& A, int grid, int b
                        cudaStream_t st) {
   void* args[] = {const_cast<ArbParams*>(&A)};
   return cudaLaunchKernel(arb_kernel_ptr(t32, types), dim3(grid), dim3(block), args, smem, st);
+}
+
+const void* arb_base_kernel_ptr(bool types) {
+  return types ? (const void*)sim_arb_base_kernel<true> : (const void*)sim_arb_base_kernel<false>;
+}
+
+const void* arb_inc_kernel_ptr(bool t32, bool types) {
+  if (t32) return types ? (const void*)sim_arb_inc_kernel<true, true> : (const void*)sim_arb_inc_kernel<true, false>;
+  return types ? (const void*)sim_arb_inc_kernel<false, true> : (const void*)sim_arb_inc_kernel<false, false>;
+}
+
+cudaError_t launch_arb_base(bool types, const ArbParams& A, size_t smem, cudaStream_t st) {
+  void* args[] = {const_cast<ArbParams*>(&A)};
+  return cudaLaunchKernel(arb_base_kernel_ptr(types), dim3(1), dim3(32), args, smem, st);
+}
+
+cudaError_t launch_arb_inc(bool t32, bool types, const ArbParams& A, int grid, int block, size_t smem,
+                           cudaStream_t st) {
+  void* args[] = {const_cast<ArbParams*>(&A)};
+  return cudaLaunchKernel(arb_inc_kernel_ptr(t32, types), dim3(grid), dim3(block), args, smem, st);
 }
 
 }  // namespace gsim

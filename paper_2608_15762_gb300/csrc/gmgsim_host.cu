@@ -58,6 +58,7 @@ constexpr int kSortCap = 128;             // power of two; raised to n_dev's pow
 constexpr int kOpsPerGeneration = 24;     // ~85 HBM events per generation (prefill graphs)
 constexpr int kBatchMinDevices = 33;      // the batched sweep serves graphs on more accelerators
 constexpr int kCheckpoints = 256;
+constexpr int kArbCheckpoints = 64;       // arbitrated bases also keep ~32 bytes per op per checkpoint
 constexpr int kCheckpointQueue = 4096;
 constexpr int kCheckpointLog = 8192;
 
@@ -471,6 +472,8 @@ struct gmg_base {
   const gmg* g;
   uint8_t* slot;
   int qs, qcap;
+  int arb;     // 1: an arbitrated snapshot, which serves arbitrated candidates only
+  ArbCk ck;    // its arbiter arenas
 };
 
 namespace {
@@ -679,13 +682,16 @@ void fill_out(SimParams& P, const sim_out_t* o, const sim_opts_t* opts) {
 // At most 32 accelerators (endpoint sets are bit masks, link ids < 1024),
 // op ids below 2^27 (an intent packs op << 5 | destination) and accelerator
 // ids that fit beside the packed key.
-int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams& A) {
+// mode: kFull (sim_batch), kBase (the arbitrated base snapshot, 64-bit
+// times) or kInc (candidates resumed from it; the slot also holds the
+// candidate's row).
+int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams& A, int mode = kFull) {
   const DevGmg& G = g->dg;
   if (G.D > 32 || !g->linkid) return GMG_EINVAL;
   if (!G.dev_key || G.n >= (1 << 27)) return GMG_ERANGE;
   const int64_t xcap = std::max<int64_t>(g->xfer_bound, 1);
   if (xcap > (int64_t(1) << 29)) return GMG_ERANGE;
-  int rc = plan_launch(g, K, o, false, L, false);
+  int rc = plan_launch(g, K, o, mode == kInc, L, false);
   if (rc) return rc;
   std::memset(&A, 0, sizeof(A));
   SimParams& P = L.P;
@@ -700,7 +706,7 @@ int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams&
   A.heads_shared = G.D <= 16 ? 1 : 0;
   const size_t n = (size_t)G.n, DD = (size_t)G.D * G.D;
   A.off_cnt = take(4 * n);
-  A.off_rmax = take((G.t32 ? 4 : 8) * n);
+  A.off_rmax = take((G.t32 && mode != kBase ? 4 : 8) * n);
   A.off_refs = take(4 * n);
   A.off_rmask = take(4 * n);
   A.off_nextop = take(4 * n);
@@ -715,8 +721,9 @@ int plan_arb(const gmg* g, int32_t K, const sim_opts_t* o, Launch& L, ArbParams&
   const int sms = device_sms();
   if (sms <= 0) return GMG_ECUDA;
   int bps = 0;
-  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, arb_kernel_ptr(G.t32 != 0, G.ntypes >= 2), 32 * L.wpb,
-                                                    L.smem) != cudaSuccess)
+  const void* fn = mode == kInc ? arb_inc_kernel_ptr(G.t32 != 0, G.ntypes >= 2)
+                                : arb_kernel_ptr(G.t32 != 0, G.ntypes >= 2);
+  if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, fn, 32 * L.wpb, L.smem) != cudaSuccess)
     return GMG_ECUDA;
   bps = std::max(bps, 1);
   const int64_t need = (std::max<int64_t>(K, 1) + L.wpb - 1) / L.wpb;
@@ -808,20 +815,27 @@ cudaError_t launch_arb_any(const gmg* g, Launch& L, ArbPlan& Q, const int32_t* p
 
 struct BasePlan {
   size_t off_row, off_rb, off_fb, off_status, off_res, off_peak, off_creq, off_cktime,
-      off_cksc, off_ckdev, off_ckcreq, off_ckqk, off_ckmk, off_ckmd, off_slot, total;
+      off_cksc, off_ckdev, off_ckcreq, off_ckqk, off_ckmk, off_ckmd, off_arena, off_slot, total;
   int nck, ckq, ckm, ld, stride;
+  bool arb;     // an arbitrated base snapshot (also keeps the arbiter's state)
+  ArbParams A;  // its launch parameters (arena offsets inside A.ck)
   Launch L;
 };
 
 int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   const DevGmg& G = g->dg;
   Launch& L = B.L;
-  int rc = plan_launch(g, 1, o, false, L);
+  B.arb = arbitrated(o);
+  int rc = B.arb ? plan_arb(g, 1, o, L, B.A, kBase) : plan_launch(g, 1, o, false, L);
   if (rc) return rc;
   L.wpb = 1;
   L.P.dev_bytes = dev_smem_bytes(G.D, 8);  // the base snapshot keeps 64-bit times
   L.smem = smem_per_warp(L.P);
-  B.nck = kCheckpoints;
+  if (B.arb) {
+    B.A.smem_std = (int64_t)L.smem;
+    L.smem += (size_t)B.A.smem_arb;
+  }
+  B.nck = B.arb ? kArbCheckpoints : kCheckpoints;
   B.ckq = std::min(L.P.qcap, kCheckpointQueue);
   B.ckm = std::min(L.P.mcap, kCheckpointLog);
   B.ld = (int)align_up(std::max(G.n, 1), 16);
@@ -846,6 +860,33 @@ int plan_base(const gmg* g, const sim_opts_t* o, BasePlan& B) {
   B.off_ckqk = take(8 * (size_t)B.ckq * B.nck);
   B.off_ckmk = take(8 * (size_t)B.ckm * B.nck);
   B.off_ckmd = take((size_t)B.ckm * B.nck);
+  B.off_arena = 0;
+  if (B.arb) {
+    // one arena per checkpoint: the arbiter's per-op arrays (times as int64),
+    // intents, pair queues, lane and warp state
+    ArbCk& K = B.A.ck;
+    size_t a = 0;
+    auto at = [&](size_t bytes) {
+      const size_t r = a;
+      a = align_up(a + std::max<size_t>(bytes, 1), 256);
+      return (int64_t)r;
+    };
+    const size_t n = (size_t)G.n, DD = (size_t)G.D * G.D, xc = (size_t)B.A.xcap;
+    K.off_cnt = at(4 * n);
+    K.off_rmax = at(8 * n);
+    K.off_refs = at(4 * n);
+    K.off_rmask = at(4 * n);
+    K.off_nextop = at(4 * n);
+    K.off_hold = at(8 * n);
+    K.off_xent = at(4 * xc);
+    K.off_xnext = at(4 * xc);
+    K.off_qhead = at(4 * DD);
+    K.off_qtail = at(4 * DD);
+    K.off_lanes = at(7 * 8 * 32);
+    K.off_warp = at(4 * 8 + 32 * 4);
+    K.bytes = (int64_t)a;
+    B.off_arena = take((size_t)K.bytes * B.nck);
+  }
   B.off_slot = take((size_t)L.P.slot_bytes);
   B.total = off;
   return GMG_OK;
@@ -1119,7 +1160,7 @@ extern "C" int sim_batch_noalloc(const gmg_t* g, const uint8_t* d_place, int32_t
 }
 
 size_t base_workspace_bytes(const gmg_t* g, const sim_opts_t* opts) {
-  if (!g || arbitrated(opts)) return 0;
+  if (!g) return 0;
   BasePlan B;
   if (plan_base(g, opts, B)) return 0;
   return B.total;
@@ -1133,13 +1174,15 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   if (opts) {
     for (int r : opts->reserved)
       if (r != 0) return GMG_EINVAL;
-    if (opts->transfer_mode != GMG_TRANSFER_LATENCY) return GMG_EINVAL;  // no resume points for the arbiter
+    if (opts->transfer_mode != GMG_TRANSFER_LATENCY && opts->transfer_mode != GMG_TRANSFER_ARBITRATED)
+      return GMG_EINVAL;
+    if (opts->gmg_staging == GMG_STAGING_SHARED) return GMG_EINVAL;
   }
   BasePlan B;
   int rc = plan_base(g, opts, B);
   if (rc) return rc;
   if (!d_base_ws || !aligned(d_base_ws, 256) || ws_bytes < B.total) return GMG_EWS;
-  gmg_base* b = new (std::nothrow) gmg_base;
+  gmg_base* b = new (std::nothrow) gmg_base();
   if (!b) return GMG_ENOMEM;
   uint8_t* w = static_cast<uint8_t*>(d_base_ws);
   DevBase& D = b->db;
@@ -1166,13 +1209,23 @@ int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* o
   b->slot = w + B.off_slot;
   b->qs = B.L.P.qs;
   b->qcap = B.L.P.qcap;
+  b->arb = B.arb ? 1 : 0;
   SimParams P = B.L.P;
   P.base = D;
   P.place = d_base_place;
   P.ld = B.ld;
   P.K = 1;
   P.scratch = b->slot;
-  cudaError_t e = launch_base(B.L.reg, P, B.L.smem, reinterpret_cast<cudaStream_t>(stream));
+  cudaError_t e;
+  if (B.arb) {
+    ArbParams A = B.A;
+    A.P = P;
+    A.ck.arena = w + B.off_arena;
+    b->ck = A.ck;
+    e = launch_arb_base(g->dg.ntypes >= 2, A, B.L.smem, reinterpret_cast<cudaStream_t>(stream));
+  } else {
+    e = launch_base(B.L.reg, P, B.L.smem, reinterpret_cast<cudaStream_t>(stream));
+  }
   if (e != cudaSuccess) {
     delete b;
     return GMG_ECUDA;
@@ -1196,9 +1249,23 @@ static size_t arb_inc_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts, s
   return oz + (size_t)L.slots * (size_t)L.P.slot_bytes;
 }
 
+// Candidates resumed from an arbitrated base snapshot (at most 32 accelerators).
+static int plan_arb_resumed(const gmg_t* g, int32_t K, const sim_opts_t* opts, Launch& L, ArbParams& A) {
+  return plan_arb(g, K, opts, L, A, kInc);
+}
+
 size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
   if (!g || K < 0) return 0;
-  if (arbitrated(opts)) return arb_inc_bytes(g, K, opts, nullptr, nullptr);
+  if (arbitrated(opts)) {
+    // enough for either base: a pure-latency one (moved rows simulated in
+    // full) or an arbitrated one (candidates resumed from it)
+    size_t need = arb_inc_bytes(g, K, opts, nullptr, nullptr);
+    Launch L;
+    ArbParams A;
+    if (g->dg.D <= 32 && plan_arb_resumed(g, K, opts, L, A) == GMG_OK)
+      need = std::max(need, (size_t)L.slots * (size_t)L.P.slot_bytes);
+    return need;
+  }
   Launch L;
   if (plan_launch(g, K, opts, true, L)) return 0;
   return (size_t)L.slots * (size_t)L.P.slot_bytes;
@@ -1213,6 +1280,32 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
   if (staged(opts)) return GMG_EINVAL;  // staging applies to sim_batch
   if (K == 0) return GMG_OK;
   if (!d_move_off) return GMG_EINVAL;
+  if (b->arb && !arbitrated(opts)) return GMG_EINVAL;  // an arbitrated snapshot serves arbitrated candidates
+  if (b->arb) {
+    // resumed from the arbitrated base snapshot
+    Launch L;
+    ArbParams A;
+    rc = plan_arb_resumed(g, K, opts, L, A);
+    if (rc) return rc;
+    if (!d_scratch || !aligned(d_scratch, 256) || scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
+      return GMG_EWS;
+    SimParams& P = L.P;
+    fill_out(P, d_out, opts);
+    P.base = b->db;
+    P.ld = b->db.ld;
+    P.K = K;
+    P.move_off = d_move_off;
+    P.move_op = d_move_op;
+    P.move_dev = d_move_dev;
+    P.scratch = static_cast<uint8_t*>(d_scratch);
+    A.P = P;
+    A.ck = b->ck;
+    A.pre_status = nullptr;
+    return launch_arb_inc(g->dg.t32 != 0, g->dg.ntypes >= 2, A, L.grid, 32 * L.wpb, L.smem,
+                          reinterpret_cast<cudaStream_t>(stream)) == cudaSuccess
+               ? GMG_OK
+               : GMG_ECUDA;
+  }
   if (arbitrated(opts)) {
     // Arbitrated transfers: every candidate's moved placement is simulated in
     // full (the base snapshot's resume points hold no transfer state).

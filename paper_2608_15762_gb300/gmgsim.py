@@ -367,9 +367,13 @@ def sim_batch_noalloc(g: Gmg, place, out: Optional[SimOut] = None, req_done=Fals
 
 
 class Base:
-    """A recorded base schedule (base_create) and the workspace it borrows."""
+    """A recorded base schedule (base_create) and the workspace it borrows.
+    ``arbitrated``: the base placement simulated with arbitrated transfers
+    (Sec. 3.5.2), with the arbiter's state at every resume point; such a base
+    serves arbitrated candidates only, which it resumes instead of
+    re-simulating (at most 32 accelerators)."""
 
-    def __init__(self, g: Gmg, base_place, queue_cap=0, stream=None):
+    def __init__(self, g: Gmg, base_place, queue_cap=0, stream=None, arbitrated=False):
         import torch
         assert base_place.dtype == torch.uint8 and base_place.is_contiguous()
         ld = (g.n_ops + 15) // 16 * 16
@@ -377,7 +381,8 @@ class Base:
         row[:base_place.numel()] = base_place[:ld].reshape(-1)
         self.row = row
         self.g = g
-        o = _opts(0, None, queue_cap)
+        o = _opts(0, None, queue_cap, arbitrated=arbitrated)
+        self.arbitrated = bool(arbitrated)
         nbytes = lib().base_workspace_bytes(g.handle, C.addressof(o))
         self.ws = _aligned_empty(nbytes, base_place.device)
         h = C.c_void_p()
@@ -400,8 +405,8 @@ class Base:
 
 
 @_traced("base_create")
-def base_create(g: Gmg, base_place, queue_cap=0, stream=None) -> Base:
-    return Base(g, base_place, queue_cap, stream)
+def base_create(g: Gmg, base_place, queue_cap=0, stream=None, arbitrated=False) -> Base:
+    return Base(g, base_place, queue_cap, stream, arbitrated)
 
 
 @_traced("sim_incremental")
@@ -409,8 +414,8 @@ def sim_incremental(g: Gmg, base: Base, move_off, move_op, move_dev, out: Option
                     scratch: Optional[Scratch] = None, req_done=False, trace_k=None, queue_cap=0,
                     warps_per_block=0, stream=None, arbitrated=False) -> SimOut:
     """K move lists (CUDA int32 off[K+1], int32 op[M], uint8 dev[M]) against ``base``;
-    ``arbitrated``: transfers go through the arbiter of Sec. 3.5.2 (each moved
-    placement is then simulated in full)."""
+    ``arbitrated``: transfers go through the arbiter of Sec. 3.5.2 -- resumed
+    from an arbitrated base, else each moved placement simulated in full."""
     K = int(move_off.numel()) - 1
     n_trace = 0 if trace_k is None else int(trace_k.numel())
     if out is None:

@@ -196,11 +196,11 @@ def test_degenerate_inputs_and_refusals():
     with pytest.raises(G.GmgError) as ei:
         G.sim_batch(G.gmg_create(dw), torch_place(rw), arbitrated=True)
     assert ei.value.code == G.GMG_ERANGE
-    # a base snapshot is only made without arbitration
+    # an arbitrated base snapshot also keeps the arbiter's checkpoints
     o = G._opts(arbitrated=True)
     import ctypes as C
-    assert G.lib().inc_scratch_bytes(g.handle, 4, C.addressof(o)) > 0   # moved placements in full
-    assert G.lib().base_workspace_bytes(g.handle, C.addressof(o)) == 0
+    assert G.lib().inc_scratch_bytes(g.handle, 4, C.addressof(o)) > 0
+    assert G.lib().base_workspace_bytes(g.handle, C.addressof(o)) > 0
 
 
 def test_decode_memtight_full_size_sampled():
@@ -302,3 +302,70 @@ def test_incremental_arbitrated_ignores_a_base_queue_limit():
     s, pk, rq = O.incremental_batch(d, base, mv, arbitrated=True)
     compare(arb.to_numpy(), s, pk, rq)
     assert (arb.status.cpu().numpy() == 0).all()
+
+
+# ---------------------------------------------------------------------------
+# Incremental candidates resumed from an arbitrated base snapshot
+# ---------------------------------------------------------------------------
+
+def _resumed(d, base_place, mv, **kw):
+    g = G.gmg_create(d)
+    b = G.base_create(g, torch.from_numpy(np.ascontiguousarray(base_place[:d.n_ops])).cuda(), arbitrated=True)
+    off, op, dv = G.moves_to_device(mv, "cuda")
+    out = G.sim_incremental(g, b, off, op, dv, req_done=True, arbitrated=True, **kw)
+    torch.cuda.synchronize()
+    s, pk, rq = O.incremental_batch(d, base_place[:d.n_ops], mv, arbitrated=True, resumed=True)
+    got = out.to_numpy()
+    compare(got, s, pk, rq)
+    return got, s
+
+
+@pytest.mark.parametrize("seed,n,D,links,kw", [
+    (90, 60, 3, None, {}),
+    (91, 300, 8, "pair", {}),
+    (92, 500, 16, "uplink", dict(explicit_cons=True)),
+    (93, 400, 32, "random", {}),
+    (94, 300, 6, None, dict(n_types=2)),
+    (95, 300, 8, "pair", dict(dur_hi=1 << 31)),   # times beyond 2^31: 64-bit instances
+    (96, 250, 5, None, dict(zero=True)),
+])
+def test_resumed_candidates_bit_exact(seed, n, D, links, kw):
+    """Move lists against an arbitrated base snapshot: each candidate resumes
+    at the latest checkpoint before its T0 -- the arbiter's queues, holds and
+    FIFOs restored, a moved op's inputs recounted, its predecessors' remote
+    sets, holds and FIFO places repaired -- and equals the full arbitrated
+    simulation of its moved placement; events counts the ops with arbitrated
+    base ready time >= T0."""
+    zero = kw.pop("zero", False)
+    d, rows = _case(seed, n, D, links, zero=zero, **kw)
+    base = rows[0, :n].copy()
+    mv = W.random_moves(seed, 96, base, D, max_moves=8)
+    mv.dev[mv.off[3]] = D                            # a device out of range
+    got, s = _resumed(d, base, mv)
+    ok = got["status"] == 0
+    assert got["status"][3] == G.SIM_MOVE_RANGE
+    assert (got["events"][ok] < n).mean() > 0.5
+
+
+def test_resumed_workload_every_candidate():
+    """All 16,384 move lists of the incremental workload (32 x 32-layer
+    graph, 16 accelerators) resumed from its arbitrated base."""
+    wl = W.make_workload(3)
+    got, s = _resumed(wl.desc, wl.base_place, wl.moves)
+    assert (got["status"] == 0).all()
+    assert got["events"].mean() < 0.9 * wl.desc.n_ops
+
+
+def test_arbitrated_base_serves_arbitrated_candidates_only():
+    d, rows = _case(97, 80, 4, None)
+    base = rows[0, :80].copy()
+    mv = W.random_moves(97, 8, base, 4, max_moves=3)
+    g = G.gmg_create(d)
+    b = G.base_create(g, torch.from_numpy(base).cuda(), arbitrated=True)
+    off, op, dv = G.moves_to_device(mv, "cuda")
+    with pytest.raises(G.GmgError) as e:
+        G.sim_incremental(g, b, off, op, dv)
+    assert e.value.code == G.GMG_EINVAL
+    wide = W.random_desc(98, 60, 40)
+    with pytest.raises(G.GmgError):
+        G.base_create(G.gmg_create(wide), torch.zeros(64, dtype=torch.uint8, device="cuda"), arbitrated=True)
