@@ -202,6 +202,10 @@ def prepare(config: int, rank: int, world: int, device, cap=None, arbitrated=Fal
     p = Prepared()
     p.wl = wl
     p.arb = arbitrated
+    # on up to 32 accelerators the arbitrated base snapshot keeps the
+    # arbiter's checkpoints and candidates resume from it; on more, every
+    # moved placement is simulated in full
+    p.arb_base = arbitrated and wl.desc.n_dev <= 32
     p.structured = structured
     p.staging = {"default": G.GMG_STAGING_DEFAULT, "shared": G.GMG_STAGING_SHARED, "l1": G.GMG_STAGING_L1}[staging]
     if arbitrated and wl.desc.n_dev > 256:
@@ -263,7 +267,7 @@ def run_step(p, ev=None):
         with torch.cuda.stream(p.side):
             if ev:
                 ev["base"][0].record()
-            b = G.base_create(p.g, p.base_place, stream=p.side)
+            b = G.base_create(p.g, p.base_place, stream=p.side, arbitrated=p.arb_base)
             if ev:
                 ev["base"][1].record()
                 ev["inc"][0].record()
@@ -272,7 +276,7 @@ def run_step(p, ev=None):
             if ev:
                 ev["inc"][1].record()
         p._base = b  # keep alive until the stream has used it
-        launches += 2 if not p.arb else 3
+        launches += 3 if p.arb and not p.arb_base else 2
     if p.n_full:
         if ev:
             ev["full"][0].record()
@@ -854,8 +858,9 @@ def main():
     arb_kern = "sim_arb_kernel" if D <= 32 else "sim_arbw_kernel"
     staged_run = p.staging == 1 or (p.staging == 0 and p.g.info["stageable"] == 1 and not p.arb)
     full_kern = "sim_full_staged_kernel" if staged_run else "sim_full_kernel"
-    kname = {"full": arb_kern if p.arb else full_kern, "inc": arb_kern if p.arb else "sim_inc_kernel",
-             "base": "sim_base_kernel"}
+    kname = {"full": arb_kern if p.arb else full_kern,
+             "inc": "sim_arb_inc_kernel" if p.arb_base else arb_kern if p.arb else "sim_inc_kernel",
+             "base": "sim_arb_base_kernel" if p.arb_base else "sim_base_kernel"}
     kcount = {"full": p.n_full, "inc": p.n_inc, "base": 1}
     out_bytes_per_cand = 8 + 8 + 4 + 4 + 4 + 4 + 8 + 4 + 8 + 8 * D
     alg_bytes = {"full": p.n_full * (W_ld(N) + out_bytes_per_cand),
@@ -866,7 +871,7 @@ def main():
     kernels = {}
     for n in names:
         ppath = profile_path(kname[n], wname)
-        extra = () if not p.arb or n == "base" else (ARB_SOURCES if D <= 32 else ARBW_SOURCES)
+        extra = () if not p.arb or (n == "base" and not p.arb_base) else (ARB_SOURCES if D <= 32 else ARBW_SOURCES)
         prof = read_profile(ppath, extra)
         kd = {"kernel": kname[n], "launch_ms": kern_ms[n], "units": kcount[n],
               "hbm_gbs": alg_bytes[n] / (kern_ms[n] / 1000) / 1e9, "inst_per_launch": None, "issue_frac": None,
@@ -905,6 +910,9 @@ def main():
         "config": {"workload": wl.name, "candidates": K_all, "full_placements": p.n_full_total,
                    "incremental_candidates": p.n_inc_total, "n_ops": N, "n_dev": D,
                    "transfers": "arbitrated" if p.arb else "latency",
+                   "incremental": ("resumed from the arbitrated base snapshot" if p.arb_base else
+                                   "moved placements simulated in full" if p.arb else
+                                   "resumed from the base snapshot") if p.n_inc_total else None,
                    "placements": "structured" if p.structured else "uniform",
                    "gmg_staging": "shared memory (bulk-copied once per CTA)" if staged_run else "L1 path",
                    "l2": "flushed between steps (256 MiB write), each step timed with CUDA events",

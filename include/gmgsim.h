@@ -265,13 +265,22 @@ size_t base_workspace_bytes(const gmg_t* g, const sim_opts_t* opts);
  * incremental candidates resume from: per-op ready and finish times and
  * snapshots of the simulator state at time boundaries (the GMG snapshot of
  * Sec. 3.3.2 from which a simulator can be rebuilt at any instant).
- * Asynchronous on `stream`; *out receives the handle. */
+ * Asynchronous on `stream`; *out receives the handle.
+ *   - opts->transfer_mode GMG_TRANSFER_ARBITRATED (at most 32 accelerators,
+ *     a graph with link ids): the base is simulated with the arbiter of
+ *     Sec. 3.5.2 and each snapshot also keeps the arbiter's state (input
+ *     counters, holds, intent FIFOs, pair queues, endpoint and link sets);
+ *     such a base serves arbitrated candidates only.  On more accelerators
+ *     the call returns GMG_EINVAL; take a pure-latency base there (arbitrated
+ *     candidates against it are simulated in full).
+ *   - GMG_STAGING_SHARED in opts->gmg_staging is refused (GMG_EINVAL). */
 int base_create(const gmg_t* g, const uint8_t* d_base_place, const sim_opts_t* opts,
                 void* d_base_ws, size_t ws_bytes, gmg_stream_t stream, gmg_base_t** out);
 
 void base_destroy(gmg_base_t* b);
 
-/* Bytes of device scratch sim_incremental needs for K candidates. */
+/* Bytes of device scratch sim_incremental needs for K candidates (with
+ * arbitrated opts: enough for either kind of base). */
 size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts);
 
 /* K candidates, each a list of moves (op, device) against the base
@@ -280,8 +289,14 @@ size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts);
  * moves can change is re-simulated, from T0 = min over effective moves x of
  * (min base finish of x's predecessors, or x's release).  Move lists are CSR
  * on the device: ops d_move_op[d_move_off[k]..d_move_off[k+1]) go to
- * d_move_dev[...].  events[k] = ops whose base ready time is >= T0
- * (n_ops with GMG_TRANSFER_ARBITRATED: the moved placement is simulated in full). */
+ * d_move_dev[...].  events[k] = ops whose base ready time is >= T0.
+ *   - With GMG_TRANSFER_ARBITRATED and an arbitrated base, candidates resume
+ *     from the base's arbiter snapshots the same way; with a pure-latency
+ *     base, each moved placement is simulated in full (events[k] = n_ops).
+ *     An arbitrated base with pure-latency opts returns GMG_EINVAL.
+ *   - The first 256 bytes of d_scratch hold a candidate counter that the call
+ *     zeroes on `stream` before its launch (warps take resumed candidates one
+ *     at a time); calls sharing one scratch buffer must be ordered. */
 int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_off,
                     const int32_t* d_move_op, const uint8_t* d_move_dev, int32_t K,
                     const sim_opts_t* opts, const sim_out_t* d_out, void* d_scratch,

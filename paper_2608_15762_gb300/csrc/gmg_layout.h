@@ -106,6 +106,8 @@ struct DevGmg {
   const int32_t* st_rel;      // [N] release
   int32_t stage_ok;           // 1: 32-bit times, one type, uniform links, lists and sizes fit the fields
   int32_t n_edges;
+  const uint8_t* ws;          // the whole device copy (every array above), for L2 prefetches
+  int64_t ws_bytes;
 };
 
 // Bytes of the staged copy in shared memory: an mbarrier, then the four
@@ -208,6 +210,14 @@ struct SimParams {
   int32_t pad_;
   // byte offsets inside a slot (off_pk < 0: the peaks are in shared memory)
   int64_t off_f, off_hold, off_bits, off_creq, off_qk, off_mk, off_md, off_row, off_pk;
+  // Incremental candidates: the next candidate a warp takes (zeroed before
+  // the launch).  Resumed candidates differ widely in length, so warps take
+  // them one at a time instead of a fixed stride.
+  uint32_t* next_k;
 };
+
+// Scratch bytes in front of the slots of a resumed incremental launch (the
+// candidate counter).
+constexpr size_t kCounterBytes = 256;
 
 }  // namespace gsim

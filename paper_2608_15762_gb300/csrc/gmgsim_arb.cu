@@ -433,22 +433,23 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT
 
   __device__ uint8_t* arena(int c) const { return A.ck.arena + (int64_t)c * A.ck.bytes; }
 
+  // The base runs with 64-bit times, so every per-op array has the arena's
+  // element size and is copied as bytes (each region of the slot and of the
+  // arena is padded to 256 bytes).
   __device__ void save_arb(int c) {
+    static_assert(kMode != kBase || !kT32, "the base snapshot keeps 64-bit times");
     const unsigned lane = lane_id();
     uint8_t* a = arena(c);
     const ArbCk& K = A.ck;
-    for (int x = lane; x < g.n; x += 32) {
-      reinterpret_cast<int32_t*>(a + K.off_cnt)[x] = cnt()[x];
-      reinterpret_cast<int64_t*>(a + K.off_rmax)[x] = (int64_t)rmax()[x];
-      reinterpret_cast<int32_t*>(a + K.off_refs)[x] = refs()[x];
-      reinterpret_cast<uint32_t*>(a + K.off_rmask)[x] = rmask()[x];
-      reinterpret_cast<int32_t*>(a + K.off_nextop)[x] = nextop()[x];
-      reinterpret_cast<int64_t*>(a + K.off_hold)[x] = (int64_t)this->holdb[x];
-    }
-    for (int x = lane; x < nx; x += 32) {
-      reinterpret_cast<uint32_t*>(a + K.off_xent)[x] = xent()[x];
-      reinterpret_cast<int32_t*>(a + K.off_xnext)[x] = xnext()[x];
-    }
+    const int64_t n = g.n;
+    warp_copy16(a + K.off_cnt, cnt(), 4 * n);
+    warp_copy16(a + K.off_rmax, rmax(), 8 * n);
+    warp_copy16(a + K.off_refs, refs(), 4 * n);
+    warp_copy16(a + K.off_rmask, rmask(), 4 * n);
+    warp_copy16(a + K.off_nextop, nextop(), 4 * n);
+    warp_copy16(a + K.off_hold, this->holdb, 8 * n);
+    warp_copy16(a + K.off_xent, xent(), 4 * (int64_t)nx);
+    warp_copy16(a + K.off_xnext, xnext(), 4 * (int64_t)nx);
     for (int x = lane; x < g.D * g.D; x += 32) {
       reinterpret_cast<int32_t*>(a + K.off_qhead)[x] = qhead()[x];
       reinterpret_cast<int32_t*>(a + K.off_qtail)[x] = qtail()[x];
@@ -478,17 +479,35 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT
     return v >= (int64_t)kNever ? kNever : (tm_t)v;
   }
 
+  // An arena's 64-bit times into this kernel's time type, four loads in
+  // flight per lane.
+  static __device__ void narrow_times(tm_t* dst, const int64_t* src, int n) {
+    int x = (int)lane_id();
+    for (; x + 96 < n; x += 128) {
+      const int64_t a = src[x], b = src[x + 32], c = src[x + 64], e = src[x + 96];
+      dst[x] = narrow_time(a);
+      dst[x + 32] = narrow_time(b);
+      dst[x + 64] = narrow_time(c);
+      dst[x + 96] = narrow_time(e);
+    }
+    for (; x < n; x += 32) dst[x] = narrow_time(src[x]);
+  }
+
   __device__ void restore_arb(int c) {
     const unsigned lane = lane_id();
     const uint8_t* a = arena(c);
     const ArbCk& K = A.ck;
-    for (int x = lane; x < g.n; x += 32) {
-      cnt()[x] = reinterpret_cast<const int32_t*>(a + K.off_cnt)[x];
-      rmax()[x] = narrow_time(reinterpret_cast<const int64_t*>(a + K.off_rmax)[x]);
-      refs()[x] = reinterpret_cast<const int32_t*>(a + K.off_refs)[x];
-      rmask()[x] = reinterpret_cast<const uint32_t*>(a + K.off_rmask)[x];
-      nextop()[x] = reinterpret_cast<const int32_t*>(a + K.off_nextop)[x];
-      this->holdb[x] = narrow_time(reinterpret_cast<const int64_t*>(a + K.off_hold)[x]);
+    const int64_t n = g.n;
+    warp_copy16(cnt(), a + K.off_cnt, 4 * n);
+    warp_copy16(refs(), a + K.off_refs, 4 * n);
+    warp_copy16(rmask(), a + K.off_rmask, 4 * n);
+    warp_copy16(nextop(), a + K.off_nextop, 4 * n);
+    if (kT32) {
+      narrow_times(rmax(), reinterpret_cast<const int64_t*>(a + K.off_rmax), g.n);
+      narrow_times(this->holdb, reinterpret_cast<const int64_t*>(a + K.off_hold), g.n);
+    } else {
+      warp_copy16(rmax(), a + K.off_rmax, 8 * n);
+      warp_copy16(this->holdb, a + K.off_hold, 8 * n);
     }
     const int64_t* w = reinterpret_cast<const int64_t*>(a + K.off_warp);
     nx = (int32_t)w[0];
@@ -496,10 +515,8 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT
     sendm = (uint32_t)w[2];
     recvm = (uint32_t)w[3];
     lbits()[lane] = reinterpret_cast<const uint32_t*>(w + 4)[lane];
-    for (int x = lane; x < nx; x += 32) {
-      xent()[x] = reinterpret_cast<const uint32_t*>(a + K.off_xent)[x];
-      xnext()[x] = reinterpret_cast<const int32_t*>(a + K.off_xnext)[x];
-    }
+    warp_copy16(xent(), a + K.off_xent, 4 * (int64_t)nx);
+    warp_copy16(xnext(), a + K.off_xnext, 4 * (int64_t)nx);
     for (int x = lane; x < g.D * g.D; x += 32) {
       qhead()[x] = reinterpret_cast<const int32_t*>(a + K.off_qhead)[x];
       qtail()[x] = reinterpret_cast<const int32_t*>(a + K.off_qtail)[x];
@@ -619,8 +636,7 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT
       this->write_invalid(k, bad ? GMG_SIM_MOVE_RANGE : GMG_SIM_MOVE_DUP);
       return;
     }
-    for (int c = lane * 16; c < B.ld; c += 512)
-      *reinterpret_cast<uint4*>(crow + c) = *reinterpret_cast<const uint4*>(B.row + c);
+    warp_copy16(crow, B.row, B.ld);
     __syncwarp();
     uint64_t t0 = kKeyMax;
     for (int t = lane; t < nm; t += 32) {
@@ -700,7 +716,7 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT
     this->opn = 0;
     this->dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
     for (int r = lane; r < g.R; r += 32) this->creq[r] = B.ck_creq[(int64_t)c * g.R + r];
-    this->zero_fin();
+    this->fill_fin();
     restore_arb(c);
     // READY keys, except those of moved ops (recomputed below)
     int nq = 0;
@@ -846,6 +862,7 @@ __global__ void __launch_bounds__(32) sim_arb_base_kernel(const __grid_constant_
   S.setup_arb(0, smem + A.smem_std);
   const DevBase& B = A.P.base;
   const unsigned lane = lane_id();
+  warp_prefetch_l2(A.P.g.ws, A.P.g.ws_bytes);
   for (int c = lane * 16; c < B.ld; c += 512)
     *reinterpret_cast<uint4*>(B.row + c) = *reinterpret_cast<const uint4*>(A.P.place + c);
   for (int c = lane; c < B.nck; c += 32) B.ck_time[c] = kI64Max;
@@ -890,14 +907,13 @@ __global__ void __launch_bounds__(128, 7) sim_arb_inc_kernel(const __grid_consta
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
-  const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
   ArbSim<kT32, kTypes, kInc> S(A);
   setup_slot(S, A.P, wib, slot, smem);
   S.setup_arb(slot, smem + A.smem_std + (size_t)wib * A.smem_arb);
   S.rb = A.P.base.rb;
   S.fb = A.P.base.fb;
   uint8_t* crow = A.P.scratch + slot * A.P.slot_bytes + A.P.off_row;
-  for (int64_t k = slot; k < A.P.K; k += nslots) S.inc_candidate(k, crow);
+  for (int64_t k = take_candidate(A.P.next_k); k < A.P.K; k = take_candidate(A.P.next_k)) S.inc_candidate(k, crow);
 }
 
 // One warp per incremental candidate: check the move list (an op or device
@@ -930,8 +946,7 @@ __global__ void __launch_bounds__(128) expand_moves_kernel(const uint8_t* base_r
       if (__any_sync(kFullMask, dup)) st = GMG_SIM_MOVE_DUP;
     }
     uint8_t* rw = rows + k * (int64_t)ld;
-    for (int32_t c = (int32_t)lane * 16; c < ld; c += 512)
-      *reinterpret_cast<uint4*>(rw + c) = *reinterpret_cast<const uint4*>(base_row + c);
+    warp_copy16(rw, base_row, ld);
     __syncwarp();
     if (st == GMG_SIM_OK)
       for (int32_t m = a + (int32_t)lane; m < b; m += 32) rw[op[m]] = dev[m];

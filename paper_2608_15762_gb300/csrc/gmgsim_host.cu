@@ -1003,6 +1003,8 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   G.st_hot = reinterpret_cast<const uint4*>(w + L.off_st_hot);
   G.st_rel = reinterpret_cast<const int32_t*>(w + L.off_st_rel);
   G.n_edges = b.E;
+  G.ws = w;
+  G.ws_bytes = (int64_t)L.total;
   // every time < 2^tb fits int32; the 32-bit instances also take the
   // accelerator id from the event key
   G.t32 = (G.tb <= 31 && G.dev_key) ? 1 : 0;
@@ -1263,12 +1265,23 @@ size_t inc_scratch_bytes(const gmg_t* g, int32_t K, const sim_opts_t* opts) {
     Launch L;
     ArbParams A;
     if (g->dg.D <= 32 && plan_arb_resumed(g, K, opts, L, A) == GMG_OK)
-      need = std::max(need, (size_t)L.slots * (size_t)L.P.slot_bytes);
+      need = std::max(need, kCounterBytes + (size_t)L.slots * (size_t)L.P.slot_bytes);
     return need;
   }
   Launch L;
   if (plan_launch(g, K, opts, true, L)) return 0;
-  return (size_t)L.slots * (size_t)L.P.slot_bytes;
+  return kCounterBytes + (size_t)L.slots * (size_t)L.P.slot_bytes;
+}
+
+// A resumed incremental launch's scratch: the candidate counter, zeroed on
+// the stream, then the slots.
+static int take_counter(SimParams& P, void* d_scratch, size_t scratch_bytes, const Launch& L, cudaStream_t st) {
+  if (!d_scratch || !aligned(d_scratch, 256) ||
+      scratch_bytes < kCounterBytes + (size_t)L.slots * (size_t)L.P.slot_bytes)
+    return GMG_EWS;
+  P.next_k = static_cast<uint32_t*>(d_scratch);
+  P.scratch = static_cast<uint8_t*>(d_scratch) + kCounterBytes;
+  return cudaMemsetAsync(P.next_k, 0, sizeof(uint32_t), st) == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }
 
 int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_off, const int32_t* d_move_op,
@@ -1287,9 +1300,9 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
     ArbParams A;
     rc = plan_arb_resumed(g, K, opts, L, A);
     if (rc) return rc;
-    if (!d_scratch || !aligned(d_scratch, 256) || scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
-      return GMG_EWS;
     SimParams& P = L.P;
+    rc = take_counter(P, d_scratch, scratch_bytes, L, reinterpret_cast<cudaStream_t>(stream));
+    if (rc) return rc;
     fill_out(P, d_out, opts);
     P.base = b->db;
     P.ld = b->db.ld;
@@ -1297,7 +1310,6 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
     P.move_off = d_move_off;
     P.move_op = d_move_op;
     P.move_dev = d_move_dev;
-    P.scratch = static_cast<uint8_t*>(d_scratch);
     A.P = P;
     A.ck = b->ck;
     A.pre_status = nullptr;
@@ -1340,10 +1352,9 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
   Launch L;
   rc = plan_launch(g, K, opts, true, L);
   if (rc) return rc;
-  if (!d_scratch || !aligned(d_scratch, 256) ||
-      scratch_bytes < (size_t)L.slots * (size_t)L.P.slot_bytes)
-    return GMG_EWS;
   SimParams& P = L.P;
+  rc = take_counter(P, d_scratch, scratch_bytes, L, reinterpret_cast<cudaStream_t>(stream));
+  if (rc) return rc;
   fill_out(P, d_out, opts);
   P.base = b->db;
   P.ld = b->db.ld;
@@ -1351,7 +1362,6 @@ int sim_incremental(const gmg_t* g, const gmg_base_t* b, const int32_t* d_move_o
   P.move_off = d_move_off;
   P.move_op = d_move_op;
   P.move_dev = d_move_dev;
-  P.scratch = static_cast<uint8_t*>(d_scratch);
   cudaError_t e = launch_inc(L.reg, P, L.grid, 32 * L.wpb, L.smem, reinterpret_cast<cudaStream_t>(stream));
   return e == cudaSuccess ? GMG_OK : GMG_ECUDA;
 }

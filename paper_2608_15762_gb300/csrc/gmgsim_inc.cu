@@ -46,8 +46,7 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, co
     return;
   }
   // The candidate's placement = base + moves.
-  for (int c = lane * 16; c < B.ld; c += 512)
-    *reinterpret_cast<uint4*>(crow + c) = *reinterpret_cast<const uint4*>(B.row + c);
+  warp_copy16(crow, B.row, B.ld);
   __syncwarp();
   uint64_t t0 = kKeyMax;
   for (int t = lane; t < nm; t += 32) {
@@ -132,9 +131,9 @@ __device__ void inc_candidate(Sim<kReg, kInc, kKey, kT32, kTypes, kBatch>& S, co
   S.opn = 0;
   S.dv.load(B.ck_dev + (int64_t)c * 3 * g.D);
   for (int r = lane; r < g.R; r += 32) S.creq[r] = B.ck_creq[(int64_t)c * g.R + r];
-  // ops started before T_c are those with base ready time < T_c (fin()
-  // reads their base finish); the others start with no finish time
-  S.zero_fin();
+  // ops started before T_c are those with base ready time < T_c: they keep
+  // their base finish; the others start with no finish time
+  S.fill_fin();
   // READY keys at T_c; a moved op's key is recomputed (its inputs' transfer
   // times change; its predecessors all finished before T_c).
   for (int x = lane; x < qsz; x += 32) {
@@ -317,13 +316,12 @@ __global__ void __launch_bounds__(128, kBatch ? kBatchBlocksPerSM : 7) sim_inc_k
   extern __shared__ __align__(16) uint8_t smem[];
   const unsigned wib = threadIdx.x >> 5;
   const int64_t slot = (int64_t)blockIdx.x * (blockDim.x >> 5) + wib;
-  const int64_t nslots = (int64_t)gridDim.x * (blockDim.x >> 5);
   Sim<kReg, kInc, kKey, kT32, kTypes, kBatch> S(P);
   setup_slot(S, P, wib, slot, smem);
   S.rb = P.base.rb;
   S.fb = P.base.fb;
   uint8_t* crow = P.scratch + slot * P.slot_bytes + P.off_row;
-  for (int64_t k = slot; k < P.K; k += nslots) inc_candidate(S, P, k, crow);
+  for (int64_t k = take_candidate(P.next_k); k < P.K; k = take_candidate(P.next_k)) inc_candidate(S, P, k, crow);
 }
 
 }  // namespace

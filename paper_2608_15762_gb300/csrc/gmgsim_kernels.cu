@@ -15,6 +15,7 @@ __global__ void __launch_bounds__(32) sim_base_kernel(const __grid_constant__ Si
   setup_slot(S, P, 0, 0, smem);
   const DevBase& B = P.base;
   const unsigned lane = lane_id();
+  warp_prefetch_l2(P.g.ws, P.g.ws_bytes);
   // keep a copy of the base placement for the candidates
   for (int c = lane * 16; c < B.ld; c += 512)
     *reinterpret_cast<uint4*>(B.row + c) = *reinterpret_cast<const uint4*>(P.place + c);

@@ -73,6 +73,45 @@ __device__ __forceinline__ uint64_t warp_max_u64(uint64_t v) {
 __device__ __forceinline__ unsigned lane_id() { return threadIdx.x & 31u; }
 __device__ __forceinline__ uint32_t lanes_below() { return (1u << lane_id()) - 1u; }
 
+// Bulk prefetch of [p, p + bytes) into L2 (no completion to wait for), 32 KB
+// pieces spread over the warp.  p is 16-byte aligned; a ragged tail below 16
+// bytes is left out.  Single-warp kernels that walk the graph serially start
+// with it, so that their dependent loads hit L2 instead of DRAM.
+__device__ __forceinline__ void warp_prefetch_l2(const void* p, int64_t bytes) {
+  const uint64_t a = (uint64_t)__cvta_generic_to_global(p);
+  constexpr int64_t kPiece = 1 << 15;
+  for (int64_t o = (int64_t)lane_id() * kPiece; o < bytes; o += 32 * kPiece) {
+    const int64_t left = bytes - o;
+    const uint32_t sz = (uint32_t)((left < kPiece ? left : kPiece) & ~int64_t(15));
+    if (sz) asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" :: "l"(a + o), "r"(sz) : "memory");
+  }
+}
+
+// The next candidate of a launch that hands them out one at a time (uniform).
+__device__ __forceinline__ int64_t take_candidate(uint32_t* next_k) {
+  uint32_t k = 0;
+  if (lane_id() == 0) k = atomicAdd(next_k, 1u);
+  return (int64_t)__shfl_sync(kFullMask, k, 0);
+}
+
+// Warp copy of `bytes` rounded up to a multiple of 16 between 16-byte
+// aligned buffers (both must extend to the rounded size), four 16-byte
+// loads in flight per lane.
+__device__ __forceinline__ void warp_copy16(void* dst, const void* src, int64_t bytes) {
+  const int64_t nv = (bytes + 15) >> 4;
+  uint4* d = static_cast<uint4*>(dst);
+  const uint4* s = static_cast<const uint4*>(src);
+  int64_t i = lane_id();
+  for (; i + 96 < nv; i += 128) {
+    const uint4 a = s[i], b = s[i + 32], c = s[i + 64], e = s[i + 96];
+    d[i] = a;
+    d[i + 32] = b;
+    d[i + 64] = c;
+    d[i + 96] = e;
+  }
+  for (; i < nv; i += 32) d[i] = s[i];
+}
+
 // 16-byte pieces of an OpRec, loaded through the read-only path.
 __device__ __forceinline__ longlong2 op_durbytes(const OpRec* ops, uint32_t i) {
   return __ldg(reinterpret_cast<const longlong2*>(ops + i));
@@ -483,8 +522,6 @@ struct Sim {
   // the finish array is zeroed per candidate; the batched sweep marks an op
   // whose READY key is queued with -1).
   __device__ __forceinline__ bool popped(uint32_t x) const { return fin(x) > 0; }
-  // Finish time of a simulated op (incremental: ops before the resume point
-  // keep their base finish).
   // The low 32 bits of a base-snapshot time (little-endian int64).
   static __device__ __forceinline__ tm_t base_time(const int64_t* a, uint32_t x) {
     if (kT32) return (tm_t)__ldg(reinterpret_cast<const int32_t*>(a) + 2 * (size_t)x);
@@ -497,10 +534,9 @@ struct Sim {
     if (kTypes) return __ldg(g.durt + (size_t)i * g.ntypes + __ldg(g.dtype + d));
     return dflt;
   }
-  __device__ __forceinline__ tm_t fin(uint32_t x) const {
-    if (kMode == kInc && base_time(rb, x) < Tc) return base_time(fb, x);
-    return fbuf[x];
-  }
+  // Finish time of a simulated op (incremental candidates start from
+  // fill_fin: ops started before the resume point keep their base finish).
+  __device__ __forceinline__ tm_t fin(uint32_t x) const { return fbuf[x]; }
 
   // Transfer estimator of one output over link d -> e (d != e), Sec. 3.3.1.
   __device__ __forceinline__ tm_t xfer(int d, int e, int64_t bytes, int64_t xq) const {
@@ -574,6 +610,34 @@ struct Sim {
     uint4* v = reinterpret_cast<uint4*>(fbuf);
     const int nv = (int)((sizeof(tm_t) * (size_t)g.n + 15) / 16);
     for (int x = lane_id(); x < nv; x += 32) v[x] = make_uint4(0u, 0u, 0u, 0u);
+    __syncwarp();
+  }
+
+  // An incremental candidate's finish times at the resume point T_c: the
+  // base finish of every op started before it (base ready time < T_c), zero
+  // for the others and for the padding.  Four ops in flight per lane.
+  __device__ void fill_fin() {
+    const int n = g.n;
+    const int np = (int)((sizeof(tm_t) * (size_t)n + 15) / 16 * 16 / sizeof(tm_t));
+    int x = (int)lane_id();
+    for (; x + 96 < np; x += 128) {
+      tm_t v[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = x + 32 * u;
+        const bool in = i < n;
+        const tm_t r = in ? base_time(rb, (uint32_t)i) : Tc;
+        const tm_t f = in ? base_time(fb, (uint32_t)i) : 0;
+        v[u] = r < Tc ? f : 0;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) fbuf[x + 32 * u] = v[u];
+    }
+    for (; x < np; x += 32) {
+      const bool in = x < n;
+      const tm_t r = in ? base_time(rb, (uint32_t)x) : Tc;
+      fbuf[x] = r < Tc ? base_time(fb, (uint32_t)x) : 0;
+    }
     __syncwarp();
   }
 
