@@ -442,14 +442,14 @@ struct ArbSim : ArbEvents<ArbSim<kT32, kTypes, kMode>, Sim<true, kMode, true, kT
     uint8_t* a = arena(c);
     const ArbCk& K = A.ck;
     const int64_t n = g.n;
-    warp_copy16(a + K.off_cnt, cnt(), 4 * n);
-    warp_copy16(a + K.off_rmax, rmax(), 8 * n);
-    warp_copy16(a + K.off_refs, refs(), 4 * n);
-    warp_copy16(a + K.off_rmask, rmask(), 4 * n);
-    warp_copy16(a + K.off_nextop, nextop(), 4 * n);
-    warp_copy16(a + K.off_hold, this->holdb, 8 * n);
-    warp_copy16(a + K.off_xent, xent(), 4 * (int64_t)nx);
-    warp_copy16(a + K.off_xnext, xnext(), 4 * (int64_t)nx);
+    warp_copy16<16>(a + K.off_cnt, cnt(), 4 * n);
+    warp_copy16<16>(a + K.off_rmax, rmax(), 8 * n);
+    warp_copy16<16>(a + K.off_refs, refs(), 4 * n);
+    warp_copy16<16>(a + K.off_rmask, rmask(), 4 * n);
+    warp_copy16<16>(a + K.off_nextop, nextop(), 4 * n);
+    warp_copy16<16>(a + K.off_hold, this->holdb, 8 * n);
+    warp_copy16<16>(a + K.off_xent, xent(), 4 * (int64_t)nx);
+    warp_copy16<16>(a + K.off_xnext, xnext(), 4 * (int64_t)nx);
     for (int x = lane; x < g.D * g.D; x += 32) {
       reinterpret_cast<int32_t*>(a + K.off_qhead)[x] = qhead()[x];
       reinterpret_cast<int32_t*>(a + K.off_qtail)[x] = qtail()[x];

@@ -95,19 +95,21 @@ __device__ __forceinline__ int64_t take_candidate(uint32_t* next_k) {
 }
 
 // Warp copy of `bytes` rounded up to a multiple of 16 between 16-byte
-// aligned buffers (both must extend to the rounded size), four 16-byte
-// loads in flight per lane.
+// aligned buffers (both must extend to the rounded size), kDepth 16-byte
+// loads in flight per lane (a single-warp kernel takes a deeper pipeline:
+// nothing else hides its load latency).
+template <int kDepth = 4>
 __device__ __forceinline__ void warp_copy16(void* dst, const void* src, int64_t bytes) {
   const int64_t nv = (bytes + 15) >> 4;
   uint4* d = static_cast<uint4*>(dst);
   const uint4* s = static_cast<const uint4*>(src);
   int64_t i = lane_id();
-  for (; i + 96 < nv; i += 128) {
-    const uint4 a = s[i], b = s[i + 32], c = s[i + 64], e = s[i + 96];
-    d[i] = a;
-    d[i + 32] = b;
-    d[i + 64] = c;
-    d[i + 96] = e;
+  for (; i + 32 * (kDepth - 1) < nv; i += 32 * kDepth) {
+    uint4 v[kDepth];
+#pragma unroll
+    for (int u = 0; u < kDepth; ++u) v[u] = s[i + 32 * u];
+#pragma unroll
+    for (int u = 0; u < kDepth; ++u) d[i + 32 * u] = v[u];
   }
   for (; i < nv; i += 32) d[i] = s[i];
 }
