@@ -175,8 +175,10 @@ typedef struct {
   int32_t batched_sweep; /* 1 if the simulation kernels start READY ops in batches (graphs on
                             more than 32 accelerators whose keys have room for a duration class) */
   int32_t t32;           /* 1 if the kernels carry times as 32-bit integers (time_bound < 2^31) */
-  int32_t stageable;     /* 1 if sim_batch can stage this graph's hot fields in shared memory
-                            (GMG_STAGING_SHARED; the default then does, with pure-latency transfers) */
+  int32_t stageable;     /* 1 if sim_batch can stage this graph's hot fields in shared memory on
+                            the current device (one accelerator type, uniform links, 32-bit times,
+                            at most 32 accelerators, and the copy fits beside one warp's areas);
+                            the default then stages, with pure-latency transfers */
   int32_t reserved_;
 } gmg_info_t;
 

@@ -1029,7 +1029,12 @@ int gmg_create(const gmg_desc_t* desc, void* d_ws, size_t ws_bytes, gmg_stream_t
   I.default_queue_cap = std::min<int64_t>(b.queue_bound, kDefaultQueueCap);
   I.batched_sweep = G.batch;
   I.t32 = G.t32;
-  I.stageable = G.stage_ok;
+  // staged only where the copy also fits beside a warp's areas on this device
+  I.stageable = 0;
+  if (G.stage_ok) {
+    Launch Ls;
+    I.stageable = plan_staged(g, 1, nullptr, Ls) == GMG_OK ? 1 : 0;
+  }
   *out = g;
   return GMG_OK;
 }

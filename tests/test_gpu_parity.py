@@ -291,3 +291,18 @@ def test_staging_refused_where_it_does_not_apply():
         with pytest.raises(G.GmgError) as e:
             G.sim_batch(g, torch_place(rows), gmg_staging=G.GMG_STAGING_SHARED, arbitrated=arb)
         assert e.value.code == G.GMG_EINVAL
+        assert g.info["stageable"] == (1 if arb else 0)   # arbitration is refused by the call only
+
+
+def test_stageable_reports_the_default():
+    """gmg_info_t.stageable says whether sim_batch stages the graph by
+    default: the prefill graph's copy fits in shared memory, the memory-tight
+    decode graph's (N = 197,632) does not, although both have the compact
+    fields; an explicit staging request on the latter is refused."""
+    assert G.gmg_create(W.make_workload(2).desc).info["stageable"] == 1
+    g4 = G.gmg_create(W.make_workload(4).desc)
+    assert g4.info["stageable"] == 0
+    rows = np.zeros((2, W.placement_ld(g4.n_ops)), np.uint8)
+    with pytest.raises(G.GmgError) as e:
+        G.sim_batch(g4, torch_place(rows), gmg_staging=G.GMG_STAGING_SHARED)
+    assert e.value.code == G.GMG_EINVAL
