@@ -741,7 +741,8 @@ def run_rounds(args):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--steps", type=int, default=None,
+                    help="timed steps (default: 20, fewer when a step is long -- about a minute of timed work)")
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--config", type=int, default=5, choices=[1, 2, 3, 4, 5, 6])
@@ -764,6 +765,8 @@ def main():
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
+    if args.steps is None and (args.impl == "reference" or args.estimators or args.rounds):
+        args.steps = 20
     if args.impl == "reference":
         return reference_arm(args)
     if args.estimators:
@@ -800,16 +803,26 @@ def main():
         torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
         return float(t.item())
 
-    for _ in range(args.warmup):
+    warm = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
+    for i in range(args.warmup):
+        if i == args.warmup - 1:
+            warm[0].record()
         run_step(p)
+        if i == args.warmup - 1:
+            warm[1].record()
     barrier()
+    steps = args.steps
+    if steps is None:
+        # about a minute of timed work: 20 steps, fewer when a step is long
+        warm_ms = max_over_ranks(warm[0].elapsed_time(warm[1])) if args.warmup else 0.0
+        steps = max(3, min(20, int(60000 // max(warm_ms, 1e-3))))
     sampler = ClockSampler(local)
     sampler.start()
     time.sleep(0.3)
     step_ev, kern_ev = [], []
     launches = 0
     names = [n for n, on in (("full", p.n_full), ("base", p.n_inc), ("inc", p.n_inc)) if on]
-    for _ in range(args.steps):
+    for _ in range(steps):
         flush.fill_(1)
         e = [torch.cuda.Event(enable_timing=True) for _ in range(2)]
         ke = {n: (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for n in names}
@@ -826,7 +839,7 @@ def main():
 
     # end to end through the public API with host buffers (fewer steps when a
     # step is long: at least 3, about a minute of work)
-    e2e_steps = max(3, min(args.steps, int(60000 // max(ms, 1e-3))))
+    e2e_steps = max(3, min(steps, int(60000 // max(ms, 1e-3))))
     run_e2e_step(p)
     barrier()
     t0 = time.perf_counter()
@@ -903,7 +916,7 @@ def main():
                         "note": "every kernel of the step (instructions from the committed ncu summaries) over "
                                 "the whole step time"}
     line = {
-        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": steps,
         "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "strong",
         "vs_baseline": None, "dtype": "int64", "data": "synthetic",
         "ms_per_step_best": min(step_ms), "ms_per_step_median": statistics.median(step_ms),
