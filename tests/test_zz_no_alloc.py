@@ -1,7 +1,8 @@
 """sim_batch_noalloc: the variant of sim_batch for callers that cannot
 allocate device memory (its scratch is a fixed buffer inside the library).
 Its results must equal sim_batch's on consecutive calls, which also shows
-that leftovers of one call in the shared buffer do not leak into the next."""
+that leftovers of one call in the shared buffer do not leak into the next,
+and the oracle's, bit for bit."""
 import ctypes as C
 
 import numpy as np
@@ -9,6 +10,8 @@ import pytest
 
 torch = pytest.importorskip("torch")
 
+from gpu_common import compare  # noqa: E402
+from oracle import oracle as O  # noqa: E402
 from paper_2608_15762_gb300 import gmgsim as G  # noqa: E402
 from paper_2608_15762_gb300 import workloads as W  # noqa: E402
 
@@ -50,17 +53,21 @@ def test_same_results_as_sim_batch_on_two_calls(which):
         a, b = ref.to_numpy(), got.to_numpy()
         for f in FIELDS:
             assert np.array_equal(a[f], b[f]), f
+        s, pk, rq = O.simulate_batch(desc, place.cpu().numpy())
+        compare(b, s, pk, rq)
 
 
-def _compare_calls(g, batches, **kw):
+def _compare_calls(g, desc, batches, arbitrated=False, **kw):
     for place in batches:
         tk = torch.tensor([0, place.shape[0] - 1], dtype=torch.int32, device="cuda")
-        ref = G.sim_batch(g, place, req_done=True, trace_k=tk, **kw)
-        got = G.sim_batch_noalloc(g, place, req_done=True, trace_k=tk, **kw)
+        ref = G.sim_batch(g, place, req_done=True, trace_k=tk, arbitrated=arbitrated, **kw)
+        got = G.sim_batch_noalloc(g, place, req_done=True, trace_k=tk, arbitrated=arbitrated, **kw)
         torch.cuda.synchronize()
         a, b = ref.to_numpy(), got.to_numpy()
         for f in FIELDS:
             assert np.array_equal(a[f], b[f]), f
+        s, pk, rq = O.simulate_batch(desc, place.cpu().numpy(), arbitrated=arbitrated)
+        compare(b, s, pk, rq)
 
 
 def test_arbitrated_transfers_on_two_calls():
@@ -68,7 +75,7 @@ def test_arbitrated_transfers_on_two_calls():
     40 accelerators (the two arbitrated kernels)."""
     for D in (8, 40):
         desc = W.random_desc(23 + D, 400, D)
-        _compare_calls(G.gmg_create(desc), [_rows(3, 97, 400, D), _rows(4, 33, 400, D)], arbitrated=True)
+        _compare_calls(G.gmg_create(desc), desc, [_rows(3, 97, 400, D), _rows(4, 33, 400, D)], arbitrated=True)
 
 
 def _chain(n, D, seed):
@@ -90,20 +97,22 @@ def test_fewer_slots_than_the_grid():
     dozen slots, fewer than sim_batch's grid, so each warp takes several
     candidates in turn."""
     n = 60_000
-    g = G.gmg_create(_chain(n, 3, 5))
+    desc = _chain(n, 3, 5)
+    g = G.gmg_create(desc)
     slot = G.sim_scratch_bytes(g, 1) // 4          # one block of 4 warps for one candidate
     assert 4 * slot <= _noalloc_bytes() < G.sim_scratch_bytes(g, 4096)
-    _compare_calls(g, [_rows(5, 211, n, 3), _rows(6, 64, n, 3)])
+    _compare_calls(g, desc, [_rows(5, 211, n, 3), _rows(6, 64, n, 3)])
 
 
 def test_one_warp_blocks_when_four_slots_do_not_fit():
     """A graph whose warp slot is about 13 MB: fewer than four slots fit, so
     the call re-plans with one-warp blocks."""
     n = 800_000
-    g = G.gmg_create(_chain(n, 2, 7))
+    desc = _chain(n, 2, 7)
+    g = G.gmg_create(desc)
     slot = G.sim_scratch_bytes(g, 1) // 4
     assert slot <= _noalloc_bytes() < 4 * slot
-    _compare_calls(g, [_rows(7, 6, n, 2), _rows(8, 3, n, 2)])
+    _compare_calls(g, desc, [_rows(7, 6, n, 2), _rows(8, 3, n, 2)])
 
 
 def _noalloc_bytes():
