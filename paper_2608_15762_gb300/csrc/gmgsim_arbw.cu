@@ -58,6 +58,7 @@ struct ArbWSim : ArbEvents<ArbWSim<kT32, kTypes>, Sim<false, kFull, true, kT32, 
   bool arb_due;
   tm_t t_arb;
   tm_t td_c;         // next DONE time, kept current
+  int td_src;        // the lowest accelerator whose transfer completes at td_c
   uint64_t ik_c;     // next INTENT key (time << ib | op), kept current
 
   __device__ ArbWSim(const ArbWParams& a) : Base(a.P), A(a) {}
@@ -87,23 +88,48 @@ struct ArbWSim : ArbEvents<ArbWSim<kT32, kTypes>, Sim<false, kFull, true, kT32, 
   }
   static __device__ __forceinline__ bool bit(const uint32_t* s, int i) { return (s[i >> 5] >> (i & 31)) & 1u; }
 
+  // The tables hold at most 256 accelerators, eight per lane: each lane loads
+  // its eight entries together, then reduces.
+  static constexpr int kPerLane = 8;
+
+  // The next completion and the lowest accelerator completing then.
   __device__ void refresh_done() {
-    tm_t m = kNever;
-    for (int a = lane_id(); a < g.D; a += 32) {
-      const tm_t v = xd()[a];
-      m = v < m ? v : m;
+    const int lane = (int)lane_id();
+    tm_t v[kPerLane];
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int a = lane + 32 * u;
+      v[u] = a < g.D ? xd()[a] : kNever;
     }
+    tm_t m = kNever;
+    int am = 0x7fffffff;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u)
+      if (v[u] < m) {
+        m = v[u];
+        am = lane + 32 * u;
+      }
     td_c = warp_min_t(m);
+    td_src = (int)__reduce_min_sync(kFullMask, (unsigned)(m == td_c ? am : 0x7fffffff));
   }
   __device__ void refresh_intent() {
+    const int lane = (int)lane_id();
+    int32_t h[kPerLane];
+    tm_t f[kPerLane];
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u) {
+      const int a = lane + 32 * u;
+      const bool in = a < g.D;
+      h[u] = in ? fh()[a] : -1;
+      f[u] = in ? fa()[a] : kNever;
+    }
     uint64_t k = kKeyMax;
-    for (int a = lane_id(); a < g.D; a += 32) {
-      const int32_t h = fh()[a];
-      if (h >= 0) {
-        const uint64_t v = ((uint64_t)(U)fa()[a] << g.ib) | (uint32_t)h;
+#pragma unroll
+    for (int u = 0; u < kPerLane; ++u)
+      if (h[u] >= 0) {
+        const uint64_t v = ((uint64_t)(U)f[u] << g.ib) | (uint32_t)h[u];
         k = v < k ? v : k;
       }
-    }
     ik_c = warp_min_u64(k);
   }
 
@@ -148,6 +174,7 @@ struct ArbWSim : ArbEvents<ArbWSim<kT32, kTypes>, Sim<false, kFull, true, kT32, 
     arb_due = false;
     t_arb = 0;
     td_c = kNever;
+    td_src = 0;
     ik_c = kKeyMax;
     __syncwarp();
   }
@@ -413,11 +440,7 @@ struct ArbWSim : ArbEvents<ArbWSim<kT32, kTypes>, Sim<false, kFull, true, kT32, 
           break;
         }
         if (td == tx) {
-          // the lowest accelerator whose transfer completes now
-          int src = 0x7fffffff;
-          for (int a = lane_id(); a < g.D; a += 32)
-            if (xd()[a] == td && a < src) src = a;
-          transfer_done((int)__reduce_min_sync(kFullMask, (unsigned)src), td);
+          transfer_done(td_src, td);
         } else {
           intents_arrive((uint32_t)(ik & this->kc.mask));
         }
