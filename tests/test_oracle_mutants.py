@@ -36,6 +36,8 @@ MUTANTS = {
                                  "mem[c.e].push_back({c.arrive, 1, i, b});")],
     "src_alloc_at_ready": [("mem[d].push_back({s[i], 1, i, b});", "mem[d].push_back({r[i], 1, i, b});")],
     "t0_shifted": [("t = std::min(t, base.finish[p]);", "t = std::min(t, base.finish[p] + 1);")],
+    "events_after_t0_only": [("ev += base.ready[i] >= t0 ? 1 : 0;", "ev += base.ready[i] > t0 ? 1 : 0;")],
+    "arb_resumed_counts_every_op": [("if (g.mode == 1 && !resumed) {", "if (g.mode == 1) {")],
     "peak_without_base": [("int64_t live = g.base[d], peak = g.base[d];", "int64_t live = g.base[d], peak = 0;")],
     "argmin_not_strict": [("better = best < 0 || s[k].score < bscore;", "better = best < 0 || s[k].score <= bscore;")],
     "arb_no_link_check": [("if (sending[src] || receiving[t.e] || links_busy.count(lk)) {",
